@@ -1,0 +1,164 @@
+/*
+ * evo.h -- C ABI of the GB300 schedule-driven cached denoiser (EVO hot path).
+ *
+ * The library runs the reverse diffusion loop of a transformer diffusion
+ * policy on one GPU.  For every cacheable unit b (self-attention,
+ * cross-attention and FFN residual branch of each decoder layer; B = 3L units,
+ * Sec. 3.1) and every loop step t in {0..T-1}, a binary lattice S decides
+ * whether the unit is recomputed -- its residual output r_{b,t} is written to
+ * the unit's activation cache c_b -- or replaced by the cached c_b (Eq. 1).
+ * Caches are reset at the start of every action query (Sec. 3.1, Sec. 3.4).
+ * The sampler, weights and action interface are those of the policy and do
+ * not change with S (Sec. 3.4).
+ *
+ * Conventions for every entry point:
+ *  - Return value: an evo_status.  Argument and shape errors are detected on
+ *    the host before anything is launched and nothing is written.
+ *  - Device pointers are plain CUDA device addresses (for example from
+ *    torch tensors); "stream" is a cudaStream_t passed as void* (NULL = the
+ *    legacy default stream).  Work is asynchronous on that stream.
+ *  - All floating-point buffers are float32, C-contiguous, in the layouts
+ *    given below.  The caller owns every buffer it passes; the handle owns
+ *    the packed weights, the activation caches and its workspace.
+ *  - Errors found on the device (a schedule read from device memory with an
+ *    entry outside {0,1}, or a wait that timed out) are recorded in the
+ *    handle's status word; evo_get_status() reads and clears it.  With
+ *    cfg.debug_sync = 1 every call synchronizes and returns that status.
+ *  - A handle may be used from one stream at a time.
+ */
+#ifndef EVO_H
+#define EVO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct evo_handle evo_handle;
+
+typedef enum {
+  EVO_OK = 0,
+  EVO_ERR_ARG = 1,          /* null pointer, bad enum value, non-positive size */
+  EVO_ERR_SHAPE = 2,        /* shape not supported or batch above max_batch */
+  EVO_ERR_SCHEDULE = 3,     /* lattice entry outside {0,1}, wrong row count, duplicate position */
+  EVO_ERR_CUDA = 4,         /* a CUDA runtime call failed */
+  EVO_ERR_TIMEOUT = 5,      /* a device-side wait exceeded its iteration limit */
+  EVO_ERR_OOM = 6,          /* device allocation failed */
+  EVO_ERR_UNSUPPORTED = 7   /* no GPU with cluster launch, or the shape does not fit on chip */
+} evo_status;
+
+enum { EVO_SAMPLER_DDPM = 0, EVO_SAMPLER_DDIM = 1 };
+enum { EVO_DTYPE_F32 = 0, EVO_DTYPE_BF16 = 1 };
+/* Empty-cache policy for a unit that has not been refreshed yet in the
+ * current query: ZERO adds nothing (the reset cache is a zero tensor);
+ * FORCE computes the unit at that first use even if S skips it. */
+enum { EVO_EMPTY_ZERO = 0, EVO_EMPTY_FORCE = 1 };
+
+typedef struct evo_config {
+  int32_t n_layer;      /* L decoder layers; B = 3L cacheable units */
+  int32_t n_emb;        /* E */
+  int32_t n_head;       /* attention heads, E % n_head == 0 */
+  int32_t horizon;      /* H action tokens per sample (<= 32) */
+  int32_t action_dim;   /* A */
+  int32_t n_obs;        /* observation tokens; memory = 1 timestep token + n_obs */
+  int32_t obs_dim;      /* D */
+  int32_t n_steps;      /* T loop steps (lattice columns) */
+  int32_t train_steps;  /* diffusion training steps of the noise schedule (n_steps divides it) */
+  int32_t sampler;      /* EVO_SAMPLER_* */
+  int32_t dtype;        /* EVO_DTYPE_*: arithmetic/storage type of weights, GEMM operands and caches */
+  int32_t empty_cache;  /* EVO_EMPTY_* */
+  int32_t cluster;      /* CTAs that cooperate on one job; 0 = choose */
+  int32_t job_samples;  /* samples per job (rows = job_samples * horizon); 0 = choose */
+  int32_t debug_sync;   /* 1: synchronize after each call and return the device status */
+} evo_config;
+
+/* Number of float32 values in the weight blob for cfg (0 if cfg is invalid).
+ * Blob order (matrices are [in][out], y = x W):
+ *   obs_w[D][E] obs_b[E] cond_pos[1+n_obs][E] cm_w1[E][4E] cm_b1[4E] cm_w2[4E][E] cm_b2[E]
+ *   in_w[A][E] in_b[E] pos[H][E]
+ *   per layer l = 0..L-1:
+ *     ln1_g[E] ln1_b[E] sa_wqkv[E][3E] sa_bqkv[3E] sa_wo[E][E] sa_bo[E]
+ *     ln2_g[E] ln2_b[E] ca_wq[E][E] ca_bq[E] ca_wkv[E][2E] ca_bkv[2E] ca_wo[E][E] ca_bo[E]
+ *     ln3_g[E] ln3_b[E] ff_w1[E][4E] ff_b1[4E] ff_w2[4E][E] ff_b2[E]
+ *   lnf_g[E] lnf_b[E] head_w[E][A] head_b[A]
+ * (sa_wqkv columns are [q | k | v], ca_wkv columns are [k | v], each E wide.) */
+size_t evo_weight_count(const evo_config* cfg);
+
+/* Create a handle: copies the HOST weight blob (n_floats values, layout of
+ * evo_weight_count) to the device, packs it for the kernels, precomputes the
+ * timestep-token keys/values of every step, and sizes caches and workspace
+ * for up to max_batch samples per call (evo_denoise: N; population: (P+1)*N_obs).
+ * The current CUDA device at the time of the call is the handle's device. */
+evo_status evo_create(const float* weights, size_t n_floats, const evo_config* cfg,
+                      int32_t max_batch, evo_handle** out);
+
+evo_status evo_destroy(evo_handle* h);
+
+/* One action query per sample (Sec. 3.4 deployment, Eq. 1 inside the sampler loop).
+ *   obs    device [N][n_obs][obs_dim]   observation condition features
+ *   noise  device [n_noise][N][H][A]    slot 0 = initial x; DDPM: slot 1+t = z of loop step t
+ *                                       (n_noise = T+1); DDIM: n_noise = 1
+ *   S      [S_rows][T] uint8 lattice, host or device memory.  S_rows = 3L (unit rows
+ *          b = 3l + {0 SA, 1 CA, 2 FFN}) or L (row l covers the three units of layer l).
+ *          A host lattice is validated before launch; a device lattice is checked on the
+ *          device (EVO_ERR_SCHEDULE in the status word, outputs untouched).
+ *   out    device [N][H][A]             final actions (normalised space, after T steps)
+ */
+evo_status evo_denoise(evo_handle* h, const float* obs, const float* noise,
+                       const uint8_t* S, int32_t S_rows, int32_t N,
+                       float* out_actions, void* stream);
+
+/* Batched candidate evaluation in one launch: P schedules, each applied to the
+ * same N_obs observations and noise, plus the all-refresh schedule as a
+ * reference.  dev_l2[p] = mean_n || x_{p,n} - x_full,n ||_2 over the H*A action
+ * values (the candidates' cost for the search of Sec. 3.2).
+ *   obs    device [N_obs][n_obs][obs_dim]
+ *   noise  device [n_noise][N_obs][H][A]
+ *   S_pop  [P][S_rows][T] uint8, host or device
+ *   out_actions device [P][N_obs][H][A] or NULL
+ *   dev_l2 device [P]
+ */
+evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* noise,
+                                  const uint8_t* S_pop, int32_t P, int32_t S_rows, int32_t N_obs,
+                                  float* out_actions, float* dev_l2, void* stream);
+
+/* Exact per-sample FLOPs of one action query under S (host memory), in the
+ * convention 2 FLOPs per multiply-accumulate of every matmul (attention score
+ * and value products over the full H x H / H x (1+n_obs) matrices): T times the
+ * fixed per-step work (observation embedding, condition MLP, input and output
+ * projections) plus, for every refreshed lattice cell (Eq. 2's |S| cells), the
+ * FLOPs of that unit.  Under EVO_EMPTY_FORCE a row whose first entry is 0 adds
+ * one refresh. */
+evo_status evo_flops(const evo_handle* h, const uint8_t* S, int32_t S_rows, int64_t* flops_per_sample);
+evo_status evo_flops_cfg(const evo_config* cfg, const uint8_t* S, int32_t S_rows, int64_t* flops_per_sample);
+
+/* Individual encoding of Eq. 3 -> lattice.  bt: K pairs (b, t) in host memory;
+ * writes S_out[n_units][T] (host).  Rejects positions outside the lattice and
+ * duplicates (EVO_ERR_SCHEDULE); S_out is written only on success. */
+evo_status evo_schedule_from_positions(const int16_t* bt, int32_t K, int32_t n_units, int32_t T,
+                                       uint8_t* S_out);
+
+/* Debug variant of evo_denoise that also records the residual added at every
+ * lattice cell: trace device [T][3L][N][H][E] float32 (refreshed cells: r_{b,t};
+ * skipped cells: the cached c_b as stored; empty cache under ZERO: 0). */
+evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise,
+                             const uint8_t* S, int32_t S_rows, int32_t N,
+                             float* out_actions, float* trace, void* stream);
+
+/* Synchronizes the handle's last stream, returns and clears the device status word. */
+evo_status evo_get_status(evo_handle* h);
+
+/* Launch geometry chosen at create: CTAs per job cluster, samples per job,
+ * clusters resident at once, dynamic shared memory per CTA (bytes). */
+evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* job_samples,
+                               int32_t* max_clusters, int32_t* smem_bytes);
+
+const char* evo_status_string(evo_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EVO_H */

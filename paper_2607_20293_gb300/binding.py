@@ -1,0 +1,215 @@
+"""ctypes binding of the C ABI in include/evo.h (argument marshalling only).
+
+Every computation happens in libevo.so.  torch is used for device memory and
+streams: device arguments are torch CUDA tensors (their data pointers are
+passed through), host lattices are numpy uint8 arrays.  load() raises if the
+library has not been built; there is no other implementation to fall back to.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libevo.so")
+
+OK, ERR_ARG, ERR_SHAPE, ERR_SCHEDULE, ERR_CUDA, ERR_TIMEOUT, ERR_OOM, ERR_UNSUPPORTED = range(8)
+SAMPLERS = {"ddpm": 0, "ddim": 1}
+DTYPES = {"fp32": 0, "bf16": 1}
+EMPTY = {"zero": 0, "force": 1}
+
+_FIELDS = ["n_layer", "n_emb", "n_head", "horizon", "action_dim", "n_obs", "obs_dim", "n_steps",
+           "train_steps", "sampler", "dtype", "empty_cache", "cluster", "job_samples", "debug_sync"]
+
+
+class EvoConfig(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int32) for f in _FIELDS]
+
+
+class EvoError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        self.code = code
+        super().__init__(f"{what}: {status_string(code)} ({code})")
+
+
+_lib = None
+
+
+def load() -> ctypes.CDLL:
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2607_20293_gb300.build.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+    cfgp = ctypes.POINTER(EvoConfig)
+    sig = {
+        "evo_weight_count": (SZ, [cfgp]),
+        "evo_create": (I32, [P, SZ, cfgp, I32, ctypes.POINTER(P)]),
+        "evo_destroy": (I32, [P]),
+        "evo_denoise": (I32, [P, P, P, P, I32, I32, P, P]),
+        "evo_denoise_trace": (I32, [P, P, P, P, I32, I32, P, P, P]),
+        "evo_denoise_population": (I32, [P, P, P, P, I32, I32, I32, P, P, P]),
+        "evo_flops": (I32, [P, P, I32, ctypes.POINTER(I64)]),
+        "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
+        "evo_schedule_from_positions": (I32, [P, I32, I32, I32, P]),
+        "evo_get_status": (I32, [P]),
+        "evo_get_launch_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(I32),
+                                      ctypes.POINTER(I32)]),
+        "evo_status_string": (ctypes.c_char_p, [I32]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    return load().evo_status_string(code).decode()
+
+
+def _check(code: int, what: str):
+    if code != OK:
+        raise EvoError(code, what)
+
+
+def make_config(cfg: dict, cluster: int = 0, job_samples: int = 0, empty: str = "zero",
+                debug_sync: bool = False) -> EvoConfig:
+    return EvoConfig(cfg["n_layer"], cfg["n_emb"], cfg["n_head"], cfg["horizon"], cfg["action_dim"],
+                     cfg["n_obs"], cfg["obs_dim"], cfg["n_steps"], cfg["train_steps"],
+                     SAMPLERS[cfg["sampler"]], DTYPES[cfg["dtype"]], EMPTY[empty], cluster, job_samples,
+                     int(debug_sync))
+
+
+def weight_names(cfg: dict) -> list[str]:
+    names = ["obs_w", "obs_b", "cond_pos", "cm_w1", "cm_b1", "cm_w2", "cm_b2", "in_w", "in_b", "pos"]
+    per = ["ln1_g", "ln1_b", "sa_wqkv", "sa_bqkv", "sa_wo", "sa_bo", "ln2_g", "ln2_b", "ca_wq", "ca_bq",
+           "ca_wkv", "ca_bkv", "ca_wo", "ca_bo", "ln3_g", "ln3_b", "ff_w1", "ff_b1", "ff_w2", "ff_b2"]
+    for l in range(cfg["n_layer"]):
+        names += [f"l{l}.{n}" for n in per]
+    return names + ["lnf_g", "lnf_b", "head_w", "head_b"]
+
+
+def pack_blob(cfg: dict, weights: dict) -> np.ndarray:
+    """Concatenate named float32 tensors in the blob order of evo_weight_count."""
+    blob = np.concatenate([np.ascontiguousarray(weights[n], dtype=np.float32).ravel() for n in weight_names(cfg)])
+    want = load().evo_weight_count(ctypes.byref(make_config(cfg)))
+    if blob.size != want:
+        raise ValueError(f"weight blob has {blob.size} floats, the library expects {want}")
+    return blob
+
+
+def _ptr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, np.ndarray):
+        return x.ctypes.data
+    return x.data_ptr()
+
+
+def _lattice(S):
+    """numpy lattices are passed as host memory (C-contiguous uint8); torch uint8
+    tensors on the GPU as device memory."""
+    if isinstance(S, np.ndarray):
+        S = np.ascontiguousarray(S, dtype=np.uint8)
+    return S
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return stream if isinstance(stream, int) else stream.cuda_stream
+
+
+def flops_cfg(cfg: dict, S, empty: str = "zero") -> int:
+    S = np.ascontiguousarray(S, dtype=np.uint8)
+    out = ctypes.c_int64()
+    c = make_config(cfg, empty=empty)
+    _check(load().evo_flops_cfg(ctypes.byref(c), S.ctypes.data, S.shape[0], ctypes.byref(out)), "evo_flops")
+    return out.value
+
+
+def schedule_from_positions(positions, n_units: int, T: int) -> np.ndarray:
+    bt = np.ascontiguousarray(np.asarray(positions, dtype=np.int16).reshape(-1, 2))
+    out = np.zeros((n_units, T), dtype=np.uint8)
+    _check(load().evo_schedule_from_positions(bt.ctypes.data if bt.size else None, bt.shape[0], n_units, T,
+                                              out.ctypes.data), "evo_schedule_from_positions")
+    return out
+
+
+class Evo:
+    """One evo_handle: packed weights, caches and workspace on the current GPU."""
+
+    def __init__(self, cfg: dict, weights: dict, max_batch: int, cluster: int = 0, job_samples: int = 0,
+                 empty: str = "zero", debug_sync: bool = False):
+        lib = load()
+        self.cfg = dict(cfg)
+        self._c = make_config(cfg, cluster, job_samples, empty, debug_sync)
+        self._blob = pack_blob(cfg, weights)
+        h = ctypes.c_void_p()
+        _check(lib.evo_create(self._blob.ctypes.data, self._blob.size, ctypes.byref(self._c), max_batch,
+                              ctypes.byref(h)), "evo_create")
+        self._h = h
+        self.max_batch = max_batch
+
+    def close(self):
+        if getattr(self, "_h", None) and self._h.value:
+            load().evo_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def launch_info(self) -> dict:
+        v = [ctypes.c_int32() for _ in range(4)]
+        _check(load().evo_get_launch_info(self._h, *[ctypes.byref(x) for x in v]), "evo_get_launch_info")
+        return dict(cluster=v[0].value, job_samples=v[1].value, max_clusters=v[2].value, smem_bytes=v[3].value)
+
+    def denoise(self, obs, noise, S, out=None, stream=None, trace=None):
+        import torch
+        N = obs.shape[0]
+        if out is None:
+            out = torch.empty((N, self.cfg["horizon"], self.cfg["action_dim"]), dtype=torch.float32,
+                              device=obs.device)
+        S = _lattice(S)
+        if trace is None:
+            rc = load().evo_denoise(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
+                                    _stream(stream))
+        else:
+            rc = load().evo_denoise_trace(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
+                                          _ptr(trace), _stream(stream))
+        _check(rc, "evo_denoise")
+        return out
+
+    def population(self, obs, noise, S_pop, out=None, dev=None, stream=None, want_actions=True):
+        import torch
+        N_obs = obs.shape[0]
+        S_pop = _lattice(S_pop)
+        P = S_pop.shape[0]
+        if out is None and want_actions:
+            out = torch.empty((P, N_obs, self.cfg["horizon"], self.cfg["action_dim"]), dtype=torch.float32,
+                              device=obs.device)
+        if dev is None:
+            dev = torch.empty((P,), dtype=torch.float32, device=obs.device)
+        rc = load().evo_denoise_population(self._h, _ptr(obs), _ptr(noise), _ptr(S_pop), P, S_pop.shape[1], N_obs,
+                                           _ptr(out), _ptr(dev), _stream(stream))
+        _check(rc, "evo_denoise_population")
+        return out, dev
+
+    def flops(self, S) -> int:
+        S = np.ascontiguousarray(S, dtype=np.uint8)
+        out = ctypes.c_int64()
+        _check(load().evo_flops(self._h, S.ctypes.data, S.shape[0], ctypes.byref(out)), "evo_flops")
+        return out.value
+
+    def status(self) -> int:
+        return load().evo_get_status(self._h)

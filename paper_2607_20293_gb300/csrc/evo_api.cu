@@ -1,0 +1,724 @@
+// Host side of the C ABI declared in include/evo.h: configuration checks,
+// weight packing, launch geometry, schedule upload and the FLOP accountant.
+//
+// Packing.  For cluster rank c, every unit's weights are cut into the two
+// slices that CTA c multiplies by (first GEMM: columns; second GEMM: rows),
+// stored contiguously per CTA and per layer so that the kernel's producer warp
+// fetches each refreshed unit's slice with a few bulk copies:
+//   SA  : [q_h | k_h | v_c] columns of W_qkv (h = head of c, v_c = c's value
+//         columns), then rows c*E/C.. of W_o
+//   CA  : q_h columns of W_q, then rows c*E/C.. of W_o
+//   FFN : columns c*4E/C.. of W_1, then rows c*4E/C.. of W_2
+// bf16 slices are laid out in mma.sync B-fragment order (k-tiles of 16 rows,
+// n-tiles of 8 columns, 8 bytes per lane) so that a warp reads a fragment
+// with one conflict-free 8-byte load per lane; fp32 slices are row-major.
+
+#include "../../include/evo.h"
+#include "evo_internal.h"
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+using namespace evo;
+
+struct evo_handle {
+  evo_config cfg;
+  int device = 0;
+  int L = 0, E = 0, U = 0, T = 0, H = 0, A = 0;
+  JobParams base{};
+  int max_batch = 0;
+  int max_clusters = 0;
+  int smem_limit = 0;
+  int es = 4;
+  // device memory
+  float* wf32 = nullptr;
+  int* woff_d = nullptr;
+  uint8_t* wpack = nullptr;
+  float* vec = nullptr;
+  float* stab = nullptr;
+  float* kstep = nullptr;
+  float* kv_time = nullptr;
+  float* kv_obs = nullptr;
+  void* cache = nullptr;
+  uint8_t* sched = nullptr;
+  size_t sched_cap = 0;
+  int* status = nullptr;      // [0] = kernel status bits, [1] = schedule check of the last device lattice
+  float* pop_x = nullptr;
+  // host staging for host-memory schedules
+  uint8_t* stage = nullptr;
+  cudaEvent_t stage_ev = nullptr;
+  std::vector<uint8_t> last_sched;
+  int last_rows = -1;
+  bool last_valid = false;
+  cudaStream_t last_stream = nullptr;
+  int woff[W_COUNT];
+};
+
+namespace {
+
+inline evo_status cuda_st(cudaError_t e) { return e == cudaSuccess ? EVO_OK : EVO_ERR_CUDA; }
+
+#define EVO_CUDA(x)                                   \
+  do {                                                \
+    cudaError_t _e = (x);                             \
+    if (_e != cudaSuccess) return EVO_ERR_CUDA;       \
+  } while (0)
+
+bool config_ok(const evo_config* c) {
+  if (!c) return false;
+  if (c->n_layer <= 0 || c->n_layer > 21) return false;          // 3L units tracked in a 64-bit mask
+  if (c->n_emb <= 0 || c->n_head <= 0 || c->n_emb % c->n_head) return false;
+  if (c->n_emb % 32 || c->n_emb > 512) return false;             // LayerNorm: <= 16 values per lane
+  if (c->horizon <= 0 || c->horizon > 32 || c->horizon % 4) return false;
+  if (c->action_dim <= 0 || c->action_dim > 32) return false;
+  if (c->n_obs <= 0 || c->n_obs > 31 || c->obs_dim <= 0) return false;
+  if (c->n_steps <= 0 || c->train_steps <= 0 || c->train_steps % c->n_steps) return false;
+  if (c->sampler != EVO_SAMPLER_DDPM && c->sampler != EVO_SAMPLER_DDIM) return false;
+  if (c->dtype != EVO_DTYPE_F32 && c->dtype != EVO_DTYPE_BF16) return false;
+  if (c->empty_cache != EVO_EMPTY_ZERO && c->empty_cache != EVO_EMPTY_FORCE) return false;
+  if (c->cluster < 0 || c->cluster > MAX_CLUSTER || c->job_samples < 0) return false;
+  const int dh = c->n_emb / c->n_head;
+  if (dh % 4 || dh > 128) return false;
+  return true;
+}
+
+void weight_offsets(const evo_config* c, int* wo) {
+  const int E = c->n_emb, A = c->action_dim, D = c->obs_dim, H = c->horizon, Cm = 1 + c->n_obs;
+  int o = 0;
+  auto take = [&](int id, int n) { wo[id] = o; o += n; };
+  take(W_OBS_W, D * E);
+  take(W_OBS_B, E);
+  take(W_COND_POS, Cm * E);
+  take(W_CM_W1, E * 4 * E);
+  take(W_CM_B1, 4 * E);
+  take(W_CM_W2, 4 * E * E);
+  take(W_CM_B2, E);
+  take(W_IN_W, A * E);
+  take(W_IN_B, E);
+  take(W_POS, H * E);
+  wo[W_LAYER0] = o;
+  int lo = 0;
+  auto ltake = [&](int id, int n) { wo[id] = lo; lo += n; };
+  ltake(WL_LN1G, E);
+  ltake(WL_LN1B, E);
+  ltake(WL_SA_WQKV, E * 3 * E);
+  ltake(WL_SA_BQKV, 3 * E);
+  ltake(WL_SA_WO, E * E);
+  ltake(WL_SA_BO, E);
+  ltake(WL_LN2G, E);
+  ltake(WL_LN2B, E);
+  ltake(WL_CA_WQ, E * E);
+  ltake(WL_CA_BQ, E);
+  ltake(WL_CA_WKV, E * 2 * E);
+  ltake(WL_CA_BKV, 2 * E);
+  ltake(WL_CA_WO, E * E);
+  ltake(WL_CA_BO, E);
+  ltake(WL_LN3G, E);
+  ltake(WL_LN3B, E);
+  ltake(WL_FF_W1, E * 4 * E);
+  ltake(WL_FF_B1, 4 * E);
+  ltake(WL_FF_W2, 4 * E * E);
+  ltake(WL_FF_B2, E);
+  wo[W_LAYER_STRIDE] = lo;
+  o += c->n_layer * lo;
+  take(W_LNF_G, E);
+  take(W_LNF_B, E);
+  take(W_HEAD_W, E * A);
+  take(W_HEAD_B, A);
+  wo[W_TOTAL] = o;
+}
+
+inline uint16_t f2bf(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7f800000u) == 0x7f800000u) return (uint16_t)(u >> 16);   // inf / nan kept
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+inline int rup(int x, int a) { return (x + a - 1) / a * a; }
+
+// decomposition constraints for a cluster of C CTAs
+bool cluster_ok(const evo_config* c, int C) {
+  const int E = c->n_emb, dh = E / c->n_head;
+  if (C < 1 || E % C) return false;
+  const int Ec = E / C, hid = 4 * E / C;
+  if (Ec % 4 || Ec > dh || dh % Ec || Ec > 64) return false;
+  if (c->dtype == EVO_DTYPE_BF16 && (Ec % 8 || hid % 16)) return false;
+  return true;
+}
+
+// sampler coefficients per loop step: inv_sqrt_ab, sqrt_1mab, c_x0, c_xt, sigma, sqrt_ab, sqrt_ab_prev, sqrt_1mab_prev
+void sampler_table(const evo_config* c, std::vector<float>& tab, std::vector<float>& kstep) {
+  const int Ttr = c->train_steps, T = c->n_steps, stride = Ttr / T;
+  std::vector<double> ac(Ttr);
+  double prod = 1.0;
+  const double pi = 3.14159265358979323846;
+  auto f = [&](double s) {
+    const double v = std::cos((s + 0.008) / 1.008 * pi / 2);
+    return v * v;
+  };
+  for (int i = 0; i < Ttr; ++i) {
+    const double beta = std::min(1.0 - f((i + 1) / (double)Ttr) / f(i / (double)Ttr), 0.999);
+    prod *= (1.0 - beta);
+    ac[i] = prod;
+  }
+  tab.assign((size_t)T * 8, 0.f);
+  kstep.assign(T, 0.f);
+  for (int t = 0; t < T; ++t) {
+    const int k = (T - 1 - t) * stride;
+    const int prev = k - stride;
+    const double ab = ac[k], abp = prev >= 0 ? ac[prev] : 1.0;
+    const double alpha = ab / abp, beta = 1.0 - alpha;
+    float* r = &tab[(size_t)t * 8];
+    r[0] = (float)(1.0 / std::sqrt(ab));
+    r[1] = (float)std::sqrt(1.0 - ab);
+    r[2] = (float)(std::sqrt(abp) * beta / (1.0 - ab));
+    r[3] = (float)(std::sqrt(alpha) * (1.0 - abp) / (1.0 - ab));
+    const double var = std::max((1.0 - abp) / (1.0 - ab) * beta, 1e-20);
+    r[4] = k > 0 ? (float)std::sqrt(var) : 0.f;
+    r[5] = (float)std::sqrt(ab);
+    r[6] = (float)std::sqrt(abp);
+    r[7] = (float)std::sqrt(1.0 - abp);
+    kstep[t] = (float)k;
+  }
+}
+
+int64_t flops_of(const evo_config* c, const uint8_t* S, int rows) {
+  const int64_t E = c->n_emb, H = c->horizon, Cm = 1 + c->n_obs, A = c->action_dim, D = c->obs_dim;
+  const int64_t fsa = 2 * H * E * 3 * E + 4 * H * H * E + 2 * H * E * E;
+  const int64_t fca = 2 * H * E * E + 4 * Cm * E * E + 4 * H * Cm * E + 2 * H * E * E;
+  const int64_t fff = 16 * H * E * E;
+  const int64_t fix = 2 * c->n_obs * D * E + 16 * Cm * E * E + 4 * H * A * E;
+  const int T = c->n_steps, U = 3 * c->n_layer;
+  int64_t total = (int64_t)T * fix;
+  for (int b = 0; b < U; ++b) {
+    const int row = rows == U ? b : b / 3;
+    int64_t n = 0;
+    for (int t = 0; t < T; ++t) n += S[(size_t)row * T + t];
+    if (c->empty_cache == EVO_EMPTY_FORCE && T > 0 && S[(size_t)row * T] == 0) n += 1;
+    const int u = b % 3;
+    total += n * (u == 0 ? fsa : (u == 1 ? fca : fff));
+  }
+  return total;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+bool lattice_ok(const uint8_t* S, size_t n) {
+  for (size_t i = 0; i < n; ++i)
+    if (S[i] > 1) return false;
+  return true;
+}
+
+// Fill p's decomposition fields for g samples per job; returns shared bytes or -1.
+int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
+  const int E = c->n_emb, dh = E / c->n_head, H = c->horizon;
+  const int es = c->dtype == EVO_DTYPE_BF16 ? 2 : 4;
+  p.L = c->n_layer;
+  p.E = E;
+  p.nh = c->n_head;
+  p.dh = dh;
+  p.H = H;
+  p.A = c->action_dim;
+  p.n_obs = c->n_obs;
+  p.T = c->n_steps;
+  p.U = 3 * c->n_layer;
+  p.Cm = 1 + c->n_obs;
+  p.C = C;
+  p.Ec = E / C;
+  p.hid = 4 * E / C;
+  p.g = g;
+  p.M = g * H;
+  p.Mp = rup(p.M, 16);
+  p.ldf = E + 4;
+  p.n1_sa = 2 * dh + p.Ec;
+  p.n1_ca = dh;
+  p.n1_ff = p.hid;
+  p.n1max = std::max(p.n1_sa, p.n1_ff);
+  p.ldg1 = p.n1_sa + 1;
+  p.kp_o = rup(p.Ec, 16);
+  p.kp_h = rup(p.hid, 16);
+  p.ldh = es == 2 ? p.kp_h + 8 : p.kp_h;
+  p.ldo = es == 2 ? p.kp_o + 8 : p.kp_o;
+  p.sampler = c->sampler;
+  p.force = c->empty_cache == EVO_EMPTY_FORCE;
+  if (es == 2) {
+    if (p.Mp > 32) return -1;
+  } else {
+    const int nmax = std::max(p.n1max, E);
+    if (p.M * nmax > 16 * NCT) return -1;
+  }
+  // largest k-tile of any piece
+  const int max_ktile = 16 * std::max(p.n1max, E) * es;
+  const int slots[] = {32768, 16384};
+  for (int head_sep = 1; head_sep >= 0; --head_sep) {
+    for (int sb : slots) {
+      if (sb < max_ktile) continue;
+      for (int ns = 4; ns >= 2; --ns) {
+        p.head_sep = head_sep;
+        p.slot_bytes = sb;
+        p.nslot = ns;
+        const int total = smem_layout(p, es);
+        if (total <= smem_limit) return total;
+      }
+    }
+  }
+  return -1;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* evo_status_string(evo_status s) {
+  switch (s) {
+    case EVO_OK: return "ok";
+    case EVO_ERR_ARG: return "invalid argument";
+    case EVO_ERR_SHAPE: return "unsupported shape or batch";
+    case EVO_ERR_SCHEDULE: return "invalid schedule lattice";
+    case EVO_ERR_CUDA: return "CUDA runtime error";
+    case EVO_ERR_TIMEOUT: return "device wait timed out";
+    case EVO_ERR_OOM: return "device out of memory";
+    case EVO_ERR_UNSUPPORTED: return "unsupported on this device";
+  }
+  return "unknown status";
+}
+
+size_t evo_weight_count(const evo_config* cfg) {
+  if (!config_ok(cfg)) return 0;
+  int wo[W_COUNT];
+  weight_offsets(cfg, wo);
+  return (size_t)wo[W_TOTAL];
+}
+
+evo_status evo_flops_cfg(const evo_config* cfg, const uint8_t* S, int32_t S_rows, int64_t* out) {
+  if (!config_ok(cfg) || !S || !out) return EVO_ERR_ARG;
+  const int U = 3 * cfg->n_layer;
+  if (S_rows != U && S_rows != cfg->n_layer) return EVO_ERR_SCHEDULE;
+  if (!lattice_ok(S, (size_t)S_rows * cfg->n_steps)) return EVO_ERR_SCHEDULE;
+  *out = flops_of(cfg, S, S_rows);
+  return EVO_OK;
+}
+
+evo_status evo_flops(const evo_handle* h, const uint8_t* S, int32_t S_rows, int64_t* out) {
+  if (!h) return EVO_ERR_ARG;
+  return evo_flops_cfg(&h->cfg, S, S_rows, out);
+}
+
+evo_status evo_schedule_from_positions(const int16_t* bt, int32_t K, int32_t n_units, int32_t T, uint8_t* S_out) {
+  if ((!bt && K > 0) || !S_out || K < 0 || n_units <= 0 || T <= 0) return EVO_ERR_ARG;
+  std::vector<uint8_t> s((size_t)n_units * T, 0);
+  for (int i = 0; i < K; ++i) {
+    const int b = bt[2 * i], t = bt[2 * i + 1];
+    if (b < 0 || b >= n_units || t < 0 || t >= T) return EVO_ERR_SCHEDULE;
+    uint8_t& cell = s[(size_t)b * T + t];
+    if (cell) return EVO_ERR_SCHEDULE;
+    cell = 1;
+  }
+  std::memcpy(S_out, s.data(), s.size());
+  return EVO_OK;
+}
+
+evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* job_samples, int32_t* max_clusters,
+                               int32_t* smem_bytes) {
+  if (!h) return EVO_ERR_ARG;
+  if (cluster) *cluster = h->base.C;
+  if (job_samples) *job_samples = h->base.g;
+  if (max_clusters) *max_clusters = h->max_clusters;
+  if (smem_bytes) *smem_bytes = h->base.sm.total;
+  return EVO_OK;
+}
+
+evo_status evo_destroy(evo_handle* h) {
+  if (!h) return EVO_ERR_ARG;
+  cudaFree(h->wf32);
+  cudaFree(h->woff_d);
+  cudaFree(h->wpack);
+  cudaFree(h->vec);
+  cudaFree(h->stab);
+  cudaFree(h->kstep);
+  cudaFree(h->kv_time);
+  cudaFree(h->kv_obs);
+  cudaFree(h->cache);
+  cudaFree(h->sched);
+  cudaFree(h->status);
+  cudaFree(h->pop_x);
+  if (h->stage) cudaFreeHost(h->stage);
+  if (h->stage_ev) cudaEventDestroy(h->stage_ev);
+  delete h;
+  return EVO_OK;
+}
+
+evo_status evo_create(const float* weights, size_t n_floats, const evo_config* cfg, int32_t max_batch,
+                      evo_handle** out) {
+  if (!weights || !cfg || !out || max_batch <= 0) return EVO_ERR_ARG;
+  *out = nullptr;
+  if (!config_ok(cfg)) return EVO_ERR_SHAPE;
+  if (n_floats != evo_weight_count(cfg)) return EVO_ERR_SHAPE;
+  int dev = 0;
+  EVO_CUDA(cudaGetDevice(&dev));
+  int cc_major = 0, smem_optin = 0, cluster_ok_attr = 0;
+  EVO_CUDA(cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, dev));
+  EVO_CUDA(cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev));
+  EVO_CUDA(cudaDeviceGetAttribute(&cluster_ok_attr, cudaDevAttrClusterLaunch, dev));
+  if (cc_major < 10 || !cluster_ok_attr) return EVO_ERR_UNSUPPORTED;
+
+  evo_handle* h = new evo_handle();
+  h->cfg = *cfg;
+  h->device = dev;
+  h->L = cfg->n_layer;
+  h->E = cfg->n_emb;
+  h->U = 3 * cfg->n_layer;
+  h->T = cfg->n_steps;
+  h->H = cfg->horizon;
+  h->A = cfg->action_dim;
+  h->es = cfg->dtype == EVO_DTYPE_BF16 ? 2 : 4;
+  h->max_batch = max_batch;
+  h->smem_limit = smem_optin;
+  weight_offsets(cfg, h->woff);
+  const int E = h->E, L = h->L, U = h->U, T = h->T, H = h->H, A = h->A;
+  const int dh = E / cfg->n_head;
+
+  // ---- decomposition ------------------------------------------------------
+  int C = cfg->cluster;
+  if (C == 0) {
+    const int cap = std::min(MAX_CLUSTER, std::max(1, E / 16));
+    for (C = cap; C >= 1; C >>= 1)
+      if (cluster_ok(cfg, C)) break;
+  }
+  if (C < 1 || !cluster_ok(cfg, C)) {
+    delete h;
+    return EVO_ERR_SHAPE;
+  }
+  int g = cfg->job_samples > 0 ? cfg->job_samples : 1;
+  JobParams& p = h->base;
+  const int smem = plan(cfg, C, g, smem_optin, p);
+  if (smem < 0) {
+    delete h;
+    return EVO_ERR_UNSUPPORTED;
+  }
+  {
+    int mc = 0;
+    cudaError_t e = job_kernel_prepare(cfg->dtype, smem, C, &mc);
+    if (e != cudaSuccess || mc <= 0) {
+      cudaGetLastError();
+      delete h;
+      return EVO_ERR_UNSUPPORTED;
+    }
+    h->max_clusters = mc;
+  }
+
+  // ---- weights -------------------------------------------------------------
+  auto fail = [&](evo_status s) {
+    evo_destroy(h);
+    return s;
+  };
+  const size_t wbytes = n_floats * sizeof(float);
+  if (cudaMalloc(&h->wf32, wbytes) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMemcpy(h->wf32, weights, wbytes, cudaMemcpyHostToDevice) != cudaSuccess) return fail(EVO_ERR_CUDA);
+  if (cudaMalloc(&h->woff_d, sizeof(h->woff)) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMemcpy(h->woff_d, h->woff, sizeof(h->woff), cudaMemcpyHostToDevice) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+
+  const int* wo = h->woff;
+  auto W = [&](int id) { return weights + wo[id]; };
+  auto WL = [&](int l, int id) { return weights + wo[W_LAYER0] + (size_t)l * wo[W_LAYER_STRIDE] + wo[id]; };
+  const int es = h->es;
+  const int Ec = p.Ec, hid = p.hid;
+  // piece sizes (bytes) and offsets within one layer block
+  const long long sz[3][2] = {{(long long)E * p.n1_sa * es, (long long)p.kp_o * E * es},
+                              {(long long)E * p.n1_ca * es, (long long)p.kp_o * E * es},
+                              {(long long)E * p.n1_ff * es, (long long)p.kp_h * E * es}};
+  long long off = 0;
+  for (int u = 0; u < 3; ++u)
+    for (int q = 0; q < 2; ++q) {
+      p.poff[u][q] = off;
+      off += sz[u][q];
+    }
+  p.layer_stride = off;
+  p.cta_stride = off * L;
+  std::vector<uint8_t> pack((size_t)p.cta_stride * C, 0);
+  auto put = [&](uint8_t* dst, int K, int N, auto get) {
+    if (es == 2) {
+      uint16_t* d = reinterpret_cast<uint16_t*>(dst);
+      const int NT = N / 8;
+      for (int kt = 0; kt < K / 16; ++kt)
+        for (int nt = 0; nt < NT; ++nt)
+          for (int lane = 0; lane < 32; ++lane)
+            for (int i = 0; i < 4; ++i) {
+              const int k = kt * 16 + (lane % 4) * 2 + (i % 2) + (i / 2) * 8;
+              const int n = nt * 8 + lane / 4;
+              d[(((size_t)kt * NT + nt) * 32 + lane) * 4 + i] = f2bf(get(k, n));
+            }
+    } else {
+      float* d = reinterpret_cast<float*>(dst);
+      for (int k = 0; k < K; ++k)
+        for (int n = 0; n < N; ++n) d[(size_t)k * N + n] = get(k, n);
+    }
+  };
+  for (int c = 0; c < C; ++c) {
+    const int h0 = (c * Ec) / dh;
+    for (int l = 0; l < L; ++l) {
+      uint8_t* base = pack.data() + (size_t)c * p.cta_stride + (size_t)l * p.layer_stride;
+      const float* wqkv = WL(l, WL_SA_WQKV);
+      const float* wo1 = WL(l, WL_SA_WO);
+      const float* wq = WL(l, WL_CA_WQ);
+      const float* wo2 = WL(l, WL_CA_WO);
+      const float* w1 = WL(l, WL_FF_W1);
+      const float* w2 = WL(l, WL_FF_W2);
+      put(base + p.poff[0][0], E, p.n1_sa, [&](int k, int n) {
+        const int col = n < dh ? h0 * dh + n : (n < 2 * dh ? E + h0 * dh + (n - dh) : 2 * E + c * Ec + (n - 2 * dh));
+        return wqkv[(size_t)k * 3 * E + col];
+      });
+      put(base + p.poff[0][1], p.kp_o, E,
+          [&](int k, int n) { return k < Ec ? wo1[(size_t)(c * Ec + k) * E + n] : 0.f; });
+      put(base + p.poff[1][0], E, p.n1_ca, [&](int k, int n) { return wq[(size_t)k * E + h0 * dh + n]; });
+      put(base + p.poff[1][1], p.kp_o, E,
+          [&](int k, int n) { return k < Ec ? wo2[(size_t)(c * Ec + k) * E + n] : 0.f; });
+      put(base + p.poff[2][0], E, p.n1_ff, [&](int k, int n) { return w1[(size_t)k * 4 * E + c * hid + n]; });
+      put(base + p.poff[2][1], p.kp_h, E,
+          [&](int k, int n) { return k < hid ? w2[(size_t)(c * hid + k) * E + n] : 0.f; });
+    }
+  }
+  if (cudaMalloc(&h->wpack, pack.size()) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMemcpy(h->wpack, pack.data(), pack.size(), cudaMemcpyHostToDevice) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+
+  // float32 vectors
+  std::vector<float> vec;
+  auto vtake = [&](long long& dst, size_t n) {
+    dst = (long long)vec.size();
+    vec.resize(vec.size() + n, 0.f);
+  };
+  vtake(p.v_ln, (size_t)U * 2 * E);
+  vtake(p.v_b1, (size_t)U * C * p.n1max);
+  vtake(p.v_b2, (size_t)U * E);
+  vtake(p.v_inw, (size_t)A * E);
+  vtake(p.v_inb, E);
+  vtake(p.v_pos, (size_t)H * E);
+  vtake(p.v_lnfg, E);
+  vtake(p.v_lnfb, E);
+  vtake(p.v_headw, (size_t)E * A);
+  vtake(p.v_headb, A);
+  for (int b = 0; b < U; ++b) {
+    const int l = b / 3, u = b % 3;
+    const int gid = u == 0 ? WL_LN1G : (u == 1 ? WL_LN2G : WL_LN3G);
+    const int bid = u == 0 ? WL_LN1B : (u == 1 ? WL_LN2B : WL_LN3B);
+    std::memcpy(&vec[p.v_ln + (size_t)b * 2 * E], WL(l, gid), E * 4);
+    std::memcpy(&vec[p.v_ln + (size_t)b * 2 * E + E], WL(l, bid), E * 4);
+    const float* b2 = u == 0 ? WL(l, WL_SA_BO) : (u == 1 ? WL(l, WL_CA_BO) : WL(l, WL_FF_B2));
+    std::memcpy(&vec[p.v_b2 + (size_t)b * E], b2, E * 4);
+    for (int c = 0; c < C; ++c) {
+      float* d = &vec[p.v_b1 + ((size_t)b * C + c) * p.n1max];
+      const int h0 = (c * Ec) / dh;
+      if (u == 0) {
+        const float* bq = WL(l, WL_SA_BQKV);
+        for (int n = 0; n < p.n1_sa; ++n)
+          d[n] = bq[n < dh ? h0 * dh + n : (n < 2 * dh ? E + h0 * dh + (n - dh) : 2 * E + c * Ec + (n - 2 * dh))];
+      } else if (u == 1) {
+        const float* bq = WL(l, WL_CA_BQ);
+        for (int n = 0; n < dh; ++n) d[n] = bq[h0 * dh + n];
+      } else {
+        const float* b1 = WL(l, WL_FF_B1);
+        for (int n = 0; n < hid; ++n) d[n] = b1[c * hid + n];
+      }
+    }
+  }
+  std::memcpy(&vec[p.v_inw], W(W_IN_W), (size_t)A * E * 4);
+  std::memcpy(&vec[p.v_inb], W(W_IN_B), E * 4);
+  std::memcpy(&vec[p.v_pos], W(W_POS), (size_t)H * E * 4);
+  std::memcpy(&vec[p.v_lnfg], W(W_LNF_G), E * 4);
+  std::memcpy(&vec[p.v_lnfb], W(W_LNF_B), E * 4);
+  std::memcpy(&vec[p.v_headw], W(W_HEAD_W), (size_t)E * A * 4);
+  std::memcpy(&vec[p.v_headb], W(W_HEAD_B), A * 4);
+  if (cudaMalloc(&h->vec, vec.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMemcpy(h->vec, vec.data(), vec.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+
+  // sampler table, timestep-token keys/values
+  std::vector<float> tab, kst;
+  sampler_table(cfg, tab, kst);
+  if (cudaMalloc(&h->stab, tab.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&h->kstep, kst.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  cudaMemcpy(h->stab, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice);
+  cudaMemcpy(h->kstep, kst.data(), kst.size() * 4, cudaMemcpyHostToDevice);
+  if (cudaMalloc(&h->kv_time, (size_t)T * L * 2 * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (launch_time_table(h->wf32, h->woff_d, h->kstep, T, L, E, h->kv_time, 0) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+
+  // per-call buffers
+  const size_t cap_samples = (size_t)max_batch + 32;
+  if (cudaMalloc(&h->kv_obs, cap_samples * cfg->n_obs * L * 2 * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&h->cache, cap_samples * H * (size_t)U * E * es) != cudaSuccess) return fail(EVO_ERR_OOM);
+  h->sched_cap = cap_samples * U * T;
+  if (cudaMalloc(&h->sched, h->sched_cap) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&h->status, 2 * sizeof(int)) != cudaSuccess) return fail(EVO_ERR_OOM);
+  cudaMemset(h->status, 0, 2 * sizeof(int));
+  if (cudaMalloc(&h->pop_x, cap_samples * H * A * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMallocHost(&h->stage, h->sched_cap) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaEventCreateWithFlags(&h->stage_ev, cudaEventDisableTiming) != cudaSuccess) return fail(EVO_ERR_CUDA);
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(EVO_ERR_CUDA);
+
+  p.stab = h->stab;
+  p.kv_time = h->kv_time;
+  p.kv_obs = h->kv_obs;
+  p.wpack = h->wpack;
+  p.vec = h->vec;
+  p.cache = h->cache;
+  p.status = h->status;
+  *out = h;
+  return EVO_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+// Copy n_sched lattices (+ optionally an all-ones reference lattice) into the
+// handle's device buffer.  Host lattices are validated here; device lattices
+// are checked by a kernel that sets status[1].
+evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int rows, bool add_ones, cudaStream_t st,
+                           const int** err_out) {
+  const size_t one = (size_t)rows * h->T;
+  const size_t bytes = one * n_sched;
+  const size_t total = bytes + (add_ones ? one : 0);
+  if (total > h->sched_cap) return EVO_ERR_SHAPE;
+  *err_out = nullptr;
+  if (!is_device_ptr(S)) {
+    if (!lattice_ok(S, bytes)) return EVO_ERR_SCHEDULE;
+    const bool same = h->last_valid && h->last_rows == rows && h->last_sched.size() == total &&
+                      std::memcmp(h->last_sched.data(), S, bytes) == 0;
+    if (same) return EVO_OK;
+    EVO_CUDA(cudaEventSynchronize(h->stage_ev));
+    std::memcpy(h->stage, S, bytes);
+    if (add_ones) std::memset(h->stage + bytes, 1, one);
+    EVO_CUDA(cudaMemcpyAsync(h->sched, h->stage, total, cudaMemcpyHostToDevice, st));
+    EVO_CUDA(cudaEventRecord(h->stage_ev, st));
+    h->last_sched.assign(h->stage, h->stage + total);
+    h->last_rows = rows;
+    h->last_valid = true;
+    return EVO_OK;
+  }
+  h->last_valid = false;
+  EVO_CUDA(cudaMemcpyAsync(h->sched, S, bytes, cudaMemcpyDeviceToDevice, st));
+  if (add_ones) EVO_CUDA(cudaMemsetAsync(h->sched + bytes, 1, one, st));
+  EVO_CUDA(cudaMemsetAsync(h->status + 1, 0, sizeof(int), st));
+  EVO_CUDA(launch_validate(h->sched, (long long)bytes, h->status + 1, st));
+  *err_out = h->status + 1;
+  return EVO_OK;
+}
+
+evo_status finish(evo_handle* h, cudaStream_t st) {
+  h->last_stream = st;
+  if (cudaGetLastError() != cudaSuccess) return EVO_ERR_CUDA;
+  if (h->cfg.debug_sync) return evo_get_status(h);
+  return EVO_OK;
+}
+
+evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int S_rows, int N, float* out,
+               float* trace, void* stream) {
+  if (!h || !obs || !noise || !S || !out) return EVO_ERR_ARG;
+  if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
+  if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int* err = nullptr;
+  evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
+  if (s != EVO_OK) return s;
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, nullptr, h->kv_obs, st));
+  JobParams p = h->base;
+  p.samples = N;
+  p.per_sched = N;
+  p.obs_mod = N;
+  p.n_jobs = (N + p.g - 1) / p.g;
+  p.S = h->sched;
+  p.S_rows = S_rows;
+  p.S_stride = (long long)S_rows * h->T;
+  p.sched_err = err;
+  p.noise = noise;
+  p.out = out;
+  p.trace = trace;
+  EVO_CUDA(launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st));
+  return finish(h, st);
+}
+
+}  // namespace
+
+extern "C" {
+
+evo_status evo_denoise(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
+                       int32_t N, float* out_actions, void* stream) {
+  return run(h, obs, noise, S, S_rows, N, out_actions, nullptr, stream);
+}
+
+evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
+                             int32_t N, float* out_actions, float* trace, void* stream) {
+  if (!trace) return EVO_ERR_ARG;
+  return run(h, obs, noise, S, S_rows, N, out_actions, trace, stream);
+}
+
+evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* noise, const uint8_t* S_pop,
+                                  int32_t P, int32_t S_rows, int32_t N_obs, float* out_actions, float* dev_l2,
+                                  void* stream) {
+  if (!h || !obs || !noise || !S_pop || !dev_l2) return EVO_ERR_ARG;
+  if (P <= 0 || N_obs <= 0) return EVO_ERR_SHAPE;
+  const long long samples = (long long)(P + 1) * N_obs;
+  if (samples > h->max_batch) return EVO_ERR_SHAPE;
+  if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int* err = nullptr;
+  evo_status s = stage_schedules(h, S_pop, P, S_rows, true, st, &err);
+  if (s != EVO_OK) return s;
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, nullptr,
+                           h->kv_obs, st));
+  JobParams p = h->base;
+  // samples of one job must share a schedule: g divides N_obs
+  int g = p.g;
+  while (g > 1 && N_obs % g) --g;
+  if (g != p.g) {
+    p.g = g;
+    p.M = g * p.H;
+    p.Mp = rup(p.M, 16);
+    smem_layout(p, h->es);
+  }
+  p.samples = (int)samples;
+  p.per_sched = N_obs;
+  p.obs_mod = N_obs;
+  p.n_jobs = (int)((samples + p.g - 1) / p.g);
+  p.S = h->sched;
+  p.S_rows = S_rows;
+  p.S_stride = (long long)S_rows * h->T;
+  p.sched_err = err;
+  p.noise = noise;
+  p.out = h->pop_x;
+  p.trace = nullptr;
+  EVO_CUDA(launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st));
+  const int HA = h->H * h->A;
+  EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
+  if (out_actions)
+    EVO_CUDA(cudaMemcpyAsync(out_actions, h->pop_x, (size_t)P * N_obs * HA * 4, cudaMemcpyDeviceToDevice, st));
+  return finish(h, st);
+}
+
+evo_status evo_get_status(evo_handle* h) {
+  if (!h) return EVO_ERR_ARG;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return EVO_ERR_CUDA;
+  int st[2] = {0, 0};
+  if (cudaMemcpy(st, h->status, sizeof(st), cudaMemcpyDeviceToHost) != cudaSuccess) return EVO_ERR_CUDA;
+  if (st[0] || st[1]) cudaMemset(h->status, 0, sizeof(st));
+  if (st[1]) return EVO_ERR_SCHEDULE;
+  if (st[0] & ST_TIMEOUT) return EVO_ERR_TIMEOUT;
+  if (st[0] & ST_SCHEDULE) return EVO_ERR_SCHEDULE;
+  return EVO_OK;
+}
+
+}  // extern "C"
