@@ -1,0 +1,387 @@
+#!/usr/bin/env python
+"""Benchmark of schedule-driven cached denoising on one GB300 (one JSON line).
+
+Default workload: the Push-T-shaped policy (8 layers, n_emb 256, 4 heads,
+horizon 16 x action dim 2, 2 observation tokens of dim 20, 100 DDPM steps),
+batch 1, bf16, with refresh lattices at fractions 1.0 / 0.5 / 0.125.  One step
+is one action chunk (a full 100-step denoising query) through evo_denoise.
+`value` is chunks/s at the headline fraction 0.125; the line also carries the
+p50 latency and chunks/s of every fraction, the FLOP ratio they imply, the
+roofline of the denoising-loop kernel, an end-to-end figure through the C ABI
+with host buffers, and the CPU oracle timed on this machine's host cores.
+
+--impl reference times the CPU oracle itself on the same workload.
+Multi-GPU (torchrun): every rank runs an independent replica (the path has no
+exchange between chunks); value = chunks of all ranks / max rank time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2607_20293_gb300 import synth  # noqa: E402
+
+WORKLOADS = {
+    # name: (config, fractions, headline fraction, schedule kind)
+    "pusht": ("pusht", [1.0, 0.5, 0.125], 0.125, "bernoulli"),
+    "tiny": ("tiny", [1.0, 0.5], 0.5, "bernoulli_t0"),
+    "manip": ("manip", [1.0, 0.5, 0.125], 0.125, "bernoulli"),
+    "scale256": ("scale256", [1.0, 0.5, 0.25, 0.125], 0.125, "bernoulli"),
+    "scale1024": ("scale1024", [1.0, 0.5, 0.25, 0.125], 0.125, "bernoulli"),
+}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def describe(cfg: dict, n: int) -> str:
+    return (f"L{cfg['n_layer']} E{cfg['n_emb']} h{cfg['n_head']} H{cfg['horizon']} A{cfg['action_dim']} "
+            f"obs {cfg['n_obs']}x{cfg['obs_dim']} T{cfg['n_steps']} {cfg['sampler'].upper()} batch {n} {cfg['dtype']}")
+
+
+def schedule(cfg: dict, frac: float, kind: str) -> np.ndarray:
+    U, T = 3 * cfg["n_layer"], cfg["n_steps"]
+    return synth.bernoulli_schedule(U, T, frac, seed=3, force_t0=(kind == "bernoulli_t0"))
+
+
+def algorithmic_bytes(cfg: dict, S: np.ndarray, n: int) -> int:
+    """Bytes the cached loop must move per launch: the weights of every refreshed
+    unit (SA: W_qkv, W_o; CA: W_q, W_o -- memory keys/values are per query;
+    FFN: W_1, W_2), the per-step input/output projections, and one cache
+    tile per lattice cell and sample (written on refresh, read on skip)."""
+    E, H, A = cfg["n_emb"], cfg["horizon"], cfg["action_dim"]
+    es = 2 if cfg["dtype"] == "bf16" else 4
+    unit_w = [4 * E * E * es, 2 * E * E * es, 8 * E * E * es]
+    U, T = S.shape
+    w = sum(int(S[b].sum()) * unit_w[b % 3] for b in range(U))
+    fixed = T * ((A * E + H * E + E * A) * 4)
+    cache = U * T * n * H * E * es
+    return w + fixed + cache
+
+
+# ---------------------------------------------------------------------------- helpers
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.proc = None
+        self.index = index
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def measured_peaks() -> dict:
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return {}
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("evo_job.cu", "evo_internal.h"):
+        h.update(open(os.path.join(ROOT, "paper_2607_20293_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the denoising-loop kernel from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    try:
+        rec = json.load(open(path))
+    except Exception:
+        return None
+    ent = rec.get(workload)
+    if not ent or ent.get("kernel_sha") != kernel_source_hash():
+        return None
+    return ent.get("bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------- CPU oracle
+
+def _oracle_chunk(args):
+    name, frac, kind, seed = args
+    from oracle import evo_oracle as O
+    cfg = synth.config(name)
+    W = synth.make_weights(cfg, 0)
+    obs = synth.make_obs(cfg, 1, 1000 + seed)
+    noise = synth.make_noise(cfg, 1, 2000 + seed)
+    S = schedule(cfg, frac, kind)
+    O.denoise(W, cfg, obs, noise, S)
+    return 1
+
+
+def oracle_round(pool, name, frac, kind, n_chunks, base_seed=0) -> float:
+    t0 = time.perf_counter()
+    pool.map(_oracle_chunk, [(name, frac, kind, base_seed + i) for i in range(n_chunks)])
+    return time.perf_counter() - t0
+
+
+def make_pool():
+    import multiprocessing as mp
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[v] = "1"
+    workers = max(1, min(16, os.cpu_count() or 1))
+    return mp.get_context("spawn").Pool(workers), workers
+
+
+def cpu_baseline(name, frac, kind, pool, workers) -> dict:
+    oracle_round(pool, name, frac, kind, workers)           # warm the workers (imports, weights)
+    n = workers * 2
+    dt = oracle_round(pool, name, frac, kind, n, base_seed=100)
+    return {"value": n / dt, "unit": "chunks/s", "cores": workers, "kind": "oracle",
+            "sample": f"{n} single-sample chunks of the same workload at refresh fraction {frac}, "
+                      f"one float64 numpy oracle process per core"}
+
+
+# ---------------------------------------------------------------------------- GPU arm
+
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2607_20293_gb300 import binding, build
+
+    torch.cuda.set_device(local)
+    build.build()
+    binding.load()
+    name, fracs, head_frac, kind = WORKLOADS[args.workload]
+    cfg = synth.config(name)
+    n = cfg["batch"]
+    W = synth.make_weights(cfg, 0)
+    obs = synth.make_obs(cfg, n, 1 + 17 * rank)
+    noise = synth.make_noise(cfg, n, 2 + 17 * rank)
+    ev = binding.Evo(cfg, W, n)
+    d_obs, d_noise = torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda()
+    out = torch.empty((n, cfg["horizon"], cfg["action_dim"]), device="cuda")
+    h_obs, h_noise = torch.from_numpy(obs).pin_memory(), torch.from_numpy(noise).pin_memory()
+    h_out = torch.empty((n, cfg["horizon"], cfg["action_dim"])).pin_memory()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, device="cuda")
+    stream = torch.cuda.current_stream()
+    k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev.set_profile_events(k0, k1)
+    dist = world > 1
+    if dist:
+        import torch.distributed as tdist
+
+    def one(S, e2e=False):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        if e2e:
+            d_obs.copy_(h_obs, non_blocking=True)
+            d_noise.copy_(h_noise, non_blocking=True)
+        ev.denoise(d_obs, d_noise, S, out=out)
+        if e2e:
+            h_out.copy_(out, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        return a.elapsed_time(b), k0.elapsed_time(k1)
+
+    sweep = {}
+    headline = None
+    for frac in sorted(fracs, key=lambda f: f != head_frac):
+        S = schedule(cfg, frac, kind)
+        for _ in range(max(3, args.warmup)):
+            one(S)
+        if dist:
+            tdist.barrier()
+        torch.cuda.synchronize()
+        clocks = Clocks(local) if frac == head_frac else None
+        if clocks:
+            clocks.start()
+        steps, kern = [], []
+        for _ in range(args.steps):
+            ms, kms = one(S)
+            steps.append(ms)
+            kern.append(kms)
+        torch.cuda.synchronize()
+        if dist:
+            tdist.barrier()
+        clk = clocks.stop() if clocks else None
+        e2e = [one(S, e2e=True)[0] for _ in range(args.steps)]
+        fl = ev.flops(S)
+        rec = {"chunks_per_s": n * 1000.0 / statistics.mean(steps), "p50_ms": statistics.median(steps),
+               "kernel_ms_mean": statistics.mean(kern), "flops_per_chunk": fl, "ms": steps, "kernel_ms": kern,
+               "e2e_ms": e2e, "clocks": clk, "alg_bytes": algorithmic_bytes(cfg, S, n), "S": S}
+        sweep[frac] = rec
+        if frac == head_frac:
+            headline = rec
+    if ev.status() != binding.OK:
+        raise RuntimeError("device status reported an error")
+
+    total_s = sum(headline["ms"]) / 1000.0
+    total_e2e = sum(headline["e2e_ms"]) / 1000.0
+    if dist:
+        t = torch.tensor([total_s, total_e2e], device="cuda")
+        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+        total_s, total_e2e = float(t[0]), float(t[1])
+    if rank != 0:
+        return None
+    chunks = n * args.steps * world
+    full = sweep.get(1.0)
+    peaks = measured_peaks()
+    kern_ms = headline["kernel_ms_mean"]
+    big = n >= 64
+    if big:
+        achieved = headline["flops_per_chunk"] * n / (kern_ms / 1000.0) / 1e12
+        peak = peaks.get("bf16_tflops", 1900.0)
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "traffic": recorded_traffic(args.workload),
+                "peak_source": "measured bf16 burst" if "bf16_tflops" in peaks else "fallback"}
+    else:
+        achieved = headline["alg_bytes"] / (kern_ms / 1000.0) / 1e9
+        peak = peaks.get("hbm_gbs", 6800.0)
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": recorded_traffic(args.workload),
+                "peak_source": "measured HBM copy" if "hbm_gbs" in peaks else "fallback"}
+    roof["kernel"] = "evo::job_kernel"
+    roof["algorithmic_per_launch"] = headline["flops_per_chunk"] * n if big else headline["alg_bytes"]
+    roof["kernel_ms"] = kern_ms
+    bytes_in = (obs.nbytes + noise.nbytes)
+    line = {
+        "metric": "action chunks/s (p50 chunk latency and refresh-fraction sweep alongside)",
+        "value": chunks / total_s,
+        "unit": "chunks/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": 1000.0 * total_s / args.steps,
+        "p50_ms": headline["p50_ms"],
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": cfg["dtype"],
+        "data": "synthetic (seeded N(0,0.02) weights, N(0,1) observation features and noise)",
+        "config": {"workload": f"{args.workload}-shaped: {describe(cfg, n)}", "batch": n,
+                   "refresh_fraction": head_frac, "schedule": f"{kind} lattice, seed 3",
+                   "l2": "flushed between timed steps (256 MiB write)",
+                   "parallelism": f"replicas x{world}"},
+        "sweep": {str(f): {"chunks_per_s": r["chunks_per_s"], "p50_ms": r["p50_ms"],
+                           "kernel_ms": r["kernel_ms_mean"], "gflop_per_chunk": r["flops_per_chunk"] / 1e9,
+                           "flop_ratio_vs_full": (full["flops_per_chunk"] / r["flops_per_chunk"]) if full else None,
+                           "speedup_vs_full": (r["chunks_per_s"] / full["chunks_per_s"]) if full else None}
+                  for f, r in sorted(sweep.items(), key=lambda kv: -kv[0])},
+        "roofline": roof,
+        "e2e": {"value": chunks / total_e2e, "unit": "chunks/s", "h2d_bytes_per_step": bytes_in,
+                "d2h_bytes_per_step": int(h_out.numel() * 4)},
+        "gpu_launches": 2 * args.steps,
+        "clocks": headline["clocks"],
+        "launch": ev.launch_info(),
+    }
+    return line, cfg
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="pusht", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+    name, fracs, head_frac, kind = WORKLOADS[args.workload]
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        pool, workers = make_pool()
+        try:
+            for _ in range(max(1, min(args.warmup, 3))):
+                oracle_round(pool, name, head_frac, kind, workers)
+            times = [oracle_round(pool, name, head_frac, kind, workers, base_seed=10 * i) for i in range(args.steps)]
+        finally:
+            pool.close()
+        total = sum(times)
+        v = workers * args.steps / total
+        cfg = synth.config(name)
+        print(json.dumps({
+            "impl": "reference", "metric": "action chunks/s (p50 chunk latency and refresh-fraction sweep alongside)",
+            "value": v, "unit": "chunks/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{args.workload}-shaped: {describe(cfg, cfg['batch'])}", "batch": cfg["batch"],
+                       "refresh_fraction": head_frac, "schedule": f"{kind} lattice, seed 3"},
+            "cpu_baseline": {"value": v, "unit": "chunks/s", "cores": workers, "kind": "oracle",
+                             "sample": f"each step: {workers} single-sample chunks, one float64 numpy oracle "
+                                       f"process per core"},
+            "e2e": {"value": v, "unit": "chunks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }))
+        return
+
+    pool = workers = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        pool, workers = make_pool()          # spawned before the first GPU call
+    dist = world > 1
+    if dist:
+        import torch
+        import torch.distributed as tdist
+        torch.cuda.set_device(local)
+        tdist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    res = run_ours(args, world, rank, local)
+    if res is not None:
+        line, cfg = res
+        if pool is not None:
+            line["cpu_baseline"] = cpu_baseline(name, head_frac, kind, pool, workers)
+            pool.close()
+        print(json.dumps(line))
+    if dist:
+        tdist.barrier()
+        tdist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

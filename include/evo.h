@@ -147,6 +147,12 @@ evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise
                              const uint8_t* S, int32_t S_rows, int32_t N,
                              float* out_actions, float* trace, void* stream);
 
+/* Profiling hook: when both events are non-NULL (cudaEvent_t passed as void*),
+ * every launch of the denoising-loop kernel is bracketed by cudaEventRecord
+ * of `start` and `stop` on the call's stream, so a caller can read that
+ * kernel's own duration.  Pass NULL, NULL to turn it off. */
+evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop);
+
 /* Synchronizes the handle's last stream, returns and clears the device status word. */
 evo_status evo_get_status(evo_handle* h);
 

@@ -57,6 +57,7 @@ def load() -> ctypes.CDLL:
         "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
         "evo_schedule_from_positions": (I32, [P, I32, I32, I32, P]),
         "evo_get_status": (I32, [P]),
+        "evo_set_profile_events": (I32, [P, P, P]),
         "evo_get_launch_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(I32),
                                       ctypes.POINTER(I32)]),
         "evo_status_string": (ctypes.c_char_p, [I32]),
@@ -210,6 +211,12 @@ class Evo:
         out = ctypes.c_int64()
         _check(load().evo_flops(self._h, S.ctypes.data, S.shape[0], ctypes.byref(out)), "evo_flops")
         return out.value
+
+    def set_profile_events(self, start=None, stop=None):
+        """Bracket every denoising-loop kernel launch with these torch.cuda.Events."""
+        sp = start.cuda_event if start is not None else None
+        ep = stop.cuda_event if stop is not None else None
+        _check(load().evo_set_profile_events(self._h, sp, ep), "evo_set_profile_events")
 
     def status(self) -> int:
         return load().evo_get_status(self._h)

@@ -53,12 +53,11 @@ struct evo_handle {
   int last_rows = -1;
   bool last_valid = false;
   cudaStream_t last_stream = nullptr;
+  cudaEvent_t prof_start = nullptr, prof_stop = nullptr;
   int woff[W_COUNT];
 };
 
 namespace {
-
-inline evo_status cuda_st(cudaError_t e) { return e == cudaSuccess ? EVO_OK : EVO_ERR_CUDA; }
 
 #define EVO_CUDA(x)                                   \
   do {                                                \
@@ -618,6 +617,17 @@ evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int row
   return EVO_OK;
 }
 
+cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st) {
+  if (h->prof_start && h->prof_stop) {
+    cudaError_t e = cudaEventRecord(h->prof_start, st);
+    if (e != cudaSuccess) return e;
+  }
+  cudaError_t e = launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st);
+  if (e != cudaSuccess) return e;
+  if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
+  return cudaSuccess;
+}
+
 evo_status finish(evo_handle* h, cudaStream_t st) {
   h->last_stream = st;
   if (cudaGetLastError() != cudaSuccess) return EVO_ERR_CUDA;
@@ -647,7 +657,7 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   p.noise = noise;
   p.out = out;
   p.trace = trace;
-  EVO_CUDA(launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st));
+  EVO_CUDA(launch_loop(h, p, st));
   return finish(h, st);
 }
 
@@ -701,12 +711,19 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   p.noise = noise;
   p.out = h->pop_x;
   p.trace = nullptr;
-  EVO_CUDA(launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st));
+  EVO_CUDA(launch_loop(h, p, st));
   const int HA = h->H * h->A;
   EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
   if (out_actions)
     EVO_CUDA(cudaMemcpyAsync(out_actions, h->pop_x, (size_t)P * N_obs * HA * 4, cudaMemcpyDeviceToDevice, st));
   return finish(h, st);
+}
+
+evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
+  if (!h || (start == nullptr) != (stop == nullptr)) return EVO_ERR_ARG;
+  h->prof_start = reinterpret_cast<cudaEvent_t>(start);
+  h->prof_stop = reinterpret_cast<cudaEvent_t>(stop);
+  return EVO_OK;
 }
 
 evo_status evo_get_status(evo_handle* h) {
