@@ -210,6 +210,8 @@ def run_ours(args, world, rank, local):
     flush = torch.empty(L2_FLUSH_BYTES // 4, device="cuda")
     stream = torch.cuda.current_stream()
     k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    k0.record(stream)                # torch creates the CUDA events on first record
+    k1.record(stream)
     ev.set_profile_events(k0, k1)
     dist = world > 1
     if dist:

@@ -213,7 +213,8 @@ class Evo:
         return out.value
 
     def set_profile_events(self, start=None, stop=None):
-        """Bracket every denoising-loop kernel launch with these torch.cuda.Events."""
+        """Bracket every denoising-loop kernel launch with these torch.cuda.Events
+        (they must have been recorded once, so that their CUDA events exist)."""
         sp = start.cuda_event if start is not None else None
         ep = stop.cuda_event if stop is not None else None
         _check(load().evo_set_profile_events(self._h, sp, ep), "evo_set_profile_events")
