@@ -69,9 +69,9 @@ bool config_ok(const evo_config* c) {
   if (!c) return false;
   if (c->n_layer <= 0 || c->n_layer > 21) return false;          // 3L units tracked in a 64-bit mask
   if (c->n_emb <= 0 || c->n_head <= 0 || c->n_emb % c->n_head) return false;
-  if (c->n_emb % 32 || c->n_emb > 512) return false;             // LayerNorm: <= 16 values per lane
+  if (c->n_emb % 64 || c->n_emb > 512) return false;             // LayerNorm: float4 chunks over half a warp
   if (c->horizon <= 0 || c->horizon > 32 || c->horizon % 4) return false;
-  if (c->action_dim <= 0 || c->action_dim > 32) return false;
+  if (c->action_dim <= 0 || c->action_dim > 16) return false;
   if (c->n_obs <= 0 || c->n_obs > 31 || c->obs_dim <= 0) return false;
   if (c->n_steps <= 0 || c->train_steps <= 0 || c->train_steps % c->n_steps) return false;
   if (c->sampler != EVO_SAMPLER_DDPM && c->sampler != EVO_SAMPLER_DDIM) return false;
@@ -219,10 +219,18 @@ bool lattice_ok(const uint8_t* S, size_t n) {
   return true;
 }
 
+inline bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+inline int ilog2(int x) {
+  int l = 0;
+  while ((1 << l) < x) ++l;
+  return l;
+}
+
 // Fill p's decomposition fields for g samples per job; returns shared bytes or -1.
 int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
   const int E = c->n_emb, dh = E / c->n_head, H = c->horizon;
   const int es = c->dtype == EVO_DTYPE_BF16 ? 2 : 4;
+  auto r84 = [](int x) { return x + ((12 - x % 8) % 8); };      // smallest y >= x with y % 8 == 4
   p.L = c->n_layer;
   p.E = E;
   p.nh = c->n_head;
@@ -239,39 +247,52 @@ int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
   p.g = g;
   p.M = g * H;
   p.Mp = rup(p.M, 16);
-  p.ldf = E + 4;
-  p.n1_sa = 2 * dh + p.Ec;
-  p.n1_ca = dh;
-  p.n1_ff = p.hid;
-  p.n1max = std::max(p.n1_sa, p.n1_ff);
-  p.ldg1 = p.n1_sa + 1;
+  if (!pow2(p.Ec) || !pow2(H) || !pow2(g)) return -1;
+  p.lEc = ilog2(p.Ec);
+  p.lH = ilog2(H);
+  p.blk = p.M * p.Ec + 4;
+  p.lda = es == 2 ? E + 8 : E + 4;
+  p.n1[0] = 2 * dh + p.Ec;
+  p.n1[1] = dh;
+  p.n1[2] = p.hid;
+  p.ldg1 = r84(p.n1[0]);
+  p.kvw = r84(dh + p.Ec);
   p.kp_o = rup(p.Ec, 16);
   p.kp_h = rup(p.hid, 16);
   p.ldh = es == 2 ? p.kp_h + 8 : p.kp_h;
   p.ldo = es == 2 ? p.kp_o + 8 : p.kp_o;
+  for (int u = 0; u < 3; ++u) p.hdr1[u] = rup(2 * E + p.n1[u] + p.Ec, 4) * 4;
   p.sampler = c->sampler;
   p.force = c->empty_cache == EVO_EMPTY_FORCE;
+  if (p.Cm > 32 || p.M * p.Ec > 4 * NCT) return -1;
   if (es == 2) {
     if (p.Mp > 32) return -1;
   } else {
-    const int nmax = std::max(p.n1max, E);
+    const int nmax = std::max(std::max(p.n1[0], p.n1[2]), E);
     if (p.M * nmax > 16 * NCT) return -1;
   }
-  // largest k-tile of any piece
-  const int max_ktile = 16 * std::max(p.n1max, E) * es;
-  const int slots[] = {32768, 16384};
-  for (int head_sep = 1; head_sep >= 0; --head_sep) {
-    for (int sb : slots) {
-      if (sb < max_ktile) continue;
-      for (int ns = 4; ns >= 2; --ns) {
-        p.head_sep = head_sep;
-        p.slot_bytes = sb;
-        p.nslot = ns;
-        const int total = smem_layout(p, es);
-        if (total <= smem_limit) return total;
-      }
-    }
-  }
+  // a ring slot must hold any piece-1 header plus one k-tile, and one k-tile of piece 2
+  int need = 16 * E * es;
+  for (int u = 0; u < 3; ++u) need = std::max(need, p.hdr1[u] + 16 * p.n1[u] * es);
+  const int slots[] = {32768, 24576, 16384};
+  // preference: caches on chip, per-step memory keys/values, double-buffered
+  // head exchange, head weights on chip, deep ring
+  for (int cache_smem = 1; cache_smem >= 0; --cache_smem)
+    for (int kvall = 1; kvall >= 0; --kvall)
+      for (int head_sep = 1; head_sep >= 0; --head_sep)
+        for (int headw = 1; headw >= 0; --headw)
+          for (int sb : slots) {
+            if (sb < need) continue;
+            for (int ns = 4; ns >= 2; --ns) {
+              p.kv_slots = kvall ? p.L : 1;
+              p.head_sep = head_sep;
+              p.headw_smem = headw;
+              p.slot_bytes = sb;
+              p.nslot = ns;
+              const int total = smem_layout(p, es, cache_smem);
+              if (total <= smem_limit) return total;
+            }
+          }
   return -1;
 }
 
@@ -435,9 +456,9 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   const int es = h->es;
   const int Ec = p.Ec, hid = p.hid;
   // piece sizes (bytes) and offsets within one layer block
-  const long long sz[3][2] = {{(long long)E * p.n1_sa * es, (long long)p.kp_o * E * es},
-                              {(long long)E * p.n1_ca * es, (long long)p.kp_o * E * es},
-                              {(long long)E * p.n1_ff * es, (long long)p.kp_h * E * es}};
+  const long long sz[3][2] = {{p.hdr1[0] + (long long)E * p.n1[0] * es, (long long)p.kp_o * E * es},
+                              {p.hdr1[1] + (long long)E * p.n1[1] * es, (long long)p.kp_o * E * es},
+                              {p.hdr1[2] + (long long)E * p.n1[2] * es, (long long)p.kp_h * E * es}};
   long long off = 0;
   for (int u = 0; u < 3; ++u)
     for (int q = 0; q < 2; ++q) {
@@ -465,8 +486,20 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
         for (int n = 0; n < N; ++n) d[(size_t)k * N + n] = get(k, n);
     }
   };
+  // piece 1 = [float32 header][k-tiles], header = LayerNorm gain, shift, the
+  // first GEMM's bias columns and this CTA's columns of the second GEMM's bias;
+  // piece 2 = [k-tiles]
+  auto header = [&](uint8_t* dst, const float* g, const float* b, const float* bias, int nbias, auto colmap,
+                    const float* bias2) {
+    float* d = reinterpret_cast<float*>(dst);
+    for (int i = 0; i < E; ++i) d[i] = g[i];
+    for (int i = 0; i < E; ++i) d[E + i] = b[i];
+    for (int i = 0; i < nbias; ++i) d[2 * E + i] = bias[colmap(i)];
+    for (int i = 0; i < Ec; ++i) d[2 * E + nbias + i] = bias2[i];
+  };
   for (int c = 0; c < C; ++c) {
     const int h0 = (c * Ec) / dh;
+    auto qkv_col = [&](int n) { return n < dh ? h0 * dh + n : (n < 2 * dh ? E + h0 * dh + (n - dh) : 2 * E + c * Ec + (n - 2 * dh)); };
     for (int l = 0; l < L; ++l) {
       uint8_t* base = pack.data() + (size_t)c * p.cta_stride + (size_t)l * p.layer_stride;
       const float* wqkv = WL(l, WL_SA_WQKV);
@@ -475,18 +508,21 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
       const float* wo2 = WL(l, WL_CA_WO);
       const float* w1 = WL(l, WL_FF_W1);
       const float* w2 = WL(l, WL_FF_W2);
-      put(base + p.poff[0][0], E, p.n1_sa, [&](int k, int n) {
-        const int col = n < dh ? h0 * dh + n : (n < 2 * dh ? E + h0 * dh + (n - dh) : 2 * E + c * Ec + (n - 2 * dh));
-        return wqkv[(size_t)k * 3 * E + col];
-      });
-      put(base + p.poff[0][1], p.kp_o, E,
-          [&](int k, int n) { return k < Ec ? wo1[(size_t)(c * Ec + k) * E + n] : 0.f; });
-      put(base + p.poff[1][0], E, p.n1_ca, [&](int k, int n) { return wq[(size_t)k * E + h0 * dh + n]; });
-      put(base + p.poff[1][1], p.kp_o, E,
-          [&](int k, int n) { return k < Ec ? wo2[(size_t)(c * Ec + k) * E + n] : 0.f; });
-      put(base + p.poff[2][0], E, p.n1_ff, [&](int k, int n) { return w1[(size_t)k * 4 * E + c * hid + n]; });
-      put(base + p.poff[2][1], p.kp_h, E,
-          [&](int k, int n) { return k < hid ? w2[(size_t)(c * hid + k) * E + n] : 0.f; });
+      // SA
+      header(base + p.poff[0][0], WL(l, WL_LN1G), WL(l, WL_LN1B), WL(l, WL_SA_BQKV), p.n1[0], qkv_col,
+             WL(l, WL_SA_BO) + c * Ec);
+      put(base + p.poff[0][0] + p.hdr1[0], E, p.n1[0], [&](int k, int n) { return wqkv[(size_t)k * 3 * E + qkv_col(n)]; });
+      put(base + p.poff[0][1], p.kp_o, E, [&](int k, int n) { return k < Ec ? wo1[(size_t)(c * Ec + k) * E + n] : 0.f; });
+      // CA
+      header(base + p.poff[1][0], WL(l, WL_LN2G), WL(l, WL_LN2B), WL(l, WL_CA_BQ), p.n1[1],
+             [&](int n) { return h0 * dh + n; }, WL(l, WL_CA_BO) + c * Ec);
+      put(base + p.poff[1][0] + p.hdr1[1], E, p.n1[1], [&](int k, int n) { return wq[(size_t)k * E + h0 * dh + n]; });
+      put(base + p.poff[1][1], p.kp_o, E, [&](int k, int n) { return k < Ec ? wo2[(size_t)(c * Ec + k) * E + n] : 0.f; });
+      // FFN
+      header(base + p.poff[2][0], WL(l, WL_LN3G), WL(l, WL_LN3B), WL(l, WL_FF_B1), p.n1[2],
+             [&](int n) { return c * hid + n; }, WL(l, WL_FF_B2) + c * Ec);
+      put(base + p.poff[2][0] + p.hdr1[2], E, p.n1[2], [&](int k, int n) { return w1[(size_t)k * 4 * E + c * hid + n]; });
+      put(base + p.poff[2][1], p.kp_h, E, [&](int k, int n) { return k < hid ? w2[(size_t)(c * hid + k) * E + n] : 0.f; });
     }
   }
   if (cudaMalloc(&h->wpack, pack.size()) != cudaSuccess) return fail(EVO_ERR_OOM);
@@ -499,9 +535,6 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
     dst = (long long)vec.size();
     vec.resize(vec.size() + n, 0.f);
   };
-  vtake(p.v_ln, (size_t)U * 2 * E);
-  vtake(p.v_b1, (size_t)U * C * p.n1max);
-  vtake(p.v_b2, (size_t)U * E);
   vtake(p.v_inw, (size_t)A * E);
   vtake(p.v_inb, E);
   vtake(p.v_pos, (size_t)H * E);
@@ -509,30 +542,6 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   vtake(p.v_lnfb, E);
   vtake(p.v_headw, (size_t)E * A);
   vtake(p.v_headb, A);
-  for (int b = 0; b < U; ++b) {
-    const int l = b / 3, u = b % 3;
-    const int gid = u == 0 ? WL_LN1G : (u == 1 ? WL_LN2G : WL_LN3G);
-    const int bid = u == 0 ? WL_LN1B : (u == 1 ? WL_LN2B : WL_LN3B);
-    std::memcpy(&vec[p.v_ln + (size_t)b * 2 * E], WL(l, gid), E * 4);
-    std::memcpy(&vec[p.v_ln + (size_t)b * 2 * E + E], WL(l, bid), E * 4);
-    const float* b2 = u == 0 ? WL(l, WL_SA_BO) : (u == 1 ? WL(l, WL_CA_BO) : WL(l, WL_FF_B2));
-    std::memcpy(&vec[p.v_b2 + (size_t)b * E], b2, E * 4);
-    for (int c = 0; c < C; ++c) {
-      float* d = &vec[p.v_b1 + ((size_t)b * C + c) * p.n1max];
-      const int h0 = (c * Ec) / dh;
-      if (u == 0) {
-        const float* bq = WL(l, WL_SA_BQKV);
-        for (int n = 0; n < p.n1_sa; ++n)
-          d[n] = bq[n < dh ? h0 * dh + n : (n < 2 * dh ? E + h0 * dh + (n - dh) : 2 * E + c * Ec + (n - 2 * dh))];
-      } else if (u == 1) {
-        const float* bq = WL(l, WL_CA_BQ);
-        for (int n = 0; n < dh; ++n) d[n] = bq[h0 * dh + n];
-      } else {
-        const float* b1 = WL(l, WL_FF_B1);
-        for (int n = 0; n < hid; ++n) d[n] = b1[c * hid + n];
-      }
-    }
-  }
   std::memcpy(&vec[p.v_inw], W(W_IN_W), (size_t)A * E * 4);
   std::memcpy(&vec[p.v_inb], W(W_IN_B), E * 4);
   std::memcpy(&vec[p.v_pos], W(W_POS), (size_t)H * E * 4);
@@ -644,7 +653,7 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, nullptr, h->kv_obs, st));
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, h->kv_obs, st));
   JobParams p = h->base;
   p.samples = N;
   p.per_sched = N;
@@ -688,17 +697,17 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S_pop, P, S_rows, true, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, nullptr,
-                           h->kv_obs, st));
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, h->kv_obs, st));
   JobParams p = h->base;
   // samples of one job must share a schedule: g divides N_obs
   int g = p.g;
-  while (g > 1 && N_obs % g) --g;
+  while (g > 1 && N_obs % g) g >>= 1;
   if (g != p.g) {
     p.g = g;
     p.M = g * p.H;
     p.Mp = rup(p.M, 16);
-    smem_layout(p, h->es);
+    p.blk = p.M * p.Ec + 4;
+    smem_layout(p, h->es, p.sm.cs >= 0);
   }
   p.samples = (int)samples;
   p.per_sched = N_obs;

@@ -12,7 +12,7 @@ constexpr int NCW = 8;              // compute warps per CTA
 constexpr int NCT = NCW * 32;       // compute threads per CTA
 constexpr int NTHREADS = NCT + 32;  // + one weight-streaming (producer) warp
 constexpr int MAX_CLUSTER = 16;
-constexpr int MAX_SLOTS = 8;
+constexpr int PLD = 33;             // row stride (floats) of the attention-probability buffer
 
 // error bits written to the device status word
 constexpr int ST_SCHEDULE = 1;
@@ -20,19 +20,22 @@ constexpr int ST_TIMEOUT = 2;
 
 // Byte offsets of the regions of one CTA's dynamic shared memory.
 struct SmemLayout {
-  int ring;    // nslot * slot_bytes, weight slabs streamed by the producer warp
-  int afull;   // [Mp][ldf] f32: gathered residual rows; normalised in place into the GEMM A operand
-  int hbuf;    // [M][ldf] f32: gathered rows for the output head (or -1: head uses afull)
-  int rs;      // [C][M][Ec] f32: reduce-scatter landing zone of the second GEMM's partial sums
-  int g1;      // first-GEMM output: q|k|v (f32, row stride ldg1) or FFN hidden (T, row stride ldh)
+  int ring;    // nslot * slot_bytes: weight slabs (with the unit's LayerNorm/bias vectors) streamed by the producer warp
+  int ablk;    // [C][blk] f32: gathered residual columns, block c from CTA c; also the staging of outgoing partial sums
+  int rs;      // [C][blk] f32: incoming partial sums of the second GEMM, block c from CTA c
+  int xln;     // [Mp][lda] T: normalised rows, the first GEMM's A operand; aliased by the first GEMM's output
+  int hblk;    // 2 x [C][blk] f32: gathered columns for the output head, by step parity (or -1: the head uses ablk)
+  int hsrc;    // 2 x [M*Ec] f32: the head's outgoing copy of this CTA's columns, by step parity
+  int pb;      // [M][PLD] f32: attention probabilities
   int oc;      // [Mp][ldo] T: attention output slice, A operand of the second GEMM
   int ac;      // [M][Ec] f32: this CTA's columns of the residual stream
-  int kvs;     // [g][1+n_obs][dh+Ec] f32: memory keys/values staged for one cross-attention unit
-  int cst;     // in_w slice [A][Ec], in_b slice [Ec], pos slice [H][Ec] (f32)
+  int cs;      // [3L][M][Ec] T: this CTA's columns of every unit's cache (or -1: caches in global memory)
+  int kvs;     // [kv_slots][g][1+n_obs][kvw] f32: memory keys/values for cross-attention
+  int cst;     // f32 constants: in_w[:, cols], in_b[cols], pos[:, cols], lnf_g, lnf_b, head_b, (head_w)
   int x;       // [M][A] f32: current sample x (replicated in every CTA of the cluster)
   int z;       // [M][A] f32: DDPM noise of the current step
-  int sch;     // [3L][T] u8: this job's lattice, one row per unit
-  int bars;    // mbarriers: full[nslot], empty[nslot], cluster
+  int sch;     // [T] u64: this job's lattice, bit b of word t = unit b refreshed at step t
+  int bars;    // mbarriers: full[nslot], empty[nslot], cluster, xg, xr, xh
   int total;
 };
 
@@ -41,13 +44,17 @@ struct JobParams {
   int L, E, nh, dh, H, A, n_obs, T, U, Cm;
   // decomposition
   int C, Ec, hid, g, M, Mp;
-  int ldf, ldg1, ldh, ldo;
-  int n1_sa, n1_ca, n1_ff, n1max;
-  int kp_o, kp_h;                 // padded K of the second GEMMs (attention: Ec, FFN: hid)
+  int blk;                        // floats per exchange block (M*Ec + 4)
+  int lda, ldg1, ldh, ldo, kvw;   // row strides (elements) of xln, q|k|v, hidden, attention output, memory k|v
+  int lEc, lH;                    // log2 of Ec and H
+  int n1[3];                      // first-GEMM width per unit kind (SA, CA, FFN)
+  int hdr1[3];                    // header bytes of piece 1: gamma, beta, first bias, second-GEMM bias slice
+  int kv_slots;                   // L: memory keys/values of every layer prefetched per step; 1: per unit
+  int kp_o, kp_h;                 // K of the second GEMMs (attention: Ec, FFN: hid), multiples of 16
   int n_jobs;
   int sampler, force;
   int nslot, slot_bytes;
-  int head_sep;
+  int head_sep, headw_smem;
   // samples
   int samples;                    // real samples in this launch
   int per_sched;                  // samples that share one schedule
@@ -70,22 +77,46 @@ struct JobParams {
   long long poff[3][2];           // piece byte offset within a layer block
   // float32 vectors
   const float* vec;
-  long long v_ln, v_b1, v_b2, v_inw, v_inb, v_pos, v_lnfg, v_lnfb, v_headw, v_headb;
-  // caches [n_jobs][U][C][M][Ec] (dtype T)
+  long long v_inw, v_inb, v_pos, v_lnfg, v_lnfb, v_headw, v_headb;
+  // caches [n_jobs][U][C][M][Ec] (dtype T), used when sm.cs < 0
   void* cache;
   float* trace;                   // [T][U][samples][H][E] or null
   int* status;
   SmemLayout sm;
 };
 
+// Slab partition of one weight piece: a header of `hdr` bytes followed by nkt
+// k-tiles of ktb bytes, cut into ring slots of `slot` bytes.  Slab 0 carries the
+// header and as many whole k-tiles as fit; later slabs carry whole k-tiles.
+struct SlabInfo {
+  int kt0, nkt, off, bytes;
+};
+
+__host__ __device__ inline int slab_count(int hdr, int ktb, int nkt, int slot) {
+  const int k0 = (slot - hdr) / ktb;
+  if (nkt <= k0) return 1;
+  const int kps = slot / ktb;
+  return 1 + (nkt - k0 + kps - 1) / kps;
+}
+
+__host__ __device__ inline SlabInfo slab_at(int s, int hdr, int ktb, int nkt, int slot) {
+  int k0 = (slot - hdr) / ktb;
+  if (k0 > nkt) k0 = nkt;
+  if (s == 0) return SlabInfo{0, k0, 0, hdr + k0 * ktb};
+  const int kps = slot / ktb;
+  const int kt0 = k0 + (s - 1) * kps;
+  const int n = (nkt - kt0) < kps ? (nkt - kt0) : kps;
+  return SlabInfo{kt0, n, hdr + kt0 * ktb, n * ktb};
+}
+
 // host helpers implemented in evo_job.cu
-int  smem_layout(JobParams& p, int elem_bytes);           // fills p.sm, returns total bytes
+int  smem_layout(JobParams& p, int elem_bytes, int cache_smem);   // fills p.sm, returns total bytes
 cudaError_t launch_job(const JobParams& p, int dtype, int n_clusters, cudaStream_t s);
 cudaError_t job_kernel_prepare(int dtype, int smem_bytes, int cluster, int* max_clusters);
 cudaError_t launch_time_table(const float* wf32, const int* woff, const float* stab_k, int T, int L, int E,
                               float* kv_time, cudaStream_t s);
 cudaError_t launch_obs_cond(const float* wf32, const int* woff, const float* obs, int N, int n_obs, int D,
-                            int L, int E, float* mem_scratch, float* kv_obs, cudaStream_t s);
+                            int L, int E, float* kv_obs, cudaStream_t s);
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s);
 cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev, cudaStream_t s);
 

@@ -12,30 +12,36 @@
 //                  : a += c_b                        (skip: a local add)
 //     eps = LN_f(a) W_head + b_head ; x <- sampler step(x, eps, z_t)
 //
-// The residual stream a is distributed over the cluster by columns; each CTA
-// owns E/C columns of a and of every unit's cache c_b, so a skipped cell costs
-// one local add of cached values.  A refreshed unit needs two cluster
-// exchanges: the CTAs all-gather a (distributed shared memory stores) to
-// normalise full rows, each computes its share of the branch (attention: the
-// queries/keys of its head and its slice of head dimensions; FFN: its slice
-// of the hidden layer), and the second matmul's partial sums are
-// reduce-scattered so that each CTA finishes its own columns.
+// The residual stream a is distributed over the cluster by columns: each CTA
+// owns E/C columns of a and of every unit's cache c_b (in shared memory when
+// the slice fits, else in global memory), so a skipped cell is a local add.
+// A refreshed unit needs two cluster exchanges, both done with bulk
+// asynchronous copies from this CTA's shared memory into the other CTAs'
+// (cp.async.bulk shared::cta -> shared::cluster, one per destination) that
+// count their bytes on the receiver's mbarrier -- no fences and no
+// cluster-wide barriers:
+//   1. all-gather of a, so every CTA normalises full rows (LayerNorm);
+//   2. reduce-scatter of the second matmul's partial sums, so every CTA
+//      finishes its own columns of r = branch output.
+// In between each CTA computes its share of the branch: attention -- the
+// queries/keys of its head and its slice of head dimensions; FFN -- its slice
+// of the hidden layer.  The order of the exchanges makes every buffer's reuse
+// safe: a CTA can only send into a buffer again after it has received data
+// that the receiver sends once it has finished reading that buffer.
 //
 // Weights never pass through registers on their way in: a producer warp per
 // CTA walks the same schedule and streams, for every refreshed unit only, the
-// CTA's pre-packed weight slices through a ring of shared-memory slots with
-// bulk asynchronous copies (cp.async.bulk + mbarrier transaction counts).
-// Skipped units generate no weight traffic, so time follows the schedule's
-// refresh count.
+// CTA's pre-packed weight slices (with the unit's LayerNorm gain/shift and
+// biases in front) through a ring of shared-memory slots with bulk
+// asynchronous copies (cp.async.bulk + mbarrier transaction counts).  Skipped
+// units generate no weight traffic, so time follows the schedule.
 //
 // bf16 mode: GEMM operands bf16, mma.sync m16n8k16 with fp32 accumulation
 // (rows per job are 16..32, far below a tcgen05 tile; the cost here is weight
-// streaming and cluster latency, not tensor throughput).  fp32 mode: FFMA.
+// streaming and on-chip latency, not tensor throughput).  fp32 mode: FFMA.
 // Caches are stored in the GEMM operand type.
 
 #include "evo_internal.h"
-
-#include <cstdio>
 
 namespace evo {
 
@@ -102,19 +108,40 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-__device__ __forceinline__ void st_cluster_v4(uint32_t addr, float4 v) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y), "f"(v.z),
-               "f"(v.w)
+// asynchronous store into (possibly remote) shared memory; the bytes are
+// counted on the mbarrier `rbar` of the receiving CTA
+__device__ __forceinline__ void st_async_v4(uint32_t raddr, float4 v, uint32_t rbar) {
+  asm volatile(
+      "st.async.weak.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+          raddr),
+      "r"(__float_as_uint(v.x)), "r"(__float_as_uint(v.y)), "r"(__float_as_uint(v.z)), "r"(__float_as_uint(v.w)),
+      "r"(rbar)
+      : "memory");
+}
+
+__device__ __forceinline__ void st_async_v2(uint32_t raddr, float a, float b, uint32_t rbar) {
+  asm volatile("st.async.weak.shared::cluster.mbarrier::complete_tx::bytes.v2.b32 [%0], {%1, %2}, [%3];" ::"r"(
+                   raddr),
+               "r"(__float_as_uint(a)), "r"(__float_as_uint(b)), "r"(rbar)
                : "memory");
 }
 
-__device__ __forceinline__ void st_cluster_v2(uint32_t addr, float a, float b) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(a), "f"(b) : "memory");
+__device__ __forceinline__ void st_async_f32(uint32_t raddr, float a, uint32_t rbar) {
+  asm volatile("st.async.weak.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+               "r"(__float_as_uint(a)), "r"(rbar)
+               : "memory");
 }
 
-__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float a) {
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(a) : "memory");
+// bulk copy of `bytes` from this CTA's shared memory to a cluster-mapped
+// address; completion counted on the (cluster-mapped) mbarrier of the receiver
+__device__ __forceinline__ void bulk_s2c(uint32_t dst, const void* src, uint32_t bytes, uint32_t rbar) {
+  asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "r"(smem_u32(src)), "r"(bytes), "r"(rbar)
+               : "memory");
 }
+
+// orders this thread's generic-proxy shared-memory writes before later bulk copies
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void fence_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
 
@@ -164,15 +191,21 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b.x), "r"(b.y));
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
+// reductions over groups of G consecutive lanes (G a power of two <= 32)
+template <int G>
+__device__ __forceinline__ float group_sum(float v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+__device__ __forceinline__ float group_sum_dyn(float v, int G) {
+  for (int o = G / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float group_max_dyn(float v, int G) {
+  for (int o = G / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
 
@@ -197,9 +230,9 @@ __device__ __forceinline__ float mish(float x) {
   return x * tanhf(sp);
 }
 
-// a bounded wait: after ~2 s of SM cycles the wait gives up, records
+// A bounded wait: after ~2 s of SM cycles the wait gives up, records
 // ST_TIMEOUT and lets the thread continue so that every CTA still reaches the
-// same barriers and the kernel ends.
+// same synchronisation points and the kernel ends.
 constexpr long long WAIT_LIMIT = 4000000000LL;
 
 struct Ctx {
@@ -207,8 +240,11 @@ struct Ctx {
   uint64_t* full;
   uint64_t* empty;
   uint64_t* cbar;
+  uint64_t* xg;    // receives the all-gather of a for a unit (and the head when it uses ablk)
+  uint64_t* xr;    // receives the reduce-scatter partial sums
+  uint64_t* xh;    // receives the head's all-gather, two barriers by step parity
   uint32_t q;      // slab counter (same sequence as the producer)
-  uint32_t cph;    // cluster barrier phase parity
+  uint32_t cph, pg, pr, ph0, ph1;   // phase parities
   int dead;
   int c, tid, warp, lane;
 };
@@ -227,13 +263,22 @@ __device__ __forceinline__ void wait_parity(uint32_t addr, uint32_t parity, bool
   }
 }
 
-// cluster-wide barrier among the compute warps only (the producer warp runs ahead)
+// cluster-wide barrier among the compute warps only (the producer warp runs
+// ahead); used where no data exchange orders a buffer's reuse
 __device__ __forceinline__ void csync(const JobParams& p, Ctx& cx) {
   fence_cluster();
   bar_compute();
   if (cx.tid < p.C) mbar_arrive_cluster(mapa(smem_u32(cx.cbar), cx.tid));
   wait_parity(smem_u32(cx.cbar), cx.cph, true, cx, p.status);
   cx.cph ^= 1u;
+}
+
+// receive one exchange phase of `bytes` on barrier `bar`
+__device__ __forceinline__ void exchange_wait(const JobParams& p, Ctx& cx, uint64_t* bar, uint32_t& parity,
+                                              uint32_t bytes) {
+  if (cx.tid == 0) mbar_arrive_expect_tx(bar, bytes);
+  wait_parity(smem_u32(bar), parity, true, cx, p.status);
+  parity ^= 1u;
 }
 
 __device__ __forceinline__ const uint8_t* ring_acquire(const JobParams& p, Ctx& cx) {
@@ -249,29 +294,23 @@ __device__ __forceinline__ void ring_release(const JobParams& p, Ctx& cx) {
   cx.q++;
 }
 
-// refresh decision for (b, t); identical in the producer and the compute warps
-__device__ __forceinline__ bool refresh_of(const JobParams& p, const uint8_t* S, int b, int t, uint64_t& valid) {
-  const int row = (p.S_rows == p.U) ? b : b / 3;
-  const bool s = S[row * p.T + t] != 0;
-  const bool v = (valid >> b) & 1ull;
-  const bool r = s || (p.force && !v);
-  if (r) valid |= (1ull << b);
-  return r;
-}
-
 __device__ __forceinline__ int piece_K(const JobParams& p, int u, int piece) {
   return piece == 0 ? p.E : (u == 2 ? p.kp_h : p.kp_o);
 }
 
 __device__ __forceinline__ int piece_N(const JobParams& p, int u, int piece) {
-  return piece == 0 ? (u == 0 ? p.n1_sa : (u == 1 ? p.n1_ca : p.n1_ff)) : p.E;
+  return piece == 0 ? p.n1[u] : p.E;
+}
+
+__device__ __forceinline__ int piece_hdr(const JobParams& p, int u, int piece) {
+  return piece == 0 ? p.hdr1[u] : 0;
 }
 
 // ---------------------------------------------------------------------------
 // producer: stream the weight slabs of refreshed units, in schedule order
 // ---------------------------------------------------------------------------
 template <typename T>
-__device__ void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
+__device__ __forceinline__ void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
   uint32_t q = 0;
   for (int job = cid; job < p.n_jobs; job += ncl) {
     const int s0 = min(job * p.g, p.samples - 1);
@@ -279,22 +318,35 @@ __device__ void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl
     uint64_t valid = 0;
     for (int t = 0; t < p.T; ++t) {
       for (int b = 0; b < p.U; ++b) {
-        if (!refresh_of(p, S, b, t, valid)) continue;
+        const int row = (p.S_rows == p.U) ? b : b / 3;
+        const bool vb = (valid >> b) & 1ull;
+        if (!(S[row * p.T + t] != 0 || (p.force && !vb))) continue;   // same rule as the compute warps
+        valid |= 1ull << b;
         const int l = b / 3, u = b % 3;
         for (int piece = 0; piece < 2; ++piece) {
-          const int K = piece_K(p, u, piece), N = piece_N(p, u, piece);
+          const int K = piece_K(p, u, piece), N = piece_N(p, u, piece), hdr = piece_hdr(p, u, piece);
           const uint8_t* src = p.wpack + (long long)cx.c * p.cta_stride + (long long)l * p.layer_stride +
                                p.poff[u][piece];
           const int ktb = N * 16 * (int)sizeof(T);
-          const int kps = max(1, p.slot_bytes / ktb);
           const int nkt = K / 16;
-          for (int kt0 = 0; kt0 < nkt; kt0 += kps) {
-            const uint32_t bytes = (uint32_t)(min(kps, nkt - kt0) * ktb);
+          const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
+          for (int s = 0; s < ns; ++s) {
+            const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
             const uint32_t slot = q % p.nslot;
             const uint32_t ph = (q / p.nslot) & 1u;
-            wait_parity(smem_u32(&cx.empty[slot]), ph ^ 1u, false, cx, p.status);
-            mbar_arrive_expect_tx(&cx.full[slot], bytes);
-            bulk_g2s(cx.smem + p.sm.ring + slot * p.slot_bytes, src + (long long)kt0 * ktb, bytes, &cx.full[slot]);
+            if (!mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
+              // the producer runs ahead of the compute warps: poll gently
+              const long long t0 = clock64();
+              while (!cx.dead && !mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
+                __nanosleep(64);
+                if (clock64() - t0 > WAIT_LIMIT) {
+                  atomicOr(p.status, ST_TIMEOUT);
+                  cx.dead = 1;
+                }
+              }
+            }
+            mbar_arrive_expect_tx(&cx.full[slot], (uint32_t)si.bytes);
+            bulk_g2s(cx.smem + p.sm.ring + slot * p.slot_bytes, src + si.off, (uint32_t)si.bytes, &cx.full[slot]);
             ++q;
           }
         }
@@ -308,40 +360,45 @@ __device__ void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl
 }
 
 // ---------------------------------------------------------------------------
-// GEMM over streamed weight slabs.  A: shared memory, row-major.
+// GEMMs over streamed weight slabs.  A: shared memory, row-major.
+// bf16: warp w owns n-tiles w, w+8, ...; NTW = n-tiles per warp (compile time).
 // ---------------------------------------------------------------------------
-template <int MT>
-__device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda, int K,
-                                          int N, float (&acc)[MT][8][4]) {
+template <int MT, int NTW>
+__device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda, int K, int N,
+                                          int hdr, const uint8_t* slab0, float (&acc)[MT][NTW][4]) {
   const int NT = N >> 3;
-  const int ntw = NT > cx.warp ? (NT - cx.warp + NCW - 1) / NCW : 0;
 #pragma unroll
   for (int m = 0; m < MT; ++m)
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < NTW; ++i)
 #pragma unroll
       for (int r = 0; r < 4; ++r) acc[m][i][r] = 0.f;
   const int ktb = N * 32;
-  const int kps = max(1, p.slot_bytes / ktb);
   const int nkt = K >> 4;
-  for (int kt0 = 0; kt0 < nkt; kt0 += kps) {
-    const uint8_t* slab = ring_acquire(p, cx);
-    const int nk = min(kps, nkt - kt0);
-    for (int kk = 0; kk < nk; ++kk) {
+  const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
+  const __nv_bfloat16* arow = A + (cx.lane & 15) * lda + (cx.lane >> 4) * 8;
+  for (int s = 0; s < ns; ++s) {
+    const uint8_t* sl = s == 0 ? slab0 : ring_acquire(p, cx);
+    const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
+    const uint8_t* wt = sl + (s == 0 ? hdr : 0) + cx.lane * 8;
+#pragma unroll 2
+    for (int kk = 0; kk < si.nkt; ++kk) {
+      const int kt = si.kt0 + kk;
       uint32_t a[MT][4];
 #pragma unroll
-      for (int m = 0; m < MT; ++m)
-        ldmatrix_x4(a[m], A + (m * 16 + (cx.lane & 15)) * lda + (kt0 + kk) * 16 + (cx.lane >> 4) * 8);
-      const uint8_t* base = slab + (size_t)kk * NT * 256 + cx.lane * 8;
+      for (int m = 0; m < MT; ++m) ldmatrix_x4(a[m], arow + m * 16 * lda + kt * 16);
+      uint2 bf[NTW];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (i < ntw) {
-          const int nt = cx.warp + i * NCW;
-          const uint2 bf = *reinterpret_cast<const uint2*>(base + nt * 256);
-#pragma unroll
-          for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], a[m], bf);
-        }
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        bf[i] = nt < NT ? *reinterpret_cast<const uint2*>(wt + (size_t)(kk * NT + nt) * 256) : make_uint2(0u, 0u);
       }
+#pragma unroll
+      for (int i = 0; i < NTW; ++i)
+        if (cx.warp + i * NCW < NT) {
+#pragma unroll
+          for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], a[m], bf[i]);
+        }
     }
     ring_release(p, cx);
   }
@@ -350,7 +407,7 @@ __device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __n
 constexpr int F32_MAXO = 16;
 
 __device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const float* A, int lda, int K, int M, int N,
-                                         float (&acc)[F32_MAXO]) {
+                                         int hdr, const uint8_t* slab0, float (&acc)[F32_MAXO]) {
   int mi[F32_MAXO], ni[F32_MAXO];
   const int nout = M * N;
 #pragma unroll
@@ -361,13 +418,15 @@ __device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const floa
     acc[i] = 0.f;
   }
   const int ktb = N * 64;
-  const int kps = max(1, p.slot_bytes / ktb);
   const int nkt = K >> 4;
-  for (int kt0 = 0; kt0 < nkt; kt0 += kps) {
-    const float* W = reinterpret_cast<const float*>(ring_acquire(p, cx));
-    const int rows = min(kps, nkt - kt0) * 16;
+  const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
+  for (int s = 0; s < ns; ++s) {
+    const uint8_t* sl = s == 0 ? slab0 : ring_acquire(p, cx);
+    const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
+    const float* W = reinterpret_cast<const float*>(sl + (s == 0 ? hdr : 0));
+    const int rows = si.nkt * 16;
     for (int r = 0; r < rows; ++r) {
-      const int k = kt0 * 16 + r;
+      const int k = si.kt0 * 16 + r;
 #pragma unroll
       for (int i = 0; i < F32_MAXO; ++i)
         if (cx.tid + i * NCT < nout) acc[i] = fmaf(A[mi[i] * lda + k], W[r * N + ni[i]], acc[i]);
@@ -380,50 +439,67 @@ __device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const floa
 // compute-warp building blocks
 // ---------------------------------------------------------------------------
 
-// write this CTA's columns of a into the [M][ldf] buffer `dst` of every CTA of the cluster
-__device__ __forceinline__ void gather_rows(const JobParams& p, Ctx& cx, const float* ac, float* dst) {
-  const uint32_t base = smem_u32(dst);
-  const int nvec = p.M * p.Ec / 4;
-  for (int v = cx.tid; v < nvec * p.C; v += NCT) {
-    const int r = v / nvec;
-    const int e = (v - r * nvec) * 4;
-    const int m = e / p.Ec, j = e - m * p.Ec;
-    const float4 val = *reinterpret_cast<const float4*>(ac + e);
-    st_cluster_v4(mapa(base + (uint32_t)((m * p.ldf + cx.c * p.Ec + j) * 4), (uint32_t)r), val);
+// Send one block of M*Ec floats to every CTA r of the cluster: block
+// src + r*src_stride lands in CTA r at dst + c*blk (c = this CTA), counted on
+// r's barrier `rbar`.  The writers of src have executed fence_proxy_async()
+// and a bar_compute() before this call.
+__device__ __forceinline__ void send_blocks(const JobParams& p, Ctx& cx, const float* src, int src_stride,
+                                            const float* dst, uint64_t* rbar) {
+  if (cx.tid < p.C) {
+    const uint32_t r = (uint32_t)cx.tid;
+    bulk_s2c(mapa(smem_u32(dst + cx.c * p.blk), r), src + r * src_stride, (uint32_t)(p.M * p.Ec * 4),
+             mapa(smem_u32(rbar), r));
   }
 }
 
-// LayerNorm of full rows m < M of `buf` in place: the row is overwritten by
-// its normalised values in type T (row stride in T elements = ldf * 4 / sizeof(T)).
+// LayerNorm of rows m < M (half a warp per row).  Row m is read from the
+// gathered blocks (column col of the row is in block col/Ec) and written to the
+// A operand xln in type T.
 template <typename T>
-__device__ __forceinline__ void layernorm_inplace(const JobParams& p, Ctx& cx, float* buf, const float (&g)[16],
-                                                  const float (&bt)[16]) {
-  const int nper = p.E >> 5;
-  for (int m = cx.warp; m < p.M; m += NCW) {
-    float* row = buf + m * p.ldf;
-    float v[16];
+__device__ __forceinline__ void layernorm_rows(const JobParams& p, Ctx& cx, const float* blk, T* xln,
+                                               const float* gam, const float* bet) {
+  const int half = cx.lane >> 4, hl = cx.lane & 15;
+  const int nv = p.E >> 6;                      // float4 chunks per lane
+  for (int m0 = 0; m0 < p.M; m0 += 2 * NCW) {
+    if (m0 + cx.warp * 2 >= p.M) break;           // warp-uniform (M is even)
+    const int m = m0 + cx.warp * 2 + half;
+    float4 v[8];
     float s = 0.f;
 #pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (j < nper) {
-        v[j] = row[cx.lane + 32 * j];
-        s += v[j];
+    for (int j = 0; j < 8; ++j)
+      if (j < nv) {
+        const int col = 4 * (hl + 16 * j);
+        v[j] = *reinterpret_cast<const float4*>(blk + (col >> p.lEc) * p.blk + (m << p.lEc) + (col & (p.Ec - 1)));
+        s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
       }
-    const float mean = warp_sum(s) / p.E;
+    const float mean = group_sum<16>(s) / p.E;
     float s2 = 0.f;
 #pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (j < nper) {
-        const float d = v[j] - mean;
-        s2 += d * d;
+    for (int j = 0; j < 8; ++j)
+      if (j < nv) {
+        const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
+        s2 += (a * a + b * b) + (c * c + d * d);
       }
-    const float rstd = 1.0f / sqrtf(warp_sum(s2) / p.E + 1e-5f);
-    __syncwarp();
-    T* out = reinterpret_cast<T*>(row);
+    const float rstd = 1.0f / sqrtf(group_sum<16>(s2) / p.E + 1e-5f);
 #pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (j < nper) out[cx.lane + 32 * j] = from_f<T>((v[j] - mean) * rstd * g[j] + bt[j]);
-    __syncwarp();
+    for (int j = 0; j < 8; ++j)
+      if (j < nv) {
+        const int col = 4 * (hl + 16 * j);
+        const float4 g = *reinterpret_cast<const float4*>(gam + col);
+        const float4 bb = *reinterpret_cast<const float4*>(bet + col);
+        const float y0 = (v[j].x - mean) * rstd * g.x + bb.x, y1 = (v[j].y - mean) * rstd * g.y + bb.y;
+        const float y2 = (v[j].z - mean) * rstd * g.z + bb.z, y3 = (v[j].w - mean) * rstd * g.w + bb.w;
+        T* dst = xln + m * p.lda + col;
+        if constexpr (sizeof(T) == 2) {
+          __nv_bfloat162 lo = __floats2bfloat162_rn(y0, y1), hi = __floats2bfloat162_rn(y2, y3);
+          uint2 pk;
+          pk.x = *reinterpret_cast<uint32_t*>(&lo);
+          pk.y = *reinterpret_cast<uint32_t*>(&hi);
+          *reinterpret_cast<uint2*>(dst) = pk;
+        } else {
+          *reinterpret_cast<float4*>(dst) = make_float4(y0, y1, y2, y3);
+        }
+      }
   }
 }
 
@@ -431,51 +507,86 @@ template <typename T>
 struct Kern {
   static constexpr bool BF = sizeof(T) == 2;
 
-  // ---- first GEMM epilogues ------------------------------------------------
-  // SA / CA: f32 rows of q|k|v (SA) or q (CA) + bias;  FFN: T(gelu(. + bias))
-  template <int MT>
-  __device__ static void gemm1(const JobParams& p, Ctx& cx, int u, const float* bias) {
-    float* xbuf = reinterpret_cast<float*>(cx.smem + p.sm.afull);
-    const int N = u == 0 ? p.n1_sa : (u == 1 ? p.n1_ca : p.n1_ff);
-    float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.g1);
-    T* hid = reinterpret_cast<T*>(cx.smem + p.sm.g1);
-    if constexpr (BF) {
-      float acc[MT][8][4];
-      gemm_bf16<MT>(p, cx, reinterpret_cast<const __nv_bfloat16*>(xbuf), p.ldf * 2, p.E, N, acc);
-      const int NT = N >> 3;
+  __device__ __forceinline__ static T* cache_ptr(const JobParams& p, Ctx& cx, int job, int b) {
+    if (p.sm.cs >= 0) return reinterpret_cast<T*>(cx.smem + p.sm.cs) + (long long)b * p.M * p.Ec;
+    return reinterpret_cast<T*>(p.cache) + ((long long)(job * p.U + b) * p.C + cx.c) * p.M * p.Ec;
+  }
+
+  // ---- first GEMM + epilogue ------------------------------------------------
+  // A = xln.  SA / CA: f32 rows of q|k|v (SA) or q (CA) + bias; FFN:
+  // T(gelu(. + bias)).  The output region aliases xln, so all warps finish
+  // their k-loop before any epilogue writes.
+  template <int MT, int NTW>
+  __device__ __forceinline__ static void gemm1_t(const JobParams& p, Ctx& cx, int u, const uint8_t* slab0) {
+    const T* xln = reinterpret_cast<const T*>(cx.smem + p.sm.xln);
+    const int N = p.n1[u];
+    const float* bias = reinterpret_cast<const float*>(slab0) + 2 * p.E;
+    float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.xln);
+    T* hid = reinterpret_cast<T*>(cx.smem + p.sm.xln);
+    const int NT = N >> 3;
+    float2 bv[NTW];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (nt < NT) {
-          const int n = nt * 8 + 2 * (cx.lane & 3);
-          const float b0 = __ldg(bias + n), b1 = __ldg(bias + n + 1);
+    for (int i = 0; i < NTW; ++i) {
+      const int nt = cx.warp + i * NCW;
+      bv[i] = nt < NT ? *reinterpret_cast<const float2*>(bias + nt * 8 + 2 * (cx.lane & 3)) : make_float2(0.f, 0.f);
+    }
+    float acc[MT][NTW][4];
+    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(xln), p.lda, p.E, N, p.hdr1[u], slab0, acc);
+    bar_compute();
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt)
+    for (int i = 0; i < NTW; ++i) {
+      const int nt = cx.warp + i * NCW;
+      if (nt < NT) {
+        const int n = nt * 8 + 2 * (cx.lane & 3);
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
-              if (m < p.M) {
-                const float v0 = acc[mt][i][2 * h] + b0, v1 = acc[mt][i][2 * h + 1] + b1;
-                if (u == 2) {
-                  hid[m * p.ldh + n] = from_f<T>(gelu_erf(v0));
-                  hid[m * p.ldh + n + 1] = from_f<T>(gelu_erf(v1));
-                } else {
-                  g1[m * p.ldg1 + n] = v0;
-                  g1[m * p.ldg1 + n + 1] = v1;
-                }
+        for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
+            if (m < p.M) {
+              const float v0 = acc[mt][i][2 * h] + bv[i].x, v1 = acc[mt][i][2 * h + 1] + bv[i].y;
+              if (u == 2) {
+                *reinterpret_cast<__nv_bfloat162*>(hid + m * p.ldh + n) =
+                    __floats2bfloat162_rn(gelu_erf(v0), gelu_erf(v1));
+              } else {
+                *reinterpret_cast<float2*>(g1 + m * p.ldg1 + n) = make_float2(v0, v1);
               }
             }
-        }
+          }
       }
+    }
+  }
+
+  template <int MT>
+  __device__ __forceinline__ static void gemm1(const JobParams& p, Ctx& cx, int u, const uint8_t* slab0) {
+    if constexpr (BF) {
+      const int ntw = ((p.n1[u] >> 3) + NCW - 1) / NCW;
+      if (ntw <= 1) gemm1_t<MT, 1>(p, cx, u, slab0);
+      else if (ntw == 2) gemm1_t<MT, 2>(p, cx, u, slab0);
+      else if (ntw == 3) gemm1_t<MT, 3>(p, cx, u, slab0);
+      else if (ntw == 4) gemm1_t<MT, 4>(p, cx, u, slab0);
+      else gemm1_t<MT, 8>(p, cx, u, slab0);
     } else {
+      const float* xln = reinterpret_cast<const float*>(cx.smem + p.sm.xln);
+      const int N = p.n1[u];
+      const float* bias = reinterpret_cast<const float*>(slab0) + 2 * p.E;
+      float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.xln);
+      T* hid = reinterpret_cast<T*>(cx.smem + p.sm.xln);
+      float bv[F32_MAXO];
+#pragma unroll
+      for (int i = 0; i < F32_MAXO; ++i) {
+        const int o = cx.tid + i * NCT;
+        bv[i] = o < p.M * N ? bias[o % N] : 0.f;
+      }
       float acc[F32_MAXO];
-      gemm_f32(p, cx, xbuf, p.ldf, p.E, p.M, N, acc);
+      gemm_f32(p, cx, xln, p.lda, p.E, p.M, N, p.hdr1[u], slab0, acc);
+      bar_compute();
 #pragma unroll
       for (int i = 0; i < F32_MAXO; ++i) {
         const int o = cx.tid + i * NCT;
         if (o < p.M * N) {
           const int m = o / N, n = o % N;
-          const float v = acc[i] + __ldg(bias + n);
+          const float v = acc[i] + bv[i];
           if (u == 2)
             hid[m * p.ldh + n] = from_f<T>(gelu_erf(v));
           else
@@ -485,271 +596,382 @@ struct Kern {
     }
   }
 
-  // ---- second GEMM: partial sums over this CTA's K slice, reduce-scattered
-  template <int MT>
-  __device__ static void gemm2(const JobParams& p, Ctx& cx, int u) {
-    const T* A = reinterpret_cast<const T*>(cx.smem + (u == 2 ? p.sm.g1 : p.sm.oc));
+  // ---- second GEMM: partial sums over this CTA's K slice, staged in ablk
+  // block layout (block r = columns r*Ec.. destined for CTA r)
+  template <int MT, int NTW>
+  __device__ __forceinline__ static void gemm2_t(const JobParams& p, Ctx& cx, int u) {
+    const T* A = reinterpret_cast<const T*>(cx.smem + (u == 2 ? p.sm.xln : p.sm.oc));
     const int lda = u == 2 ? p.ldh : p.ldo;
     const int K = u == 2 ? p.kp_h : p.kp_o;
-    const uint32_t rs = smem_u32(cx.smem + p.sm.rs);
-    if constexpr (BF) {
-      float acc[MT][8][4];
-      gemm_bf16<MT>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, K, p.E, acc);
-      const int NT = p.E >> 3;
+    float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
+    float acc[MT][NTW][4];
+    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, K, p.E, 0, ring_acquire(p, cx), acc);
+    const int NT = p.E >> 3;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (nt < NT) {
-          const int n = nt * 8 + 2 * (cx.lane & 3);
-          const int r = n / p.Ec, jj = n - r * p.Ec;
+    for (int i = 0; i < NTW; ++i) {
+      const int nt = cx.warp + i * NCW;
+      if (nt < NT) {
+        const int n = nt * 8 + 2 * (cx.lane & 3);
+        float* dst = stage + (n >> p.lEc) * p.blk + (n & (p.Ec - 1));
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt)
+        for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
-              if (m < p.M)
-                st_cluster_v2(mapa(rs + (uint32_t)(((cx.c * p.M + m) * p.Ec + jj) * 4), (uint32_t)r),
-                              acc[mt][i][2 * h], acc[mt][i][2 * h + 1]);
-            }
-        }
+          for (int h = 0; h < 2; ++h) {
+            const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
+            if (m < p.M)
+              *reinterpret_cast<float2*>(dst + (m << p.lEc)) = make_float2(acc[mt][i][2 * h], acc[mt][i][2 * h + 1]);
+          }
       }
+    }
+  }
+
+  template <int MT>
+  __device__ __forceinline__ static void gemm2(const JobParams& p, Ctx& cx, int u) {
+    if constexpr (BF) {
+      const int ntw = ((p.E >> 3) + NCW - 1) / NCW;
+      if (ntw <= 1) gemm2_t<MT, 1>(p, cx, u);
+      else if (ntw == 2) gemm2_t<MT, 2>(p, cx, u);
+      else if (ntw <= 4) gemm2_t<MT, 4>(p, cx, u);
+      else gemm2_t<MT, 8>(p, cx, u);
     } else {
+      const T* A = reinterpret_cast<const T*>(cx.smem + (u == 2 ? p.sm.xln : p.sm.oc));
+      const int lda = u == 2 ? p.ldh : p.ldo;
+      const int K = u == 2 ? p.kp_h : p.kp_o;
+      float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
       float acc[F32_MAXO];
-      gemm_f32(p, cx, reinterpret_cast<const float*>(A), lda, K, p.M, p.E, acc);
+      gemm_f32(p, cx, reinterpret_cast<const float*>(A), lda, K, p.M, p.E, 0, ring_acquire(p, cx), acc);
 #pragma unroll
       for (int i = 0; i < F32_MAXO; ++i) {
         const int o = cx.tid + i * NCT;
         if (o < p.M * p.E) {
           const int m = o / p.E, n = o % p.E;
-          const int r = n / p.Ec, jj = n - r * p.Ec;
-          st_cluster_f32(mapa(rs + (uint32_t)(((cx.c * p.M + m) * p.Ec + jj) * 4), (uint32_t)r), acc[i]);
+          stage[(n >> p.lEc) * p.blk + (m << p.lEc) + (n & (p.Ec - 1))] = acc[i];
         }
       }
     }
   }
 
   // ---- attention for this CTA's head-dimension slice ------------------------
-  // SA: causal over the H tokens of the same sample; q, k of the CTA's head and
-  // v of its slice are in g1.  CA: keys/values of the memory tokens in kvs.
-  __device__ static void attention(const JobParams& p, Ctx& cx, int u) {
-    const float* g1 = reinterpret_cast<const float*>(cx.smem + p.sm.g1);
-    const float* kvs = reinterpret_cast<const float*>(cx.smem + p.sm.kvs);
+  // scores: one (query row, key) pair per thread, softmax over groups of G
+  // lanes, probabilities to pb; then one output (row, dim) per thread.
+  // SA: causal over the H tokens of the same sample (q, k of the CTA's head and
+  // v of its slice, rows of the first GEMM's output).  CA: the 1 + n_obs memory
+  // tokens in kvs.
+  __device__ __forceinline__ static void attention(const JobParams& p, Ctx& cx, int u, const float* kvs) {
+    const float* g1 = reinterpret_cast<const float*>(cx.smem + p.sm.xln);
+    float* pb = reinterpret_cast<float*>(cx.smem + p.sm.pb);
     T* oc = reinterpret_cast<T*>(cx.smem + p.sm.oc);
     const float scale = 1.0f / sqrtf((float)p.dh);
-    const int kvw = p.dh + p.Ec;
-    for (int m = cx.warp; m < p.M; m += NCW) {
-      const int i = m / p.H, qi = m - i * p.H;
-      const float* q = g1 + m * p.ldg1;
-      const int nkey = u == 0 ? qi + 1 : p.Cm;
+    const int nk = u == 0 ? p.H : p.Cm;
+    int G = 1;
+    while (G < nk) G <<= 1;
+    const int rows_per_pass = NCT / G;
+    const int nd4 = p.dh >> 2;
+    for (int base = 0; base < p.M; base += rows_per_pass) {
+      const int m = base + cx.tid / G, j = cx.tid % G;
       float s = -INFINITY;
-      if (cx.lane < nkey) {
-        const float* kr = u == 0 ? g1 + (i * p.H + cx.lane) * p.ldg1 + p.dh : kvs + (i * p.Cm + cx.lane) * kvw;
-        float d = 0.f;
-        for (int e = 0; e < p.dh; ++e) d = fmaf(q[e], kr[e], d);
-        s = d * scale;
+      const bool live = m < p.M && j < nk;
+      if (live) {
+        const int i = m >> p.lH, qi = m & (p.H - 1);
+        if (u != 0 || j <= qi) {
+          const float4* q4 = reinterpret_cast<const float4*>(g1 + m * p.ldg1);
+          const float4* k4 = u == 0 ? reinterpret_cast<const float4*>(g1 + ((i << p.lH) + j) * p.ldg1 + p.dh)
+                                    : reinterpret_cast<const float4*>(kvs + (i * p.Cm + j) * p.kvw);
+          float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll 4
+          for (int e = 0; e < nd4; ++e) {
+            const float4 a = q4[e], b = k4[e];
+            d0 = fmaf(a.x, b.x, d0);
+            d1 = fmaf(a.y, b.y, d1);
+            d2 = fmaf(a.z, b.z, d2);
+            d3 = fmaf(a.w, b.w, d3);
+          }
+          s = ((d0 + d1) + (d2 + d3)) * scale;
+        }
       }
-      const float mx = warp_max(s);
-      const float pj = cx.lane < nkey ? expf(s - mx) : 0.f;
-      const float inv = 1.0f / warp_sum(pj);
-      float o0 = 0.f, o1 = 0.f;
-      for (int j = 0; j < nkey; ++j) {
-        const float pb = __shfl_sync(0xffffffffu, pj, j);
-        const float* vr = u == 0 ? g1 + (i * p.H + j) * p.ldg1 + 2 * p.dh : kvs + (i * p.Cm + j) * kvw + p.dh;
-        if (cx.lane < p.Ec) o0 = fmaf(pb, vr[cx.lane], o0);
-        if (cx.lane + 32 < p.Ec) o1 = fmaf(pb, vr[cx.lane + 32], o1);
+      const float mx = group_max_dyn(s, G);
+      const float ex = s == -INFINITY ? 0.f : expf(s - mx);
+      const float sum = group_sum_dyn(ex, G);
+      if (live) pb[m * PLD + j] = ex / sum;
+    }
+    bar_compute();
+    for (int o = cx.tid; o < p.M * p.Ec; o += NCT) {
+      const int m = o >> p.lEc, e = o & (p.Ec - 1);
+      const int i = m >> p.lH, qi = m & (p.H - 1);
+      const int nj = u == 0 ? qi + 1 : p.Cm;
+      const float* prow = pb + m * PLD;
+      float a0 = 0.f, a1 = 0.f;
+      int j = 0;
+      if (u == 0) {
+        const float* v = g1 + (i << p.lH) * p.ldg1 + 2 * p.dh + e;
+        for (; j + 1 < nj; j += 2) {
+          a0 = fmaf(prow[j], v[j * p.ldg1], a0);
+          a1 = fmaf(prow[j + 1], v[(j + 1) * p.ldg1], a1);
+        }
+        if (j < nj) a0 = fmaf(prow[j], v[j * p.ldg1], a0);
+      } else {
+        const float* v = kvs + (i * p.Cm) * p.kvw + p.dh + e;
+        for (; j < nj; ++j) a0 = fmaf(prow[j], v[j * p.kvw], a0);
       }
-      if (cx.lane < p.Ec) oc[m * p.ldo + cx.lane] = from_f<T>(o0 * inv);
-      if (cx.lane + 32 < p.Ec) oc[m * p.ldo + cx.lane + 32] = from_f<T>(o1 * inv);
+      oc[m * p.ldo + e] = from_f<T>(a0 + a1);
+    }
+  }
+
+  // stage the memory tokens' keys (this CTA's head) and values (its slice) of
+  // layer l at step t into kvs (cp.async; waited before use)
+  __device__ __forceinline__ static void stage_kv(const JobParams& p, Ctx& cx, int l, int t, int sample0, float* kvs) {
+    const int h = (cx.c * p.Ec) / p.dh;
+    const int kq = p.dh / 4, vq = p.Ec / 4;
+    const int per_tok = kq + vq;
+    const int total = p.g * p.Cm * per_tok;
+    for (int v = cx.tid; v < total; v += NCT) {
+      const int i = v / (p.Cm * per_tok);
+      const int rem = v - i * p.Cm * per_tok;
+      const int tok = rem / per_tok, w = rem - tok * per_tok;
+      const int s = min(sample0 + i, p.samples - 1);
+      const float* src = tok == 0 ? p.kv_time + ((long long)t * p.L + l) * 2 * p.E
+                                  : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (tok - 1)) * p.L + l) * 2 * p.E;
+      const float* s4 = w < kq ? src + h * p.dh + 4 * w : src + p.E + cx.c * p.Ec + 4 * (w - kq);
+      float* d4 = kvs + (i * p.Cm + tok) * p.kvw + (w < kq ? 4 * w : p.dh + 4 * (w - kq));
+      cp_async16(d4, s4);
     }
   }
 
   // ---- one refreshed unit (Eq. 1, (b,t) in S) --------------------------------
   template <int MT>
-  __device__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0) {
+  __device__ __forceinline__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0) {
     const int l = b / 3, u = b % 3;
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
-    float* afull = reinterpret_cast<float*>(cx.smem + p.sm.afull);
-    // prefetch LayerNorm parameters (lane-strided columns) and the finishing bias
-    float gam[16], bet[16];
-    const float* lnv = p.vec + p.v_ln + (long long)b * 2 * p.E;
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (j < (p.E >> 5)) {
-        gam[j] = __ldg(lnv + cx.lane + 32 * j);
-        bet[j] = __ldg(lnv + p.E + cx.lane + 32 * j);
-      }
-    // cross-attention: stage the memory tokens' keys (this head) and values (this slice)
+    float* ablk = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
+    float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
     if (u == 1) {
-      float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
-      const int kvw = p.dh + p.Ec;
-      const int h = (cx.c * p.Ec) / p.dh;
-      const int kq = p.dh / 4, vq = p.Ec / 4;
-      const int per_tok = kq + vq;
-      const int total = p.g * p.Cm * per_tok;
-      for (int v = cx.tid; v < total; v += NCT) {
-        const int i = v / (p.Cm * per_tok);
-        const int rem = v - i * p.Cm * per_tok;
-        const int tok = rem / per_tok, w = rem - tok * per_tok;
-        const int s = min(sample0 + i, p.samples - 1);
-        const float* src = tok == 0 ? p.kv_time + ((long long)t * p.L + l) * 2 * p.E
-                                    : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (tok - 1)) * p.L + l) * 2 * p.E;
-        const float* s4 = w < kq ? src + h * p.dh + 4 * w : src + p.E + cx.c * p.Ec + 4 * (w - kq);
-        float* d4 = kvs + (i * p.Cm + tok) * kvw + (w < kq ? 4 * w : p.dh + 4 * (w - kq));
-        cp_async16(d4, s4);
-      }
+      if (p.kv_slots == 1) stage_kv(p, cx, l, t, sample0, kvs);
+      else kvs += l * p.g * p.Cm * p.kvw;
     }
+    // exchange 1: every CTA receives every CTA's columns of a
+    fence_proxy_async();
     bar_compute();                     // ac final for this unit
-    gather_rows(p, cx, ac, afull);
-    csync(p, cx);                      // exchange 1: full rows of a everywhere
-    layernorm_inplace<T>(p, cx, afull, gam, bet);
+    send_blocks(p, cx, ac, 0, ablk, cx.xg);
+    exchange_wait(p, cx, cx.xg, cx.pg, (uint32_t)(p.M * p.E * 4));
+    // slab 0 of piece 1: [gamma | beta | first bias | second-GEMM bias slice | k-tiles]
+    const uint8_t* s1 = ring_acquire(p, cx);
+    const float* hdr = reinterpret_cast<const float*>(s1);
+    float b2[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = cx.tid + k * NCT;
+      b2[k] = e < p.M * p.Ec ? hdr[2 * p.E + p.n1[u] + (e & (p.Ec - 1))] : 0.f;
+    }
+    layernorm_rows<T>(p, cx, ablk, reinterpret_cast<T*>(cx.smem + p.sm.xln), hdr, hdr + p.E);
+    bar_compute();
+    gemm1<MT>(p, cx, u, s1);
     if (u == 1) cp_async_wait_all();
     bar_compute();
-    gemm1<MT>(p, cx, u, p.vec + p.v_b1 + ((long long)b * p.C + cx.c) * p.n1max);
-    bar_compute();
     if (u != 2) {
-      attention(p, cx, u);
+      attention(p, cx, u, kvs);
       bar_compute();
     }
     gemm2<MT>(p, cx, u);
-    csync(p, cx);                      // exchange 2: partial sums landed
+    // exchange 2: block r of the staged partial sums goes to CTA r
+    fence_proxy_async();
+    bar_compute();
+    send_blocks(p, cx, ablk, p.blk, reinterpret_cast<const float*>(cx.smem + p.sm.rs), cx.xr);
+    exchange_wait(p, cx, cx.xr, cx.pr, (uint32_t)(p.M * p.E * 4));
     // finish this CTA's columns: r = sum of partials + bias; c_b <- r; a += r
     const float* rs = reinterpret_cast<const float*>(cx.smem + p.sm.rs);
-    T* cache = reinterpret_cast<T*>(p.cache) + ((long long)(job * p.U + b) * p.C + cx.c) * p.M * p.Ec;
-    const float* b2 = p.vec + p.v_b2 + (long long)b * p.E + cx.c * p.Ec;
-    for (int e = cx.tid; e < p.M * p.Ec; e += NCT) {
-      const int m = e / p.Ec, j = e - m * p.Ec;
-      float r = 0.f;
-      for (int cc = 0; cc < p.C; ++cc) r += rs[(cc * p.M + m) * p.Ec + j];
-      r += __ldg(b2 + j);
-      cache[e] = from_f<T>(r);
-      ac[e] += r;
-      if (p.trace) {
-        const int s = sample0 + m / p.H;
-        if (s < p.samples)
-          p.trace[(((long long)t * p.U + b) * p.samples + s) * p.H * p.E + (m % p.H) * p.E + cx.c * p.Ec + j] = r;
+    T* cache = cache_ptr(p, cx, job, b);
+    const int MEc = p.M * p.Ec;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e = cx.tid + k * NCT;
+      if (e < MEc) {
+        float r0 = 0.f, r1 = 0.f;
+        int cc = 0;
+        for (; cc + 1 < p.C; cc += 2) {
+          r0 += rs[cc * p.blk + e];
+          r1 += rs[(cc + 1) * p.blk + e];
+        }
+        if (cc < p.C) r0 += rs[cc * p.blk + e];
+        const float r = (r0 + r1) + b2[k];
+        cache[e] = from_f<T>(r);
+        ac[e] += r;
+        if (p.trace) {
+          const int m = e >> p.lEc, j = e & (p.Ec - 1);
+          const int s = sample0 + (m >> p.lH);
+          if (s < p.samples)
+            p.trace[(((long long)t * p.U + b) * p.samples + s) * p.H * p.E + (m & (p.H - 1)) * p.E + cx.c * p.Ec + j] = r;
+        }
       }
     }
   }
 
-  // ---- skipped unit: a += c_b on this CTA's columns ----------------------------
-  __device__ static void skip_add(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0, bool valid) {
+  // ---- skipped units b0..b1-1: a += c_b on this CTA's columns (in unit order) ---
+  __device__ __forceinline__ static void skip_run(const JobParams& p, Ctx& cx, int job, int b0, int b1, int t,
+                                                  int sample0, uint64_t valid) {
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
-    const T* cache = reinterpret_cast<const T*>(p.cache) + ((long long)(job * p.U + b) * p.C + cx.c) * p.M * p.Ec;
-    for (int e = cx.tid; e < p.M * p.Ec; e += NCT) {
-      const float cv = valid ? to_f<T>(cache[e]) : 0.f;
-      if (valid) ac[e] += cv;
+    const int MEc = p.M * p.Ec;
+    for (int e = cx.tid; e < MEc; e += NCT) {
+      float cv[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        cv[k] = (b0 + k < b1 && ((valid >> (b0 + k)) & 1ull)) ? to_f<T>(cache_ptr(p, cx, job, b0 + k)[e]) : 0.f;
+      float a = ac[e];
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (b0 + k < b1 && ((valid >> (b0 + k)) & 1ull)) a += cv[k];
+      ac[e] = a;
       if (p.trace) {
-        const int m = e / p.Ec, j = e - m * p.Ec;
-        const int s = sample0 + m / p.H;
-        if (s < p.samples)
-          p.trace[(((long long)t * p.U + b) * p.samples + s) * p.H * p.E + (m % p.H) * p.E + cx.c * p.Ec + j] = cv;
+        const int m = e >> p.lEc, j = e & (p.Ec - 1);
+        const int s = sample0 + (m >> p.lH);
+        if (s < p.samples) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            if (b0 + k < b1)
+              p.trace[(((long long)t * p.U + b0 + k) * p.samples + s) * p.H * p.E + (m & (p.H - 1)) * p.E +
+                      cx.c * p.Ec + j] = cv[k];
+        }
       }
     }
   }
 
   // ---- output head + sampler step ---------------------------------------------
-  __device__ static void head_step(const JobParams& p, Ctx& cx, int t, bool any_refresh, const float (&gf)[16],
-                                   const float (&bf)[16]) {
+  __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t, const float4 tab0,
+                                                   const float4 tab1) {
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
-    float* hb = reinterpret_cast<float*>(cx.smem + (p.head_sep ? p.sm.hbuf : p.sm.afull));
     float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
     const float* z = reinterpret_cast<const float*>(cx.smem + p.sm.z);
-    if (p.head_sep && !any_refresh) csync(p, cx);   // previous head's readers are done with hbuf
-    bar_compute();
-    gather_rows(p, cx, ac, hb);
-    csync(p, cx);
+    const float* cst = reinterpret_cast<const float*>(cx.smem + p.sm.cst);
+    const float* lnf_g = cst + p.A * p.Ec + p.Ec + p.H * p.Ec;
+    const float* lnf_b = lnf_g + p.E;
+    const float* head_b = lnf_b + p.E;
+    const float* hw = p.headw_smem ? head_b + ((p.A + 3) & ~3) : p.vec + p.v_headw;
+    const float* hb;
+    if (p.head_sep) {
+      // double-buffered by step parity: source, landing blocks and barrier
+      const int par = t & 1;
+      float* src = reinterpret_cast<float*>(cx.smem + p.sm.hsrc) + par * p.M * p.Ec;
+      for (int e = cx.tid; e < p.M * p.Ec; e += NCT) src[e] = ac[e];
+      hb = reinterpret_cast<const float*>(cx.smem + p.sm.hblk) + par * p.C * p.blk;
+      fence_proxy_async();
+      bar_compute();
+      send_blocks(p, cx, src, 0, hb, cx.xh + par);
+      exchange_wait(p, cx, cx.xh + par, par ? cx.ph1 : cx.ph0, (uint32_t)(p.M * p.E * 4));
+    } else {
+      hb = reinterpret_cast<const float*>(cx.smem + p.sm.ablk);
+      fence_proxy_async();
+      bar_compute();
+      send_blocks(p, cx, ac, 0, hb, cx.xg);
+      exchange_wait(p, cx, cx.xg, cx.pg, (uint32_t)(p.M * p.E * 4));
+    }
     cp_async_wait_all();
     bar_compute();
-    const float* tab = p.stab + t * 8;
-    const float inv_sa = tab[0], s1 = tab[1], cx0 = tab[2], cxt = tab[3], sig = tab[4];
-    const float sab = tab[5], sabp = tab[6], s1p = tab[7];
-    const int nper = p.E >> 5;
-    const float* hw = p.vec + p.v_headw;
-    for (int m = cx.warp; m < p.M; m += NCW) {
-      const float* row = hb + m * p.ldf;
-      float v[16];
+    const float inv_sa = tab0.x, s1 = tab0.y, cx0 = tab0.z, cxt = tab0.w, sig = tab1.x;
+    const float sab = tab1.y, sabp = tab1.z, s1p = tab1.w;
+    const int half = cx.lane >> 4, hl = cx.lane & 15;
+    const int nv = p.E >> 6;
+    for (int m0 = 0; m0 < p.M; m0 += 2 * NCW) {
+      if (m0 + cx.warp * 2 >= p.M) break;
+      const int m = m0 + cx.warp * 2 + half;
+      float4 v[8];
       float s = 0.f;
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (j < nper) {
-          v[j] = row[cx.lane + 32 * j];
-          s += v[j];
+      for (int j = 0; j < 8; ++j)
+        if (j < nv) {
+          const int col = 4 * (hl + 16 * j);
+          v[j] = *reinterpret_cast<const float4*>(hb + (col >> p.lEc) * p.blk + (m << p.lEc) + (col & (p.Ec - 1)));
+          s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
         }
-      const float mean = warp_sum(s) / p.E;
+      const float mean = group_sum<16>(s) / p.E;
       float s2 = 0.f;
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (j < nper) {
-          const float d = v[j] - mean;
-          s2 += d * d;
+      for (int j = 0; j < 8; ++j)
+        if (j < nv) {
+          const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
+          s2 += (a * a + b * b) + (c * c + d * d);
         }
-      const float rstd = 1.0f / sqrtf(warp_sum(s2) / p.E + 1e-5f);
+      const float rstd = 1.0f / sqrtf(group_sum<16>(s2) / p.E + 1e-5f);
+      float part[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
-        if (j < nper) v[j] = (v[j] - mean) * rstd * gf[j] + bf[j];
-      float eps_mine = 0.f;
-      for (int a = 0; a < p.A; ++a) {
-        float part = 0.f;
+      for (int a = 0; a < 16; ++a) part[a] = 0.f;
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (j < nper) part = fmaf(v[j], __ldg(hw + (cx.lane + 32 * j) * p.A + a), part);
-        const float e = warp_sum(part);
-        if (cx.lane == a) eps_mine = e + __ldg(p.vec + p.v_headb + a);
-      }
-      if (cx.lane < p.A) {
-        const float xv = x[m * p.A + cx.lane];
-        float x0 = (xv - s1 * eps_mine) * inv_sa;
+      for (int j = 0; j < 8; ++j)
+        if (j < nv) {
+          const int col = 4 * (hl + 16 * j);
+          const float y[4] = {(v[j].x - mean) * rstd * lnf_g[col] + lnf_b[col],
+                              (v[j].y - mean) * rstd * lnf_g[col + 1] + lnf_b[col + 1],
+                              (v[j].z - mean) * rstd * lnf_g[col + 2] + lnf_b[col + 2],
+                              (v[j].w - mean) * rstd * lnf_g[col + 3] + lnf_b[col + 3]};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float* w = hw + (col + q) * p.A;
+#pragma unroll
+            for (int a = 0; a < 16; ++a)
+              if (a < p.A) part[a] = fmaf(y[q], w[a], part[a]);
+          }
+        }
+      float eps = 0.f;
+#pragma unroll
+      for (int a = 0; a < 16; ++a)
+        if (a < p.A) {
+          const float e = group_sum<16>(part[a]);
+          if (hl == a) eps = e + head_b[a];
+        }
+      if (hl < p.A) {
+        const float xv = x[m * p.A + hl];
+        float x0 = (xv - s1 * eps) * inv_sa;
         x0 = fminf(1.0f, fmaxf(-1.0f, x0));
         float xn;
         if (p.sampler == 0) {
-          xn = cx0 * x0 + cxt * xv + sig * z[m * p.A + cx.lane];
+          xn = cx0 * x0 + cxt * xv + sig * z[m * p.A + hl];
         } else {
           xn = sabp * x0 + s1p * ((xv - sab * x0) / s1);
         }
-        x[m * p.A + cx.lane] = xn;
+        x[m * p.A + hl] = xn;
       }
     }
-    if (!p.head_sep) csync(p, cx);                    // afull is rewritten by the next gather
+    if (!p.head_sep) csync(p, cx);                    // ablk is the next gather's landing zone
     bar_compute();
   }
 
   template <int MT>
-  __device__ static void compute(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
+  __device__ __forceinline__ static void compute(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
     float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
     float* z = reinterpret_cast<float*>(cx.smem + p.sm.z);
-    uint8_t* sch = cx.smem + p.sm.sch;
+    uint64_t* sch = reinterpret_cast<uint64_t*>(cx.smem + p.sm.sch);
+    float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
     const float* cst = reinterpret_cast<const float*>(cx.smem + p.sm.cst);
     const float* c_inw = cst;
     const float* c_inb = cst + p.A * p.Ec;
     const float* c_pos = c_inb + p.Ec;
-    // per-kernel constants: LN_f parameters in registers
-    float gf[16], bf[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      if (j < (p.E >> 5)) {
-        gf[j] = __ldg(p.vec + p.v_lnfg + cx.lane + 32 * j);
-        bf[j] = __ldg(p.vec + p.v_lnfb + cx.lane + 32 * j);
-      }
     for (int job = cid; job < p.n_jobs; job += ncl) {
       const int sample0 = job * p.g;
       const int s_first = min(sample0, p.samples - 1);
       const uint8_t* S = p.S + (long long)(s_first / p.per_sched) * p.S_stride;
-      // schedule rows (expanded to units) and initial x
-      for (int v = cx.tid; v < p.U * p.T; v += NCT) {
-        const int b = v / p.T, t = v - b * p.T;
-        const int row = (p.S_rows == p.U) ? b : b / 3;
-        sch[v] = S[row * p.T + t];
+      // the job's lattice as one refresh mask per step, and the initial x
+      for (int t = cx.tid; t < p.T; t += NCT) {
+        uint64_t mask = 0;
+        for (int b = 0; b < p.U; ++b) {
+          const int row = (p.S_rows == p.U) ? b : b / 3;
+          if (S[row * p.T + t] != 0) mask |= 1ull << b;
+        }
+        sch[t] = mask;
       }
       for (int v = cx.tid; v < p.M * p.A; v += NCT) {
         const int m = v / p.A;
-        const int s = min(sample0 + m / p.H, p.samples - 1);
-        x[v] = p.noise[((long long)(s % p.obs_mod) * p.H + (m % p.H)) * p.A + (v % p.A)];
+        const int s = min(sample0 + (m >> p.lH), p.samples - 1);
+        x[v] = p.noise[((long long)(s % p.obs_mod) * p.H + (m & (p.H - 1))) * p.A + (v % p.A)];
       }
       bar_compute();
       uint64_t valid = 0;
       for (int t = 0; t < p.T; ++t) {
-        // stage z_t for the sampler step (DDPM)
+        const uint64_t st = sch[t];
+        const uint64_t refresh = st | (p.force ? ~valid : 0ull);
+        // sampler coefficients of this step (used at the head)
+        const float4 tab0 = *reinterpret_cast<const float4*>(p.stab + t * 8);
+        const float4 tab1 = *reinterpret_cast<const float4*>(p.stab + t * 8 + 4);
+        // stage z_t (DDPM) and, when every layer has a slot, the memory keys/values
+        // of this step's refreshed cross-attention units
         if (p.sampler == 0) {
           const int per = p.H * p.A / 4;
           for (int v = cx.tid; v < p.g * per; v += NCT) {
@@ -759,26 +981,30 @@ struct Kern {
                        p.noise + ((long long)(1 + t) * p.obs_mod + (s % p.obs_mod)) * p.H * p.A + 4 * w);
           }
         }
+        if (p.kv_slots > 1)
+          for (int l = 0; l < p.L; ++l)
+            if ((refresh >> (3 * l + 1)) & 1ull) stage_kv(p, cx, l, t, sample0, kvs + l * p.g * p.Cm * p.kvw);
         // input embedding into this CTA's columns
         for (int e = cx.tid; e < p.M * p.Ec; e += NCT) {
-          const int m = e / p.Ec, j = e - m * p.Ec;
+          const int m = e >> p.lEc, j = e & (p.Ec - 1);
           float acc = 0.f;
           for (int a = 0; a < p.A; ++a) acc = fmaf(x[m * p.A + a], c_inw[a * p.Ec + j], acc);
-          ac[e] = acc + c_inb[j] + c_pos[(m % p.H) * p.Ec + j];
+          ac[e] = acc + c_inb[j] + c_pos[(m & (p.H - 1)) * p.Ec + j];
         }
-        bool any = false;
-        for (int b = 0; b < p.U; ++b) {
-          const bool vb = (valid >> b) & 1ull;
-          const bool r = sch[b * p.T + t] != 0 || (p.force && !vb);
-          if (r) {
+        int b = 0;
+        while (b < p.U) {
+          if ((refresh >> b) & 1ull) {
             valid |= 1ull << b;
-            any = true;
             unit<MT>(p, cx, job, b, t, sample0);
+            ++b;
           } else {
-            skip_add(p, cx, job, b, t, sample0, vb);
+            int b1 = b + 1;
+            while (b1 < p.U && b1 - b < 8 && !((refresh >> b1) & 1ull)) ++b1;
+            skip_run(p, cx, job, b, b1, t, sample0, valid);
+            b = b1;
           }
         }
-        head_step(p, cx, t, any, gf, bf);
+        head_step(p, cx, t, tab0, tab1);
       }
       // write the finished chunk
       if (cx.c == 0) {
@@ -804,8 +1030,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   cx.full = reinterpret_cast<uint64_t*>(smem + p.sm.bars);
   cx.empty = cx.full + p.nslot;
   cx.cbar = cx.full + 2 * p.nslot;
+  cx.xg = cx.cbar + 1;
+  cx.xr = cx.cbar + 2;
+  cx.xh = cx.cbar + 3;
   cx.q = 0;
-  cx.cph = 0;
+  cx.cph = cx.pg = cx.pr = cx.ph0 = cx.ph1 = 0;
   cx.dead = 0;
   const uint32_t cid = cluster_idx(), ncl = cluster_count();
 
@@ -815,20 +1044,35 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
       mbar_init(&cx.empty[i], NCW);
     }
     mbar_init(cx.cbar, p.C);
+    mbar_init(cx.xg, 1);
+    mbar_init(cx.xr, 1);
+    mbar_init(cx.xh, 1);
+    mbar_init(cx.xh + 1, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  // zero the GEMM operand buffers once: padded rows / columns must read as 0
-  for (int v = threadIdx.x; v < (p.sm.ac - p.sm.afull) / 16; v += NTHREADS)
-    reinterpret_cast<float4*>(smem + p.sm.afull)[v] = make_float4(0.f, 0.f, 0.f, 0.f);
-  // per-kernel constant slices: in_w[:, cols], in_b[cols], pos[:, cols]
+  // zero the operand and exchange buffers once: padded rows and columns must read as 0
+  for (int v = threadIdx.x; v < (p.sm.ac - p.sm.ablk) / 16; v += NTHREADS)
+    reinterpret_cast<float4*>(smem + p.sm.ablk)[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+  // per-kernel constants: in_w[:, cols], in_b[cols], pos[:, cols], lnf_g, lnf_b, head_b, head_w
   {
     float* cst = reinterpret_cast<float*>(smem + p.sm.cst);
     const int c0 = cx.c * p.Ec;
     for (int v = threadIdx.x; v < p.A * p.Ec; v += NTHREADS)
       cst[v] = p.vec[p.v_inw + (v / p.Ec) * p.E + c0 + (v % p.Ec)];
-    for (int v = threadIdx.x; v < p.Ec; v += NTHREADS) cst[p.A * p.Ec + v] = p.vec[p.v_inb + c0 + v];
-    for (int v = threadIdx.x; v < p.H * p.Ec; v += NTHREADS)
-      cst[p.A * p.Ec + p.Ec + v] = p.vec[p.v_pos + (v / p.Ec) * p.E + c0 + (v % p.Ec)];
+    float* d = cst + p.A * p.Ec;
+    for (int v = threadIdx.x; v < p.Ec; v += NTHREADS) d[v] = p.vec[p.v_inb + c0 + v];
+    d += p.Ec;
+    for (int v = threadIdx.x; v < p.H * p.Ec; v += NTHREADS) d[v] = p.vec[p.v_pos + (v / p.Ec) * p.E + c0 + (v % p.Ec)];
+    d += p.H * p.Ec;
+    for (int v = threadIdx.x; v < p.E; v += NTHREADS) {
+      d[v] = p.vec[p.v_lnfg + v];
+      d[p.E + v] = p.vec[p.v_lnfb + v];
+    }
+    d += 2 * p.E;
+    for (int v = threadIdx.x; v < p.A; v += NTHREADS) d[v] = p.vec[p.v_headb + v];
+    d += (p.A + 3) & ~3;
+    if (p.headw_smem)
+      for (int v = threadIdx.x; v < p.E * p.A; v += NTHREADS) d[v] = p.vec[p.v_headw + v];
   }
   __syncthreads();
   hw_cluster_sync();
@@ -939,7 +1183,7 @@ __global__ void pop_dev_kernel(const float* x, int P, int N_obs, int HA, float* 
       const float d = xp[(long long)n * HA + v] - ref[(long long)n * HA + v];
       s = fmaf(d, d, s);
     }
-    s = warp_sum(s);
+    s = group_sum<32>(s);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -956,41 +1200,53 @@ __global__ void pop_dev_kernel(const float* x, int P, int N_obs, int HA, float* 
 // host-side helpers
 // ---------------------------------------------------------------------------
 
-int smem_layout(JobParams& p, int es) {
+int smem_layout(JobParams& p, int es, int cache_smem) {
   auto al = [](int x, int a) { return (x + a - 1) / a * a; };
   SmemLayout s{};
   int off = 0;
   s.ring = off;
   off += p.nslot * p.slot_bytes;
-  s.afull = off;
-  off += al(p.Mp * p.ldf * 4, 128);
-  if (p.head_sep) {
-    s.hbuf = off;
-    off += al(p.M * p.ldf * 4, 128);
-  } else {
-    s.hbuf = -1;
-  }
+  // zero-initialised block: ablk .. oc
+  s.ablk = off;
+  off += al(p.C * p.blk * 4, 128);
   s.rs = off;
-  off += al(p.C * p.M * p.Ec * 4, 128);
-  const int g1b = max(p.M * p.ldg1 * 4, p.Mp * p.ldh * es);
-  s.g1 = off;
-  off += al(g1b, 128);
+  off += al(p.C * p.blk * 4, 128);
+  const int xb = p.Mp * p.lda * es;
+  const int g1b = p.M * p.ldg1 * 4 > p.Mp * p.ldh * es ? p.M * p.ldg1 * 4 : p.Mp * p.ldh * es;
+  s.xln = off;
+  off += al(xb > g1b ? xb : g1b, 128);
+  if (p.head_sep) {
+    s.hblk = off;
+    off += al(2 * p.C * p.blk * 4, 128);
+    s.hsrc = off;
+    off += al(2 * p.M * p.Ec * 4, 128);
+  } else {
+    s.hblk = s.hsrc = -1;
+  }
+  s.pb = off;
+  off += al(p.M * PLD * 4, 128);
   s.oc = off;
   off += al(p.Mp * p.ldo * es, 128);
-  s.ac = off;
+  s.ac = off;                                   // end of the zero-initialised block
   off += al(p.M * p.Ec * 4, 128);
+  if (cache_smem) {
+    s.cs = off;
+    off += al(p.U * p.M * p.Ec * es, 128);
+  } else {
+    s.cs = -1;
+  }
   s.kvs = off;
-  off += al(p.g * p.Cm * (p.dh + p.Ec) * 4, 128);
+  off += al(p.kv_slots * p.g * p.Cm * p.kvw * 4, 128);
   s.cst = off;
-  off += al((p.A * p.Ec + p.Ec + p.H * p.Ec) * 4, 128);
+  off += al((p.A * p.Ec + p.Ec + p.H * p.Ec + 2 * p.E + ((p.A + 3) & ~3) + (p.headw_smem ? p.E * p.A : 0)) * 4, 128);
   s.x = off;
   off += al(p.M * p.A * 4, 16);
   s.z = off;
   off += al(p.M * p.A * 4, 16);
   s.sch = off;
-  off += al(p.U * p.T, 16);
+  off += al(p.T * 8, 16);
   s.bars = off;
-  off += (2 * p.nslot + 1) * 8;
+  off += (2 * p.nslot + 5) * 8;
   s.total = al(off, 128);
   p.sm = s;
   return s.total;
@@ -1056,7 +1312,7 @@ cudaError_t launch_time_table(const float* w, const int* wo, const float* kstep,
 }
 
 cudaError_t launch_obs_cond(const float* w, const int* wo, const float* obs, int N, int n_obs, int D, int L, int E,
-                            float* /*unused*/, float* kv_obs, cudaStream_t s) {
+                            float* kv_obs, cudaStream_t s) {
   const size_t sh = (size_t)6 * E * sizeof(float);
   obs_cond_kernel<<<N * n_obs, 256, sh, s>>>(w, wo, obs, n_obs, D, L, E, kv_obs);
   return cudaGetLastError();
