@@ -52,6 +52,7 @@ def load() -> ctypes.CDLL:
         "evo_destroy": (I32, [P]),
         "evo_denoise": (I32, [P, P, P, P, I32, I32, P, P]),
         "evo_denoise_trace": (I32, [P, P, P, P, I32, I32, P, P, P]),
+        "evo_denoise_noalloc": (I32, [P, P, P, P, I32, I32, P, P]),
         "evo_denoise_population": (I32, [P, P, P, P, I32, I32, I32, P, P, P]),
         "evo_flops": (I32, [P, P, I32, ctypes.POINTER(I64)]),
         "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
@@ -189,6 +190,15 @@ class Evo:
             rc = load().evo_denoise_trace(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
                                           _ptr(trace), _stream(stream))
         _check(rc, "evo_denoise")
+        return out
+
+    def denoise_noalloc(self, obs, noise, S, out, stream=None):
+        """evo_denoise with its per-call scratch in the library's static device
+        array (no device allocation); `out` must be provided."""
+        S = _lattice(S)
+        rc = load().evo_denoise_noalloc(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], obs.shape[0],
+                                        _ptr(out), _stream(stream))
+        _check(rc, "evo_denoise_noalloc")
         return out
 
     def population(self, obs, noise, S_pop, out=None, dev=None, stream=None, want_actions=True):

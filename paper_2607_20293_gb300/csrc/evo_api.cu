@@ -19,6 +19,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 using namespace evo;
@@ -683,6 +684,70 @@ evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise
                              int32_t N, float* out_actions, float* trace, void* stream) {
   if (!trace) return EVO_ERR_ARG;
   return run(h, obs, noise, S, S_rows, N, out_actions, trace, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Scratch of evo_denoise_noalloc: a file-scope device array (no allocation at
+// call time).  Host code may not use the symbol as a device address; its
+// address is looked up once per device with cudaGetSymbolAddress.
+constexpr size_t NOALLOC_SCRATCH_BYTES = size_t(8) << 20;
+__device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_SCRATCH_BYTES];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[256] = {};
+
+evo_status noalloc_scratch(int dev, float** out) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (dev < 0 || dev >= 256) return EVO_ERR_UNSUPPORTED;
+  if (!g_noalloc_addr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return EVO_ERR_CUDA;
+    g_noalloc_addr[dev] = ptr;
+  }
+  *out = static_cast<float*>(g_noalloc_addr[dev]);
+  return EVO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
+                               int32_t N, float* out_actions, void* stream) {
+  if (!h || !obs || !noise || !S || !out_actions) return EVO_ERR_ARG;
+  if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
+  if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
+  const size_t kv_bytes = (size_t)N * h->cfg.n_obs * h->L * 2 * h->E * sizeof(float);
+  if (kv_bytes > NOALLOC_SCRATCH_BYTES) return EVO_ERR_SHAPE;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EVO_ERR_CUDA;
+  if (dev != h->device) return EVO_ERR_ARG;
+  float* kv = nullptr;
+  const evo_status ss = noalloc_scratch(dev, &kv);
+  if (ss != EVO_OK) return ss;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int* err = nullptr;
+  evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
+  if (s != EVO_OK) return s;
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, kv, st));
+  JobParams p = h->base;
+  p.kv_obs = kv;
+  p.samples = N;
+  p.per_sched = N;
+  p.obs_mod = N;
+  p.n_jobs = (N + p.g - 1) / p.g;
+  p.S = h->sched;
+  p.S_rows = S_rows;
+  p.S_stride = (long long)S_rows * h->T;
+  p.sched_err = err;
+  p.noise = noise;
+  p.out = out_actions;
+  p.trace = nullptr;
+  EVO_CUDA(launch_loop(h, p, st));
+  return finish(h, st);
 }
 
 evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* noise, const uint8_t* S_pop,
