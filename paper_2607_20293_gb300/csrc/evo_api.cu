@@ -265,9 +265,13 @@ int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
   for (int u = 0; u < 3; ++u) p.hdr1[u] = rup(2 * E + p.n1[u] + p.Ec, 4) * 4;
   p.sampler = c->sampler;
   p.force = c->empty_cache == EVO_EMPTY_FORCE;
+  p.invE = 1.0f / (float)E;
   if (p.Cm > 32 || p.M * p.Ec > 4 * NCT) return -1;
+  if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
   if (es == 2) {
     if (p.Mp > 32) return -1;
+    // a single 16-row tile keeps at most four 8-column tiles per warp (N <= 256)
+    if (p.Mp <= 16 && std::max(std::max(p.n1[0], p.n1[2]), E) > 8 * 4 * NCW) return -1;
   } else {
     const int nmax = std::max(std::max(p.n1[0], p.n1[2]), E);
     if (p.M * nmax > 16 * NCT) return -1;
@@ -291,7 +295,21 @@ int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
               p.slot_bytes = sb;
               p.nslot = ns;
               const int total = smem_layout(p, es, cache_smem);
-              if (total <= smem_limit) return total;
+              if (total <= smem_limit) {
+                for (int u = 0; u < 3; ++u)
+                  for (int q = 0; q < 2; ++q) {
+                    PieceInfo& pi = p.pc[u][q];
+                    pi.K = q == 0 ? E : (u == 2 ? p.kp_h : p.kp_o);
+                    pi.N = q == 0 ? p.n1[u] : E;
+                    pi.hdr = q == 0 ? p.hdr1[u] : 0;
+                    pi.ktb = 16 * pi.N * es;
+                    const int nkt = pi.K / 16;
+                    pi.ns = slab_count(pi.hdr, pi.ktb, nkt, sb);
+                    pi.k0 = std::min((sb - pi.hdr) / pi.ktb, nkt);
+                    pi.kps = sb / pi.ktb;
+                  }
+                return total;
+              }
             }
           }
   return -1;

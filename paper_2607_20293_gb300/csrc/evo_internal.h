@@ -39,6 +39,13 @@ struct SmemLayout {
   int total;
 };
 
+// One weight piece of a unit kind: K x N GEMM slice behind a `hdr`-byte header,
+// k-tiles of ktb bytes; slab 0 carries the header and k0 k-tiles, later slabs
+// kps k-tiles each; ns slabs in total.
+struct PieceInfo {
+  int K, N, hdr, ktb, ns, k0, kps;
+};
+
 struct JobParams {
   // model shape
   int L, E, nh, dh, H, A, n_obs, T, U, Cm;
@@ -50,6 +57,9 @@ struct JobParams {
   int n1[3];                      // first-GEMM width per unit kind (SA, CA, FFN)
   int hdr1[3];                    // header bytes of piece 1: gamma, beta, first bias, second-GEMM bias slice
   int kv_slots;                   // L: memory keys/values of every layer prefetched per step; 1: per unit
+  float invE;                     // 1 / E
+  // slab partition of every weight piece [unit kind][piece], precomputed on the host
+  PieceInfo pc[3][2];
   int kp_o, kp_h;                 // K of the second GEMMs (attention: Ec, FFN: hid), multiples of 16
   int n_jobs;
   int sampler, force;

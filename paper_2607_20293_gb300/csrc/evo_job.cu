@@ -247,6 +247,12 @@ struct Ctx {
   uint32_t cph, pg, pr, ph0, ph1;   // phase parities
   int dead;
   int c, tid, warp, lane;
+  // this thread's 16-byte chunk of a memory key/value staging (kv_i < 0: none):
+  // sample kv_i of the job, token kv_tok, float offset kv_src within the token's
+  // [k | v] row, float offset kv_dst within the staging slot; kv_base = the
+  // token's rows for the current job (timestep table or observation keys/values)
+  int kv_i, kv_tok, kv_src, kv_dst;
+  const float* kv_base;
 };
 
 __device__ __forceinline__ void wait_parity(uint32_t addr, uint32_t parity, bool cluster_acq, Ctx& cx,
@@ -294,16 +300,12 @@ __device__ __forceinline__ void ring_release(const JobParams& p, Ctx& cx) {
   cx.q++;
 }
 
-__device__ __forceinline__ int piece_K(const JobParams& p, int u, int piece) {
-  return piece == 0 ? p.E : (u == 2 ? p.kp_h : p.kp_o);
-}
-
-__device__ __forceinline__ int piece_N(const JobParams& p, int u, int piece) {
-  return piece == 0 ? p.n1[u] : p.E;
-}
-
-__device__ __forceinline__ int piece_hdr(const JobParams& p, int u, int piece) {
-  return piece == 0 ? p.hdr1[u] : 0;
+// slab s of a piece: first k-tile, k-tile count, byte offset and bytes (no divisions)
+__device__ __forceinline__ SlabInfo slab_of(const PieceInfo& pi, int s) {
+  if (s == 0) return SlabInfo{0, pi.k0, 0, pi.hdr + pi.k0 * pi.ktb};
+  const int kt0 = pi.k0 + (s - 1) * pi.kps;
+  const int n = min(pi.kps, pi.K / 16 - kt0);
+  return SlabInfo{kt0, n, pi.hdr + kt0 * pi.ktb, n * pi.ktb};
 }
 
 // ---------------------------------------------------------------------------
@@ -324,14 +326,11 @@ __device__ __forceinline__ void producer(const JobParams& p, Ctx& cx, uint32_t c
         valid |= 1ull << b;
         const int l = b / 3, u = b % 3;
         for (int piece = 0; piece < 2; ++piece) {
-          const int K = piece_K(p, u, piece), N = piece_N(p, u, piece), hdr = piece_hdr(p, u, piece);
+          const PieceInfo& pi = p.pc[u][piece];
           const uint8_t* src = p.wpack + (long long)cx.c * p.cta_stride + (long long)l * p.layer_stride +
                                p.poff[u][piece];
-          const int ktb = N * 16 * (int)sizeof(T);
-          const int nkt = K / 16;
-          const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
-          for (int s = 0; s < ns; ++s) {
-            const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
+          for (int s = 0; s < pi.ns; ++s) {
+            const SlabInfo si = slab_of(pi, s);
             const uint32_t slot = q % p.nslot;
             const uint32_t ph = (q / p.nslot) & 1u;
             if (!mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
@@ -364,23 +363,20 @@ __device__ __forceinline__ void producer(const JobParams& p, Ctx& cx, uint32_t c
 // bf16: warp w owns n-tiles w, w+8, ...; NTW = n-tiles per warp (compile time).
 // ---------------------------------------------------------------------------
 template <int MT, int NTW>
-__device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda, int K, int N,
-                                          int hdr, const uint8_t* slab0, float (&acc)[MT][NTW][4]) {
-  const int NT = N >> 3;
+__device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda,
+                                          const PieceInfo& pi, const uint8_t* slab0, float (&acc)[MT][NTW][4]) {
+  const int NT = pi.N >> 3;
 #pragma unroll
   for (int m = 0; m < MT; ++m)
 #pragma unroll
     for (int i = 0; i < NTW; ++i)
 #pragma unroll
       for (int r = 0; r < 4; ++r) acc[m][i][r] = 0.f;
-  const int ktb = N * 32;
-  const int nkt = K >> 4;
-  const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
   const __nv_bfloat16* arow = A + (cx.lane & 15) * lda + (cx.lane >> 4) * 8;
-  for (int s = 0; s < ns; ++s) {
+  for (int s = 0; s < pi.ns; ++s) {
     const uint8_t* sl = s == 0 ? slab0 : ring_acquire(p, cx);
-    const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
-    const uint8_t* wt = sl + (s == 0 ? hdr : 0) + cx.lane * 8;
+    const SlabInfo si = slab_of(pi, s);
+    const uint8_t* wt = sl + (s == 0 ? pi.hdr : 0) + cx.lane * 8;
 #pragma unroll 2
     for (int kk = 0; kk < si.nkt; ++kk) {
       const int kt = si.kt0 + kk;
@@ -406,8 +402,9 @@ __device__ __forceinline__ void gemm_bf16(const JobParams& p, Ctx& cx, const __n
 
 constexpr int F32_MAXO = 16;
 
-__device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const float* A, int lda, int K, int M, int N,
-                                         int hdr, const uint8_t* slab0, float (&acc)[F32_MAXO]) {
+__device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const float* A, int lda, const PieceInfo& pi,
+                                         const uint8_t* slab0, float (&acc)[F32_MAXO]) {
+  const int M = p.M, N = pi.N;
   int mi[F32_MAXO], ni[F32_MAXO];
   const int nout = M * N;
 #pragma unroll
@@ -417,13 +414,10 @@ __device__ __forceinline__ void gemm_f32(const JobParams& p, Ctx& cx, const floa
     ni[i] = o < nout ? o % N : 0;
     acc[i] = 0.f;
   }
-  const int ktb = N * 64;
-  const int nkt = K >> 4;
-  const int ns = slab_count(hdr, ktb, nkt, p.slot_bytes);
-  for (int s = 0; s < ns; ++s) {
+  for (int s = 0; s < pi.ns; ++s) {
     const uint8_t* sl = s == 0 ? slab0 : ring_acquire(p, cx);
-    const SlabInfo si = slab_at(s, hdr, ktb, nkt, p.slot_bytes);
-    const float* W = reinterpret_cast<const float*>(sl + (s == 0 ? hdr : 0));
+    const SlabInfo si = slab_of(pi, s);
+    const float* W = reinterpret_cast<const float*>(sl + (s == 0 ? pi.hdr : 0));
     const int rows = si.nkt * 16;
     for (int r = 0; r < rows; ++r) {
       const int k = si.kt0 * 16 + r;
@@ -472,7 +466,7 @@ __device__ __forceinline__ void layernorm_rows(const JobParams& p, Ctx& cx, cons
         v[j] = *reinterpret_cast<const float4*>(blk + (col >> p.lEc) * p.blk + (m << p.lEc) + (col & (p.Ec - 1)));
         s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
       }
-    const float mean = group_sum<16>(s) / p.E;
+    const float mean = group_sum<16>(s) * p.invE;
     float s2 = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j)
@@ -480,7 +474,7 @@ __device__ __forceinline__ void layernorm_rows(const JobParams& p, Ctx& cx, cons
         const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
         s2 += (a * a + b * b) + (c * c + d * d);
       }
-    const float rstd = 1.0f / sqrtf(group_sum<16>(s2) / p.E + 1e-5f);
+    const float rstd = rsqrtf(group_sum<16>(s2) * p.invE + 1e-5f);
 #pragma unroll
     for (int j = 0; j < 8; ++j)
       if (j < nv) {
@@ -531,7 +525,7 @@ struct Kern {
       bv[i] = nt < NT ? *reinterpret_cast<const float2*>(bias + nt * 8 + 2 * (cx.lane & 3)) : make_float2(0.f, 0.f);
     }
     float acc[MT][NTW][4];
-    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(xln), p.lda, p.E, N, p.hdr1[u], slab0, acc);
+    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(xln), p.lda, p.pc[u][0], slab0, acc);
     bar_compute();
 #pragma unroll
     for (int i = 0; i < NTW; ++i) {
@@ -564,7 +558,7 @@ struct Kern {
       if (ntw <= 1) gemm1_t<MT, 1>(p, cx, u, slab0);
       else if (ntw == 2) gemm1_t<MT, 2>(p, cx, u, slab0);
       else if (ntw == 3) gemm1_t<MT, 3>(p, cx, u, slab0);
-      else if (ntw == 4) gemm1_t<MT, 4>(p, cx, u, slab0);
+      else if (MT == 1 || ntw == 4) gemm1_t<MT, 4>(p, cx, u, slab0);   // one 16-row tile: N <= 256 (host check)
       else gemm1_t<MT, 8>(p, cx, u, slab0);
     } else {
       const float* xln = reinterpret_cast<const float*>(cx.smem + p.sm.xln);
@@ -579,7 +573,7 @@ struct Kern {
         bv[i] = o < p.M * N ? bias[o % N] : 0.f;
       }
       float acc[F32_MAXO];
-      gemm_f32(p, cx, xln, p.lda, p.E, p.M, N, p.hdr1[u], slab0, acc);
+      gemm_f32(p, cx, xln, p.lda, p.pc[u][0], slab0, acc);
       bar_compute();
 #pragma unroll
       for (int i = 0; i < F32_MAXO; ++i) {
@@ -602,10 +596,9 @@ struct Kern {
   __device__ __forceinline__ static void gemm2_t(const JobParams& p, Ctx& cx, int u) {
     const T* A = reinterpret_cast<const T*>(cx.smem + (u == 2 ? p.sm.xln : p.sm.oc));
     const int lda = u == 2 ? p.ldh : p.ldo;
-    const int K = u == 2 ? p.kp_h : p.kp_o;
     float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
     float acc[MT][NTW][4];
-    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, K, p.E, 0, ring_acquire(p, cx), acc);
+    gemm_bf16<MT, NTW>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, p.pc[u][1], ring_acquire(p, cx), acc);
     const int NT = p.E >> 3;
 #pragma unroll
     for (int i = 0; i < NTW; ++i) {
@@ -631,15 +624,14 @@ struct Kern {
       const int ntw = ((p.E >> 3) + NCW - 1) / NCW;
       if (ntw <= 1) gemm2_t<MT, 1>(p, cx, u);
       else if (ntw == 2) gemm2_t<MT, 2>(p, cx, u);
-      else if (ntw <= 4) gemm2_t<MT, 4>(p, cx, u);
+      else if (MT == 1 || ntw <= 4) gemm2_t<MT, 4>(p, cx, u);          // one 16-row tile: N <= 256 (host check)
       else gemm2_t<MT, 8>(p, cx, u);
     } else {
       const T* A = reinterpret_cast<const T*>(cx.smem + (u == 2 ? p.sm.xln : p.sm.oc));
       const int lda = u == 2 ? p.ldh : p.ldo;
-      const int K = u == 2 ? p.kp_h : p.kp_o;
       float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
       float acc[F32_MAXO];
-      gemm_f32(p, cx, reinterpret_cast<const float*>(A), lda, K, p.M, p.E, 0, ring_acquire(p, cx), acc);
+      gemm_f32(p, cx, reinterpret_cast<const float*>(A), lda, p.pc[u][1], ring_acquire(p, cx), acc);
 #pragma unroll
       for (int i = 0; i < F32_MAXO; ++i) {
         const int o = cx.tid + i * NCT;
@@ -663,12 +655,13 @@ struct Kern {
     T* oc = reinterpret_cast<T*>(cx.smem + p.sm.oc);
     const float scale = 1.0f / sqrtf((float)p.dh);
     const int nk = u == 0 ? p.H : p.Cm;
-    int G = 1;
-    while (G < nk) G <<= 1;
-    const int rows_per_pass = NCT / G;
+    int lG = 0;
+    while ((1 << lG) < nk) ++lG;
+    const int G = 1 << lG;
+    const int rows_per_pass = NCT >> lG;
     const int nd4 = p.dh >> 2;
     for (int base = 0; base < p.M; base += rows_per_pass) {
-      const int m = base + cx.tid / G, j = cx.tid % G;
+      const int m = base + (cx.tid >> lG), j = cx.tid & (G - 1);
       float s = -INFINITY;
       const bool live = m < p.M && j < nk;
       if (live) {
@@ -692,7 +685,7 @@ struct Kern {
       const float mx = group_max_dyn(s, G);
       const float ex = s == -INFINITY ? 0.f : expf(s - mx);
       const float sum = group_sum_dyn(ex, G);
-      if (live) pb[m * PLD + j] = ex / sum;
+      if (live) pb[m * PLD + j] = ex * __frcp_rn(sum);
     }
     bar_compute();
     for (int o = cx.tid; o < p.M * p.Ec; o += NCT) {
@@ -719,22 +712,19 @@ struct Kern {
 
   // stage the memory tokens' keys (this CTA's head) and values (its slice) of
   // layer l at step t into kvs (cp.async; waited before use)
-  __device__ __forceinline__ static void stage_kv(const JobParams& p, Ctx& cx, int l, int t, int sample0, float* kvs) {
-    const int h = (cx.c * p.Ec) / p.dh;
-    const int kq = p.dh / 4, vq = p.Ec / 4;
-    const int per_tok = kq + vq;
-    const int total = p.g * p.Cm * per_tok;
-    for (int v = cx.tid; v < total; v += NCT) {
-      const int i = v / (p.Cm * per_tok);
-      const int rem = v - i * p.Cm * per_tok;
-      const int tok = rem / per_tok, w = rem - tok * per_tok;
-      const int s = min(sample0 + i, p.samples - 1);
-      const float* src = tok == 0 ? p.kv_time + ((long long)t * p.L + l) * 2 * p.E
-                                  : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (tok - 1)) * p.L + l) * 2 * p.E;
-      const float* s4 = w < kq ? src + h * p.dh + 4 * w : src + p.E + cx.c * p.Ec + 4 * (w - kq);
-      float* d4 = kvs + (i * p.Cm + tok) * p.kvw + (w < kq ? 4 * w : p.dh + 4 * (w - kq));
-      cp_async16(d4, s4);
+  __device__ __forceinline__ static void stage_kv(const JobParams& p, Ctx& cx, int l, int t, float* kvs) {
+    if (cx.kv_i >= 0) {
+      const float* src = cx.kv_base + (cx.kv_tok == 0 ? (long long)t * p.L * 2 * p.E : 0ll) + l * 2 * p.E + cx.kv_src;
+      cp_async16(kvs + cx.kv_dst, src);
     }
+  }
+
+  // per-job part of the staging map (which sample's observation rows this thread copies)
+  __device__ __forceinline__ static void stage_kv_job(const JobParams& p, Ctx& cx, int sample0) {
+    if (cx.kv_i < 0) return;
+    const int s = min(sample0 + cx.kv_i, p.samples - 1);
+    cx.kv_base = cx.kv_tok == 0 ? p.kv_time
+                                : p.kv_obs + ((long long)(s % p.obs_mod) * p.n_obs + (cx.kv_tok - 1)) * p.L * 2 * p.E;
   }
 
   // ---- one refreshed unit (Eq. 1, (b,t) in S) --------------------------------
@@ -745,7 +735,7 @@ struct Kern {
     float* ablk = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
     float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
     if (u == 1) {
-      if (p.kv_slots == 1) stage_kv(p, cx, l, t, sample0, kvs);
+      if (p.kv_slots == 1) stage_kv(p, cx, l, t, kvs);
       else kvs += l * p.g * p.Cm * p.kvw;
     }
     // exchange 1: every CTA receives every CTA's columns of a
@@ -785,14 +775,14 @@ struct Kern {
     for (int k = 0; k < 4; ++k) {
       const int e = cx.tid + k * NCT;
       if (e < MEc) {
-        float r0 = 0.f, r1 = 0.f;
-        int cc = 0;
-        for (; cc + 1 < p.C; cc += 2) {
-          r0 += rs[cc * p.blk + e];
-          r1 += rs[(cc + 1) * p.blk + e];
-        }
-        if (cc < p.C) r0 += rs[cc * p.blk + e];
-        const float r = (r0 + r1) + b2[k];
+        float part[MAX_CLUSTER];
+#pragma unroll
+        for (int cc = 0; cc < MAX_CLUSTER; ++cc) part[cc] = cc < p.C ? rs[cc * p.blk + e] : 0.f;
+#pragma unroll
+        for (int w = MAX_CLUSTER / 2; w > 0; w >>= 1)
+#pragma unroll
+          for (int cc = 0; cc < w; ++cc) part[cc] += part[cc + w];
+        const float r = part[0] + b2[k];
         cache[e] = from_f<T>(r);
         ac[e] += r;
         if (p.trace) {
@@ -810,15 +800,18 @@ struct Kern {
                                                   int sample0, uint64_t valid) {
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
     const int MEc = p.M * p.Ec;
+    // units of the run whose cache holds a value (bit k = unit b0 + k)
+    const uint32_t live = (uint32_t)((valid >> b0) & ((1ull << (b1 - b0)) - 1ull));
+    const T* cb = cache_ptr(p, cx, job, b0);
+    const long long cstride = p.sm.cs >= 0 ? (long long)MEc : (long long)p.C * MEc;
     for (int e = cx.tid; e < MEc; e += NCT) {
       float cv[8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k)
-        cv[k] = (b0 + k < b1 && ((valid >> (b0 + k)) & 1ull)) ? to_f<T>(cache_ptr(p, cx, job, b0 + k)[e]) : 0.f;
+      for (int k = 0; k < 8; ++k) cv[k] = ((live >> k) & 1u) ? to_f<T>(cb[k * cstride + e]) : 0.f;
       float a = ac[e];
 #pragma unroll
       for (int k = 0; k < 8; ++k)
-        if (b0 + k < b1 && ((valid >> (b0 + k)) & 1ull)) a += cv[k];
+        if ((live >> k) & 1u) a += cv[k];
       ac[e] = a;
       if (p.trace) {
         const int m = e >> p.lEc, j = e & (p.Ec - 1);
@@ -881,7 +874,7 @@ struct Kern {
           v[j] = *reinterpret_cast<const float4*>(hb + (col >> p.lEc) * p.blk + (m << p.lEc) + (col & (p.Ec - 1)));
           s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
         }
-      const float mean = group_sum<16>(s) / p.E;
+      const float mean = group_sum<16>(s) * p.invE;
       float s2 = 0.f;
 #pragma unroll
       for (int j = 0; j < 8; ++j)
@@ -889,33 +882,32 @@ struct Kern {
           const float a = v[j].x - mean, b = v[j].y - mean, c = v[j].z - mean, d = v[j].w - mean;
           s2 += (a * a + b * b) + (c * c + d * d);
         }
-      const float rstd = 1.0f / sqrtf(group_sum<16>(s2) / p.E + 1e-5f);
-      float part[16];
-#pragma unroll
-      for (int a = 0; a < 16; ++a) part[a] = 0.f;
+      const float rstd = rsqrtf(group_sum<16>(s2) * p.invE + 1e-5f);
+      // normalised values of this lane's columns, then one reduced dot per action dim
 #pragma unroll
       for (int j = 0; j < 8; ++j)
         if (j < nv) {
           const int col = 4 * (hl + 16 * j);
-          const float y[4] = {(v[j].x - mean) * rstd * lnf_g[col] + lnf_b[col],
-                              (v[j].y - mean) * rstd * lnf_g[col + 1] + lnf_b[col + 1],
-                              (v[j].z - mean) * rstd * lnf_g[col + 2] + lnf_b[col + 2],
-                              (v[j].w - mean) * rstd * lnf_g[col + 3] + lnf_b[col + 3]};
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float* w = hw + (col + q) * p.A;
-#pragma unroll
-            for (int a = 0; a < 16; ++a)
-              if (a < p.A) part[a] = fmaf(y[q], w[a], part[a]);
-          }
+          v[j].x = (v[j].x - mean) * rstd * lnf_g[col] + lnf_b[col];
+          v[j].y = (v[j].y - mean) * rstd * lnf_g[col + 1] + lnf_b[col + 1];
+          v[j].z = (v[j].z - mean) * rstd * lnf_g[col + 2] + lnf_b[col + 2];
+          v[j].w = (v[j].w - mean) * rstd * lnf_g[col + 3] + lnf_b[col + 3];
         }
       float eps = 0.f;
+      for (int a = 0; a < p.A; ++a) {
+        float part = 0.f;
 #pragma unroll
-      for (int a = 0; a < 16; ++a)
-        if (a < p.A) {
-          const float e = group_sum<16>(part[a]);
-          if (hl == a) eps = e + head_b[a];
-        }
+        for (int j = 0; j < 8; ++j)
+          if (j < nv) {
+            const float* w = hw + 4 * (hl + 16 * j) * p.A + a;
+            part = fmaf(v[j].x, w[0], part);
+            part = fmaf(v[j].y, w[p.A], part);
+            part = fmaf(v[j].z, w[2 * p.A], part);
+            part = fmaf(v[j].w, w[3 * p.A], part);
+          }
+        const float e = group_sum<16>(part);
+        if (hl == a) eps = e + head_b[a];
+      }
       if (hl < p.A) {
         const float xv = x[m * p.A + hl];
         float x0 = (xv - s1 * eps) * inv_sa;
@@ -962,6 +954,7 @@ struct Kern {
         const int s = min(sample0 + (m >> p.lH), p.samples - 1);
         x[v] = p.noise[((long long)(s % p.obs_mod) * p.H + (m & (p.H - 1))) * p.A + (v % p.A)];
       }
+      stage_kv_job(p, cx, sample0);
       bar_compute();
       uint64_t valid = 0;
       for (int t = 0; t < p.T; ++t) {
@@ -983,7 +976,7 @@ struct Kern {
         }
         if (p.kv_slots > 1)
           for (int l = 0; l < p.L; ++l)
-            if ((refresh >> (3 * l + 1)) & 1ull) stage_kv(p, cx, l, t, sample0, kvs + l * p.g * p.Cm * p.kvw);
+            if ((refresh >> (3 * l + 1)) & 1ull) stage_kv(p, cx, l, t, kvs + l * p.g * p.Cm * p.kvw);
         // input embedding into this CTA's columns
         for (int e = cx.tid; e < p.M * p.Ec; e += NCT) {
           const int m = e >> p.lEc, j = e & (p.Ec - 1);
@@ -1018,7 +1011,9 @@ struct Kern {
   }
 };
 
-template <typename T>
+// MT = 16-row tiles per job (1: up to 16 rows, 2: up to 32): one instantiation
+// per tile count keeps each launch's code and register budget to its own shapes
+template <typename T, int MT>
 __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant__ JobParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   Ctx cx;
@@ -1036,6 +1031,23 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   cx.q = 0;
   cx.cph = cx.pg = cx.pr = cx.ph0 = cx.ph1 = 0;
   cx.dead = 0;
+  {
+    // staging map: chunk v = tid over [g][1+n_obs][k chunks (dh/4) | v chunks (Ec/4)]
+    const int kq = p.dh >> 2, per_tok = kq + (p.Ec >> 2);
+    const int v = threadIdx.x;
+    cx.kv_i = -1;
+    cx.kv_base = nullptr;
+    if (v < p.g * p.Cm * per_tok) {
+      const int i = v / (p.Cm * per_tok);
+      const int rem = v - i * p.Cm * per_tok;
+      const int tok = rem / per_tok, w = rem - tok * per_tok;
+      const int head = (cx.c * p.Ec) / p.dh;
+      cx.kv_i = i;
+      cx.kv_tok = tok;
+      cx.kv_src = w < kq ? head * p.dh + 4 * w : p.E + cx.c * p.Ec + 4 * (w - kq);
+      cx.kv_dst = (i * p.Cm + tok) * p.kvw + (w < kq ? 4 * w : p.dh + 4 * (w - kq));
+    }
+  }
   const uint32_t cid = cluster_idx(), ncl = cluster_count();
 
   if (threadIdx.x == 0) {
@@ -1082,10 +1094,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
       if (cx.lane == 0) producer<T>(p, cx, cid, ncl);
       __syncwarp();
     } else {
-      if (p.Mp > 16)
-        Kern<T>::template compute<2>(p, cx, cid, ncl);
-      else
-        Kern<T>::template compute<1>(p, cx, cid, ncl);
+      Kern<T>::template compute<MT>(p, cx, cid, ncl);
     }
   }
   __syncwarp();
@@ -1252,12 +1261,12 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   return s.total;
 }
 
-template <typename T>
+template <typename T, int MT>
 static cudaError_t prepare_t(int smem_bytes, int cluster, int* max_clusters) {
-  cudaError_t e = cudaFuncSetAttribute(job_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  cudaError_t e = cudaFuncSetAttribute(job_kernel<T, MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
   if (cluster > 8) {
-    e = cudaFuncSetAttribute(job_kernel<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    e = cudaFuncSetAttribute(job_kernel<T, MT>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
   }
   cudaLaunchConfig_t cfg = {};
@@ -1272,18 +1281,25 @@ static cudaError_t prepare_t(int smem_bytes, int cluster, int* max_clusters) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  e = cudaOccupancyMaxActiveClusters(&n, job_kernel<T>, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&n, job_kernel<T, MT>, &cfg);
   if (e != cudaSuccess) return e;
   *max_clusters = n;
   return cudaSuccess;
 }
 
 cudaError_t job_kernel_prepare(int dtype, int smem_bytes, int cluster, int* max_clusters) {
-  return dtype == 1 ? prepare_t<__nv_bfloat16>(smem_bytes, cluster, max_clusters)
-                    : prepare_t<float>(smem_bytes, cluster, max_clusters);
+  // both tile-count instantiations get the attributes; the cluster count is that of the smaller one
+  int n1 = 0, n2 = 0;
+  cudaError_t e = dtype == 1 ? prepare_t<__nv_bfloat16, 1>(smem_bytes, cluster, &n1)
+                             : prepare_t<float, 1>(smem_bytes, cluster, &n1);
+  if (e != cudaSuccess) return e;
+  e = dtype == 1 ? prepare_t<__nv_bfloat16, 2>(smem_bytes, cluster, &n2) : prepare_t<float, 2>(smem_bytes, cluster, &n2);
+  if (e != cudaSuccess) return e;
+  *max_clusters = n1 < n2 ? n1 : n2;
+  return cudaSuccess;
 }
 
-template <typename T>
+template <typename T, int MT>
 static cudaError_t launch_t(const JobParams& p, int n_clusters, cudaStream_t s) {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
@@ -1297,11 +1313,13 @@ static cudaError_t launch_t(const JobParams& p, int n_clusters, cudaStream_t s) 
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, job_kernel<T>, p);
+  return cudaLaunchKernelEx(&cfg, job_kernel<T, MT>, p);
 }
 
 cudaError_t launch_job(const JobParams& p, int dtype, int n_clusters, cudaStream_t s) {
-  return dtype == 1 ? launch_t<__nv_bfloat16>(p, n_clusters, s) : launch_t<float>(p, n_clusters, s);
+  if (p.Mp > 16)
+    return dtype == 1 ? launch_t<__nv_bfloat16, 2>(p, n_clusters, s) : launch_t<float, 2>(p, n_clusters, s);
+  return dtype == 1 ? launch_t<__nv_bfloat16, 1>(p, n_clusters, s) : launch_t<float, 1>(p, n_clusters, s);
 }
 
 cudaError_t launch_time_table(const float* w, const int* wo, const float* kstep, int T, int L, int E,
