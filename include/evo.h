@@ -159,10 +159,11 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop);
  * allocation after start-up, or an application whose own allocator owns the
  * device memory.  The paper has no counterpart; this is an interface choice.
  * Arguments, layouts and results are those of evo_denoise.  The per-call
- * scratch (the observation tokens' cross-attention keys/values) lives in one
- * file-scope device array of 8 MiB that every GPU which loads this library
- * holds until the process exits; N * n_obs * n_layer * 2 * n_emb * 4 bytes
- * must fit in it, else EVO_ERR_SHAPE and nothing is launched.  No cudaMalloc,
+ * scratch (the observation tokens' cross-attention keys/values and the
+ * condition MLP's intermediates) lives in one file-scope device array of
+ * 8 MiB that every GPU which loads this library holds until the process
+ * exits; N * n_obs * (2 * n_layer + 6) * n_emb * 4 bytes must fit in it, else
+ * EVO_ERR_SHAPE and nothing is launched.  No cudaMalloc,
  * cudaFree or allocating library routine is called.  The first call on a
  * device looks up the array's device address (cudaGetSymbolAddress) and
  * keeps it, so make that first call before any stream capture.  All calls

@@ -42,6 +42,7 @@ struct evo_handle {
   float* kstep = nullptr;
   float* kv_time = nullptr;
   float* kv_obs = nullptr;
+  float* cond_scratch = nullptr;   // 6E floats per condition token
   void* cache = nullptr;
   uint8_t* sched = nullptr;
   size_t sched_cap = 0;
@@ -388,6 +389,7 @@ evo_status evo_destroy(evo_handle* h) {
   cudaFree(h->kstep);
   cudaFree(h->kv_time);
   cudaFree(h->kv_obs);
+  cudaFree(h->cond_scratch);
   cudaFree(h->cache);
   cudaFree(h->sched);
   cudaFree(h->status);
@@ -580,11 +582,13 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   cudaMemcpy(h->stab, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice);
   cudaMemcpy(h->kstep, kst.data(), kst.size() * 4, cudaMemcpyHostToDevice);
   if (cudaMalloc(&h->kv_time, (size_t)T * L * 2 * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (launch_time_table(h->wf32, h->woff_d, h->kstep, T, L, E, h->kv_time, 0) != cudaSuccess)
-    return fail(EVO_ERR_CUDA);
-
   // per-call buffers
   const size_t cap_samples = (size_t)max_batch + 32;
+  const size_t cond_tokens = std::max((size_t)T, cap_samples * cfg->n_obs);
+  if (cudaMalloc(&h->cond_scratch, cond_tokens * 6 * E * sizeof(float)) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (launch_time_table(h->wf32, h->woff_d, h->woff, h->kstep, T, L, E, h->cond_scratch, h->kv_time, 0) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+
   if (cudaMalloc(&h->kv_obs, cap_samples * cfg->n_obs * L * 2 * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMalloc(&h->cache, cap_samples * H * (size_t)U * E * es) != cudaSuccess) return fail(EVO_ERR_OOM);
   h->sched_cap = cap_samples * U * T;
@@ -672,7 +676,8 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, h->kv_obs, st));
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
+                           h->cond_scratch, h->kv_obs, st));
   JobParams p = h->base;
   p.samples = N;
   p.per_sched = N;
@@ -738,8 +743,10 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
   if (!h || !obs || !noise || !S || !out_actions) return EVO_ERR_ARG;
   if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
   if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
-  const size_t kv_bytes = (size_t)N * h->cfg.n_obs * h->L * 2 * h->E * sizeof(float);
-  if (kv_bytes > NOALLOC_SCRATCH_BYTES) return EVO_ERR_SHAPE;
+  // observation keys/values, then the condition MLP's intermediates (6E floats per token)
+  const size_t kv_floats = (size_t)N * h->cfg.n_obs * h->L * 2 * h->E;
+  const size_t need = (kv_floats + (size_t)N * h->cfg.n_obs * 6 * h->E) * sizeof(float);
+  if (need > NOALLOC_SCRATCH_BYTES) return EVO_ERR_SHAPE;
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return EVO_ERR_CUDA;
   if (dev != h->device) return EVO_ERR_ARG;
@@ -750,7 +757,8 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, kv, st));
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
+                           kv + kv_floats, kv, st));
   JobParams p = h->base;
   p.kv_obs = kv;
   p.samples = N;
@@ -780,7 +788,8 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S_pop, P, S_rows, true, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, h->kv_obs, st));
+  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
+                           h->cond_scratch, h->kv_obs, st));
   JobParams p = h->base;
   // samples of one job must share a schedule: g divides N_obs
   int g = p.g;

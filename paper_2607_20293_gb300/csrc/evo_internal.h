@@ -123,10 +123,11 @@ __host__ __device__ inline SlabInfo slab_at(int s, int hdr, int ktb, int nkt, in
 int  smem_layout(JobParams& p, int elem_bytes, int cache_smem);   // fills p.sm, returns total bytes
 cudaError_t launch_job(const JobParams& p, int dtype, int n_clusters, cudaStream_t s);
 cudaError_t job_kernel_prepare(int dtype, int smem_bytes, int cluster, int* max_clusters);
-cudaError_t launch_time_table(const float* wf32, const int* woff, const float* stab_k, int T, int L, int E,
-                              float* kv_time, cudaStream_t s);
-cudaError_t launch_obs_cond(const float* wf32, const int* woff, const float* obs, int N, int n_obs, int D,
-                            int L, int E, float* kv_obs, cudaStream_t s);
+// condition path; scratch holds 6E floats per token
+cudaError_t launch_time_table(const float* wf32, const int* woff_dev, const int* woff, const float* kstep, int T,
+                              int L, int E, float* scratch, float* kv_time, cudaStream_t s);
+cudaError_t launch_obs_cond(const float* wf32, const int* woff_dev, const int* woff, const float* obs, int N,
+                            int n_obs, int D, int L, int E, float* scratch, float* kv_obs, cudaStream_t s);
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s);
 cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev, cudaStream_t s);
 

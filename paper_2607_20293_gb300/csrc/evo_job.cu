@@ -1102,77 +1102,109 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
 }
 
 // ---------------------------------------------------------------------------
-// condition path: timestep-token keys/values (once per handle) and
-// observation-token keys/values (once per call)
+// condition path: keys/values of the memory tokens for every layer.  Tokens are
+// the timestep token of every loop step (once per handle) and the observation
+// tokens of every sample (once per call).  token -> embedding -> MLP E -> 4E
+// (Mish) -> E -> per-layer [k | v] = m W_kv + b_kv.  Each matmul is one
+// column-parallel launch over all tokens.
 // ---------------------------------------------------------------------------
 
-// memory token -> per-token MLP E -> 4E (Mish) -> E, for one token per block
-__device__ void cond_mlp(const float* w, const int* wo, float* tok, float* hbuf, float* out, int E) {
-  const float* w1 = w + wo[W_CM_W1];
-  const float* b1 = w + wo[W_CM_B1];
-  const float* w2 = w + wo[W_CM_W2];
-  const float* b2 = w + wo[W_CM_B2];
-  __syncthreads();
-  for (int j = threadIdx.x; j < 4 * E; j += blockDim.x) {
-    float a = 0.f;
-    for (int e = 0; e < E; ++e) a = fmaf(tok[e], w1[(long long)e * 4 * E + j], a);
-    hbuf[j] = mish(a + b1[j]);
-  }
-  __syncthreads();
-  for (int e = threadIdx.x; e < E; e += blockDim.x) {
-    float a = 0.f;
-    for (int j = 0; j < 4 * E; ++j) a = fmaf(hbuf[j], w2[(long long)j * E + e], a);
-    out[e] = a + b2[e];
-  }
-  __syncthreads();
-}
-
-__device__ void memory_kv(const float* w, const int* wo, const float* mem, int L, int E, float* dst /*[L][2E]*/) {
-  for (int v = threadIdx.x; v < L * 2 * E; v += blockDim.x) {
-    const int l = v / (2 * E), n = v - l * 2 * E;
-    const float* wl = w + wo[W_LAYER0] + (long long)l * wo[W_LAYER_STRIDE];
-    const float* wkv = wl + wo[WL_CA_WKV];
-    float a = 0.f;
-    for (int e = 0; e < E; ++e) a = fmaf(mem[e], wkv[(long long)e * 2 * E + n], a);
-    dst[v] = a + wl[wo[WL_CA_BKV] + n];
+// X[tok][E]: mode 0 = observation token j = tok % n_obs of sample tok / n_obs
+// (obs W_obs + b_obs + cond_pos[1+j]); mode 1 = timestep token of loop step tok
+// (sinusoidal embedding of the diffusion timestep + cond_pos[0]).
+__global__ void cond_embed_kernel(const float* w, const int* wo, const float* obs, const float* kstep, int n_obs, int D,
+                                  int E, int mode, float* X) {
+  const int tok = blockIdx.x;
+  float* x = X + (long long)tok * E;
+  if (mode == 0) {
+    const int j = tok % n_obs;
+    const float* o = obs + (long long)tok * D;
+    for (int e = threadIdx.x; e < E; e += blockDim.x) {
+      float a = 0.f;
+      for (int d = 0; d < D; ++d) a = fmaf(o[d], w[wo[W_OBS_W] + (long long)d * E + e], a);
+      x[e] = a + w[wo[W_OBS_B] + e] + w[wo[W_COND_POS] + (1 + j) * E + e];
+    }
+  } else {
+    const double k = (double)kstep[tok];
+    const int half = E / 2;
+    for (int i = threadIdx.x; i < half; i += blockDim.x) {
+      const double f = exp(-log(10000.0) * (double)i / (double)(half - 1));
+      x[i] = (float)sin(k * f) + w[wo[W_COND_POS] + i];
+      x[half + i] = (float)cos(k * f) + w[wo[W_COND_POS] + half + i];
+    }
   }
 }
 
-// kv_time[t][l][2E]: keys/values of the timestep token of loop step t
-__global__ void time_table_kernel(const float* w, const int* wo, const float* kstep, int L, int E, float* kv_time) {
-  extern __shared__ float sh[];
-  float* tok = sh;
-  float* hb = sh + E;
-  float* mem = hb + 4 * E;
-  const int t = blockIdx.x;
-  const double k = (double)kstep[t];
-  const int half = E / 2;
-  for (int i = threadIdx.x; i < half; i += blockDim.x) {
-    const double f = exp(-log(10000.0) * (double)i / (double)(half - 1));
-    tok[i] = (float)sin(k * f) + w[wo[W_COND_POS] + i];
-    tok[half + i] = (float)cos(k * f) + w[wo[W_COND_POS] + half + i];
+constexpr int GV_TOK = 8;    // tokens per block
+constexpr int GV_COLS = 32;  // output columns per block (one per lane)
+constexpr int GV_KG = 8;     // K split over the block's 8 warps
+
+// Y[tok][c] = act(X[tok] . W[:, c] + bias[c]) for c < ncols.  Column c lies in
+// segment c / seg_cols: W = W0 + seg * seg_stride (row stride ldw), bias =
+// b0 + seg * bseg_stride.  act 1 = Mish.
+__global__ void __launch_bounds__(256) gemv_cols_kernel(const float* X, int ntok, int K, int ncols, const float* W0,
+                                                        long long seg_stride, int seg_cols, int ldw, const float* b0,
+                                                        long long bseg_stride, float* Y, int act) {
+  extern __shared__ float xs[];                 // [GV_TOK][K], then [GV_KG][GV_TOK][GV_COLS]
+  float* red = xs + GV_TOK * K;
+  const int t0 = blockIdx.y * GV_TOK;
+  const int nt = min(GV_TOK, ntok - t0);
+  for (int v = threadIdx.x; v < nt * K; v += blockDim.x) xs[v] = X[(long long)t0 * K + v];
+  __syncthreads();
+  const int lane = threadIdx.x & 31, kg = threadIdx.x >> 5;
+  const int c = blockIdx.x * GV_COLS + lane;
+  float acc[GV_TOK];
+#pragma unroll
+  for (int i = 0; i < GV_TOK; ++i) acc[i] = 0.f;
+  if (c < ncols) {
+    const int seg = c / seg_cols, cc = c - seg * seg_cols;
+    const float* wcol = W0 + seg * seg_stride + cc;
+    const int kper = (K + GV_KG - 1) / GV_KG;
+    const int k0 = kg * kper, k1 = min(K, k0 + kper);
+#pragma unroll 4
+    for (int k = k0; k < k1; ++k) {
+      const float wk = wcol[(long long)k * ldw];
+#pragma unroll
+      for (int i = 0; i < GV_TOK; ++i) acc[i] = fmaf(xs[i * K + k], wk, acc[i]);
+    }
   }
-  cond_mlp(w, wo, tok, hb, mem, E);
-  memory_kv(w, wo, mem, L, E, kv_time + (long long)t * L * 2 * E);
+#pragma unroll
+  for (int i = 0; i < GV_TOK; ++i) red[(kg * GV_TOK + i) * GV_COLS + lane] = acc[i];
+  __syncthreads();
+  // warp kg finishes token kg of the block
+  if (kg < nt && c < ncols) {
+    float v = 0.f;
+#pragma unroll
+    for (int g = 0; g < GV_KG; ++g) v += red[(g * GV_TOK + kg) * GV_COLS + lane];
+    const int seg = c / seg_cols, cc = c - seg * seg_cols;
+    v += b0[seg * bseg_stride + cc];
+    if (act) v = mish(v);
+    Y[(long long)(t0 + kg) * ncols + c] = v;
+  }
 }
 
-// kv_obs[s][j][l][2E] for observation token j of sample s (one block per token)
-__global__ void obs_cond_kernel(const float* w, const int* wo, const float* obs, int n_obs, int D, int L, int E,
-                                float* kv_obs) {
-  extern __shared__ float sh[];
-  float* tok = sh;
-  float* hb = sh + E;
-  float* mem = hb + 4 * E;
-  const int tokid = blockIdx.x;             // s * n_obs + j
-  const int j = tokid % n_obs;
-  const float* o = obs + (long long)tokid * D;
-  for (int e = threadIdx.x; e < E; e += blockDim.x) {
-    float a = 0.f;
-    for (int d = 0; d < D; ++d) a = fmaf(o[d], w[wo[W_OBS_W] + (long long)d * E + e], a);
-    tok[e] = a + w[wo[W_OBS_B] + e] + w[wo[W_COND_POS] + (1 + j) * E + e];
+// tokens [ntok][E] -> keys/values kv[ntok][L][2E]; scratch: ntok * 5E floats
+static cudaError_t cond_tokens_to_kv(const float* w, const int* wo_dev, const int* wo, int L, int E, int ntok,
+                                     const float* X, float* scratch, float* kv, cudaStream_t s) {
+  float* Hd = scratch;                          // [ntok][4E]
+  float* Md = scratch + (size_t)ntok * 4 * E;   // [ntok][E]
+  const int ty = (ntok + GV_TOK - 1) / GV_TOK;
+  auto smem = [](int K) { return (size_t)(GV_TOK * K + GV_KG * GV_TOK * GV_COLS) * sizeof(float); };
+  if (smem(4 * E) > 48 * 1024) {
+    // above the default dynamic shared memory limit (n_emb > 256)
+    const cudaError_t e = cudaFuncSetAttribute(gemv_cols_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem(4 * E));
+    if (e != cudaSuccess) return e;
   }
-  cond_mlp(w, wo, tok, hb, mem, E);
-  memory_kv(w, wo, mem, L, E, kv_obs + (long long)tokid * L * 2 * E);
+  gemv_cols_kernel<<<dim3((4 * E + GV_COLS - 1) / GV_COLS, ty), 256, smem(E), s>>>(
+      X, ntok, E, 4 * E, w + wo[W_CM_W1], 0, 4 * E, 4 * E, w + wo[W_CM_B1], 0, Hd, 1);
+  gemv_cols_kernel<<<dim3((E + GV_COLS - 1) / GV_COLS, ty), 256, smem(4 * E), s>>>(
+      Hd, ntok, 4 * E, E, w + wo[W_CM_W2], 0, E, E, w + wo[W_CM_B2], 0, Md, 0);
+  gemv_cols_kernel<<<dim3((L * 2 * E + GV_COLS - 1) / GV_COLS, ty), 256, smem(E), s>>>(
+      Md, ntok, E, L * 2 * E, w + wo[W_LAYER0] + wo[WL_CA_WKV], wo[W_LAYER_STRIDE], 2 * E, 2 * E,
+      w + wo[W_LAYER0] + wo[WL_CA_BKV], wo[W_LAYER_STRIDE], kv, 0);
+  (void)wo_dev;
+  return cudaGetLastError();
 }
 
 __global__ void validate_kernel(const uint8_t* S, long long n, int* err) {
@@ -1322,18 +1354,19 @@ cudaError_t launch_job(const JobParams& p, int dtype, int n_clusters, cudaStream
   return dtype == 1 ? launch_t<__nv_bfloat16, 1>(p, n_clusters, s) : launch_t<float, 1>(p, n_clusters, s);
 }
 
-cudaError_t launch_time_table(const float* w, const int* wo, const float* kstep, int T, int L, int E,
-                              float* kv_time, cudaStream_t s) {
-  const size_t sh = (size_t)6 * E * sizeof(float);
-  time_table_kernel<<<T, 256, sh, s>>>(w, wo, kstep, L, E, kv_time);
-  return cudaGetLastError();
+cudaError_t launch_time_table(const float* w, const int* wo_dev, const int* wo, const float* kstep, int T, int L,
+                              int E, float* scratch, float* kv_time, cudaStream_t s) {
+  float* X = scratch + (size_t)T * 5 * E;
+  cond_embed_kernel<<<T, 256, 0, s>>>(w, wo_dev, nullptr, kstep, 1, 1, E, 1, X);
+  return cond_tokens_to_kv(w, wo_dev, wo, L, E, T, X, scratch, kv_time, s);
 }
 
-cudaError_t launch_obs_cond(const float* w, const int* wo, const float* obs, int N, int n_obs, int D, int L, int E,
-                            float* kv_obs, cudaStream_t s) {
-  const size_t sh = (size_t)6 * E * sizeof(float);
-  obs_cond_kernel<<<N * n_obs, 256, sh, s>>>(w, wo, obs, n_obs, D, L, E, kv_obs);
-  return cudaGetLastError();
+cudaError_t launch_obs_cond(const float* w, const int* wo_dev, const int* wo, const float* obs, int N, int n_obs,
+                            int D, int L, int E, float* scratch, float* kv_obs, cudaStream_t s) {
+  const int ntok = N * n_obs;
+  float* X = scratch + (size_t)ntok * 5 * E;
+  cond_embed_kernel<<<ntok, 256, 0, s>>>(w, wo_dev, obs, nullptr, n_obs, D, E, 0, X);
+  return cond_tokens_to_kv(w, wo_dev, wo, L, E, ntok, X, scratch, kv_obs, s);
 }
 
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s) {

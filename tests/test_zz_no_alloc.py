@@ -51,7 +51,7 @@ def test_noalloc_matches_denoise_on_consecutive_calls(torch, B):
 
 
 def test_noalloc_rejects_sizes_beyond_the_static_array(torch, B):
-    # one Push-T-shaped sample needs n_obs * L * 2E * 4 = 32 KiB of the 8 MiB array
+    # one Push-T-shaped sample needs n_obs * (2L + 6) * E * 4 = 44 KiB of the 8 MiB array
     cfg = synth.config("pusht")
     n = 300
     ev = B.Evo(cfg, synth.make_weights(cfg, 0), n)
