@@ -29,6 +29,7 @@ struct evo_handle {
   int device = 0;
   int L = 0, E = 0, U = 0, T = 0, H = 0, A = 0;
   JobParams base{};
+  int shape = -1;               // compiled loop-kernel shape (evo_shapes.h)
   int max_batch = 0;
   int max_clusters = 0;
   int smem_limit = 0;
@@ -228,8 +229,9 @@ inline int ilog2(int x) {
   return l;
 }
 
-// Fill p's decomposition fields for g samples per job; returns shared bytes or -1.
-int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
+// Fill p's decomposition fields for g samples per job and the ring geometry
+// (slot bytes, slots) of the compiled shape; returns shared bytes or -1.
+int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit, JobParams& p) {
   const int E = c->n_emb, dh = E / c->n_head, H = c->horizon;
   const int es = c->dtype == EVO_DTYPE_BF16 ? 2 : 4;
   auto r84 = [](int x) { return x + ((12 - x % 8) % 8); };      // smallest y >= x with y % 8 == 4
@@ -271,8 +273,6 @@ int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
   if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
   if (es == 2) {
     if (p.Mp > 32) return -1;
-    // a single 16-row tile keeps at most four 8-column tiles per warp (N <= 256)
-    if (p.Mp <= 16 && std::max(std::max(p.n1[0], p.n1[2]), E) > 8 * 4 * NCW) return -1;
   } else {
     const int nmax = std::max(std::max(p.n1[0], p.n1[2]), E);
     if (p.M * nmax > 16 * NCT) return -1;
@@ -280,39 +280,21 @@ int plan(const evo_config* c, int C, int g, int smem_limit, JobParams& p) {
   // a ring slot must hold any piece-1 header plus one k-tile, and one k-tile of piece 2
   int need = 16 * E * es;
   for (int u = 0; u < 3; ++u) need = std::max(need, p.hdr1[u] + 16 * p.n1[u] * es);
-  const int slots[] = {32768, 24576, 16384};
+  if (slot < need) return -1;
+  p.slot_bytes = slot;
+  p.nslot = nslot;
   // preference: caches on chip, per-step memory keys/values, double-buffered
-  // head exchange, head weights on chip, deep ring
+  // head exchange, head weights on chip
   for (int cache_smem = 1; cache_smem >= 0; --cache_smem)
     for (int kvall = 1; kvall >= 0; --kvall)
       for (int head_sep = 1; head_sep >= 0; --head_sep)
-        for (int headw = 1; headw >= 0; --headw)
-          for (int sb : slots) {
-            if (sb < need) continue;
-            for (int ns = 4; ns >= 2; --ns) {
-              p.kv_slots = kvall ? p.L : 1;
-              p.head_sep = head_sep;
-              p.headw_smem = headw;
-              p.slot_bytes = sb;
-              p.nslot = ns;
-              const int total = smem_layout(p, es, cache_smem);
-              if (total <= smem_limit) {
-                for (int u = 0; u < 3; ++u)
-                  for (int q = 0; q < 2; ++q) {
-                    PieceInfo& pi = p.pc[u][q];
-                    pi.K = q == 0 ? E : (u == 2 ? p.kp_h : p.kp_o);
-                    pi.N = q == 0 ? p.n1[u] : E;
-                    pi.hdr = q == 0 ? p.hdr1[u] : 0;
-                    pi.ktb = 16 * pi.N * es;
-                    const int nkt = pi.K / 16;
-                    pi.ns = slab_count(pi.hdr, pi.ktb, nkt, sb);
-                    pi.k0 = std::min((sb - pi.hdr) / pi.ktb, nkt);
-                    pi.kps = sb / pi.ktb;
-                  }
-                return total;
-              }
-            }
-          }
+        for (int headw = 1; headw >= 0; --headw) {
+          p.kv_slots = kvall ? p.L : 1;
+          p.head_sep = head_sep;
+          p.headw_smem = headw;
+          const int total = smem_layout(p, es, cache_smem);
+          if (total <= smem_limit) return total;
+        }
   return -1;
 }
 
@@ -431,26 +413,32 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   const int dh = E / cfg->n_head;
 
   // ---- decomposition ------------------------------------------------------
-  int C = cfg->cluster;
+  const int g = cfg->job_samples > 0 ? cfg->job_samples : 1;
+  int C = cfg->cluster, slot = 0, nslot = 0;
   if (C == 0) {
+    // the largest cluster with a compiled kernel for this shape
     const int cap = std::min(MAX_CLUSTER, std::max(1, E / 16));
     for (C = cap; C >= 1; C >>= 1)
-      if (cluster_ok(cfg, C)) break;
+      if (cluster_ok(cfg, C) && shape_find(cfg->dtype, E, cfg->n_head, H, C, g, &slot, &nslot) >= 0) break;
   }
   if (C < 1 || !cluster_ok(cfg, C)) {
     delete h;
     return EVO_ERR_SHAPE;
   }
-  int g = cfg->job_samples > 0 ? cfg->job_samples : 1;
+  h->shape = shape_find(cfg->dtype, E, cfg->n_head, H, C, g, &slot, &nslot);
+  if (h->shape < 0) {
+    delete h;
+    return EVO_ERR_UNSUPPORTED;
+  }
   JobParams& p = h->base;
-  const int smem = plan(cfg, C, g, smem_optin, p);
+  const int smem = plan(cfg, C, g, slot, nslot, smem_optin, p);
   if (smem < 0) {
     delete h;
     return EVO_ERR_UNSUPPORTED;
   }
   {
     int mc = 0;
-    cudaError_t e = job_kernel_prepare(cfg->dtype, smem, C, &mc);
+    cudaError_t e = job_kernel_prepare(h->shape, smem, &mc);
     if (e != cudaSuccess || mc <= 0) {
       cudaGetLastError();
       delete h;
@@ -649,12 +637,12 @@ evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int row
   return EVO_OK;
 }
 
-cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st) {
+cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, int shape = -1) {
   if (h->prof_start && h->prof_stop) {
     cudaError_t e = cudaEventRecord(h->prof_start, st);
     if (e != cudaSuccess) return e;
   }
-  cudaError_t e = launch_job(p, h->cfg.dtype, std::min(p.n_jobs, h->max_clusters), st);
+  cudaError_t e = launch_job(shape >= 0 ? shape : h->shape, p, std::min(p.n_jobs, h->max_clusters), st);
   if (e != cudaSuccess) return e;
   if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
   return cudaSuccess;
@@ -792,14 +780,24 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
                            h->cond_scratch, h->kv_obs, st));
   JobParams p = h->base;
   // samples of one job must share a schedule: g divides N_obs
-  int g = p.g;
+  int g = p.g, shape = h->shape;
   while (g > 1 && N_obs % g) g >>= 1;
   if (g != p.g) {
-    p.g = g;
-    p.M = g * p.H;
-    p.Mp = rup(p.M, 16);
-    p.blk = p.M * p.Ec + 4;
-    smem_layout(p, h->es, p.sm.cs >= 0);
+    // fewer samples per job: the compiled shape for g, with its own ring geometry
+    int slot = 0, nslot = 0;
+    shape = shape_find(h->cfg.dtype, h->E, h->cfg.n_head, h->H, p.C, g, &slot, &nslot);
+    if (shape < 0) return EVO_ERR_UNSUPPORTED;
+    const int smem = plan(&h->cfg, p.C, g, slot, nslot, h->smem_limit, p);
+    if (smem < 0) return EVO_ERR_UNSUPPORTED;
+    int mc = 0;
+    EVO_CUDA(job_kernel_prepare(shape, smem, &mc));
+    p.stab = h->stab;
+    p.kv_time = h->kv_time;
+    p.kv_obs = h->kv_obs;
+    p.wpack = h->wpack;
+    p.vec = h->vec;
+    p.cache = h->cache;
+    p.status = h->status;
   }
   p.samples = (int)samples;
   p.per_sched = N_obs;
@@ -812,7 +810,7 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   p.noise = noise;
   p.out = h->pop_x;
   p.trace = nullptr;
-  EVO_CUDA(launch_loop(h, p, st));
+  EVO_CUDA(launch_loop(h, p, st, shape));
   const int HA = h->H * h->A;
   EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
   if (out_actions)

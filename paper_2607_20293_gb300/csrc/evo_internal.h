@@ -39,13 +39,6 @@ struct SmemLayout {
   int total;
 };
 
-// One weight piece of a unit kind: K x N GEMM slice behind a `hdr`-byte header,
-// k-tiles of ktb bytes; slab 0 carries the header and k0 k-tiles, later slabs
-// kps k-tiles each; ns slabs in total.
-struct PieceInfo {
-  int K, N, hdr, ktb, ns, k0, kps;
-};
-
 struct JobParams {
   // model shape
   int L, E, nh, dh, H, A, n_obs, T, U, Cm;
@@ -58,8 +51,6 @@ struct JobParams {
   int hdr1[3];                    // header bytes of piece 1: gamma, beta, first bias, second-GEMM bias slice
   int kv_slots;                   // L: memory keys/values of every layer prefetched per step; 1: per unit
   float invE;                     // 1 / E
-  // slab partition of every weight piece [unit kind][piece], precomputed on the host
-  PieceInfo pc[3][2];
   int kp_o, kp_h;                 // K of the second GEMMs (attention: Ec, FFN: hid), multiples of 16
   int n_jobs;
   int sampler, force;
@@ -95,34 +86,13 @@ struct JobParams {
   SmemLayout sm;
 };
 
-// Slab partition of one weight piece: a header of `hdr` bytes followed by nkt
-// k-tiles of ktb bytes, cut into ring slots of `slot` bytes.  Slab 0 carries the
-// header and as many whole k-tiles as fit; later slabs carry whole k-tiles.
-struct SlabInfo {
-  int kt0, nkt, off, bytes;
-};
-
-__host__ __device__ inline int slab_count(int hdr, int ktb, int nkt, int slot) {
-  const int k0 = (slot - hdr) / ktb;
-  if (nkt <= k0) return 1;
-  const int kps = slot / ktb;
-  return 1 + (nkt - k0 + kps - 1) / kps;
-}
-
-__host__ __device__ inline SlabInfo slab_at(int s, int hdr, int ktb, int nkt, int slot) {
-  int k0 = (slot - hdr) / ktb;
-  if (k0 > nkt) k0 = nkt;
-  if (s == 0) return SlabInfo{0, k0, 0, hdr + k0 * ktb};
-  const int kps = slot / ktb;
-  const int kt0 = k0 + (s - 1) * kps;
-  const int n = (nkt - kt0) < kps ? (nkt - kt0) : kps;
-  return SlabInfo{kt0, n, hdr + kt0 * ktb, n * ktb};
-}
-
 // host helpers implemented in evo_job.cu
 int  smem_layout(JobParams& p, int elem_bytes, int cache_smem);   // fills p.sm, returns total bytes
-cudaError_t launch_job(const JobParams& p, int dtype, int n_clusters, cudaStream_t s);
-cudaError_t job_kernel_prepare(int dtype, int smem_bytes, int cluster, int* max_clusters);
+// compiled loop-kernel shapes (evo_shapes.h): id for a configuration or -1,
+// with the ring geometry that shape was compiled for
+int shape_find(int dtype, int E, int NH, int H, int C, int G, int* slot, int* nslot);
+cudaError_t job_kernel_prepare(int shape, int smem_bytes, int* max_clusters);
+cudaError_t launch_job(int shape, const JobParams& p, int n_clusters, cudaStream_t s);
 // condition path; scratch holds 6E floats per token
 cudaError_t launch_time_table(const float* wf32, const int* woff_dev, const int* woff, const float* kstep, int T,
                               int L, int E, float* scratch, float* kv_time, cudaStream_t s);

@@ -1,0 +1,970 @@
+// The denoising-loop kernel, compiled per model shape.
+//
+// One persistent kernel runs whole action queries.  A "job" is a group of G
+// samples that share one schedule; a thread-block cluster of C CTAs runs the
+// job's complete T-step reverse-diffusion loop (Sec. 3.1: T steps, B = 3L
+// cacheable units) without returning to the host:
+//
+//   for t in 0..T-1:
+//     a = x W_in + b_in + P_pos                      (this CTA's E/C columns)
+//     for b in 0..3L-1:                              (Eq. 1)
+//       (b,t) in S ? r = branch_b(a), c_b <- r, a += r
+//                  : a += c_b                        (skip: a local add)
+//     eps = LN_f(a) W_head + b_head ; x <- sampler step(x, eps, z_t)
+//
+// The residual stream a is distributed over the cluster by columns: each CTA
+// owns E/C columns of a and of every unit's cache c_b (in shared memory when
+// the slice fits, else in global memory), so a skipped cell is a local add.
+// A refreshed unit needs two cluster exchanges, both done with bulk
+// asynchronous copies from this CTA's shared memory into the other CTAs'
+// (cp.async.bulk shared::cta -> shared::cluster, one per destination) that
+// count their bytes on the receiver's mbarrier -- no fences and no
+// cluster-wide barriers:
+//   1. all-gather of a, so every CTA normalises full rows (LayerNorm);
+//   2. reduce-scatter of the second matmul's partial sums, so every CTA
+//      finishes its own columns of r = branch output.
+// In between each CTA computes its share of the branch: attention -- the
+// queries/keys of its head and its slice of head dimensions; FFN -- its slice
+// of the hidden layer.  The order of the exchanges makes every buffer's reuse
+// safe: a CTA can only send into a buffer again after it has received data
+// that the receiver sends once it has finished reading that buffer (argued at
+// each buffer below).
+//
+// Weights never pass through registers on their way in: a producer warp per
+// CTA walks the same schedule and streams, for every refreshed unit only, the
+// CTA's pre-packed weight slices (with the unit's LayerNorm gain/shift and
+// biases in front) through a ring of shared-memory slots with bulk
+// asynchronous copies (cp.async.bulk + mbarrier transaction counts).  Skipped
+// units generate no weight traffic, so time follows the schedule.
+//
+// bf16 mode: GEMM operands bf16, mma.sync m16n8k16 with fp32 accumulation
+// (rows per job are 16..32, far below a tcgen05 tile; the cost here is weight
+// streaming and on-chip latency, not tensor throughput).  fp32 mode: FFMA.
+// Caches are stored in the GEMM operand type.
+//
+// Every size below is a compile-time constant of the Shape, so the inner
+// loops unroll completely and addresses fold to constants: at these sizes the
+// kernel is bound by dependent latencies and control flow, not by arithmetic.
+#pragma once
+
+#include "evo_ptx.cuh"
+
+namespace evo {
+
+__host__ __device__ constexpr int ct_ilog2(int x) { return x <= 1 ? 0 : 1 + ct_ilog2(x / 2); }
+__host__ __device__ constexpr int ct_rup(int x, int a) { return (x + a - 1) / a * a; }
+__host__ __device__ constexpr int ct_r84(int x) { return x + ((12 - x % 8) % 8); }   // smallest y >= x with y % 8 == 4
+__host__ __device__ constexpr int ct_min(int a, int b) { return a < b ? a : b; }
+
+// Model shape of one compiled loop kernel: embedding E, NH heads, horizon H,
+// cluster size C, G samples per job, ES bytes per GEMM operand, ring of NSLOT
+// slots of SLOT bytes.  The host plan computes the same values (checked at launch).
+template <int E_, int NH_, int H_, int C_, int G_, int ES_, int SLOT_, int NSLOT_>
+struct Shape {
+  static constexpr int E = E_, NH = NH_, H = H_, C = C_, G = G_, ES = ES_, SLOT = SLOT_, NSLOT = NSLOT_;
+  static constexpr int dh = E / NH, Ec = E / C, hid = 4 * E / C;
+  static constexpr int M = G * H, MT = (M + 15) / 16, Mp = MT * 16;
+  static constexpr int lEc = ct_ilog2(Ec), lH = ct_ilog2(H);
+  static constexpr int blk = M * Ec + 4;
+  static constexpr int lda = ES == 2 ? E + 8 : E + 4;
+  static constexpr int n1_sa = 2 * dh + Ec, n1_ca = dh, n1_ff = hid;
+  static constexpr int ldg1 = ct_r84(n1_sa), kvw = ct_r84(dh + Ec);
+  static constexpr int kp_o = ct_rup(Ec, 16), kp_h = ct_rup(hid, 16);
+  static constexpr int ldh = ES == 2 ? kp_h + 8 : kp_h, ldo = ES == 2 ? kp_o + 8 : kp_o;
+  static constexpr float invE = 1.0f / E;
+  __host__ __device__ static constexpr int n1(int u) { return u == 0 ? n1_sa : (u == 1 ? n1_ca : n1_ff); }
+  __host__ __device__ static constexpr int hdr1(int u) { return ct_rup(2 * E + n1(u) + Ec, 4) * 4; }
+  // piece q of unit kind u: K x N slice behind a header, cut into ring slabs
+  __host__ __device__ static constexpr int pK(int u, int q) { return q == 0 ? E : (u == 2 ? kp_h : kp_o); }
+  __host__ __device__ static constexpr int pN(int u, int q) { return q == 0 ? n1(u) : E; }
+  __host__ __device__ static constexpr int pHdr(int u, int q) { return q == 0 ? hdr1(u) : 0; }
+  __host__ __device__ static constexpr int pKtb(int u, int q) { return 16 * pN(u, q) * ES; }
+  __host__ __device__ static constexpr int pK0(int u, int q) { return ct_min((SLOT - pHdr(u, q)) / pKtb(u, q), pK(u, q) / 16); }
+  __host__ __device__ static constexpr int pKps(int u, int q) { return SLOT / pKtb(u, q); }
+  __host__ __device__ static constexpr int pNs(int u, int q) {
+    return pK(u, q) / 16 <= pK0(u, q) ? 1 : 1 + (pK(u, q) / 16 - pK0(u, q) + pKps(u, q) - 1) / pKps(u, q);
+  }
+  static_assert((NSLOT & (NSLOT - 1)) == 0, "ring slots: a power of two");
+  static_assert((Ec & (Ec - 1)) == 0 && (H & (H - 1)) == 0, "Ec and H: powers of two");
+  static_assert(M * Ec <= 4 * NCT, "at most four residual columns per thread");
+  // slab 0 of a piece holds its header and at least one k-tile
+  static_assert(pK0(0, 0) >= 1 && pK0(1, 0) >= 1 && pK0(2, 0) >= 1 && pK0(0, 1) >= 1 && pK0(2, 1) >= 1,
+                "slab 0 must hold one k-tile");
+};
+
+template <typename T, class S>
+struct Loop {
+  static constexpr bool BF = sizeof(T) == 2;
+  static constexpr int M = S::M, MT = S::MT, E = S::E, Ec = S::Ec, C = S::C, H = S::H, dh = S::dh;
+  static constexpr int MEc = M * Ec;
+  static constexpr int EPT = (MEc + NCT - 1) / NCT;          // residual elements per thread (1..4)
+  static constexpr uint32_t XBYTES = (uint32_t)(M * E * 4);    // bytes one exchange delivers to a CTA
+
+  // ---------------------------------------------------------------- rings and barriers
+  // wait for the oldest unreleased slab (cx.q)
+  __device__ __forceinline__ static const uint8_t* ring_acquire(const JobParams& p, Ctx& cx) {
+    const uint32_t slot = cx.q & (S::NSLOT - 1);
+    const uint32_t ph = (cx.q / S::NSLOT) & 1u;
+    wait_parity(smem_u32(&cx.full[slot]), ph, false, cx, p.status);
+    return cx.smem + p.sm.ring + slot * S::SLOT;
+  }
+
+  __device__ __forceinline__ static void ring_release(Ctx& cx) {
+    __syncwarp();
+    if (cx.lane == 0) mbar_arrive(&cx.empty[cx.q & (S::NSLOT - 1)]);
+    cx.q++;
+  }
+
+  // cluster-wide barrier among the compute warps only (the producer warp runs
+  // ahead); used where no data exchange orders a buffer's reuse
+  __device__ __forceinline__ static void csync(const JobParams& p, Ctx& cx) {
+    fence_cluster();
+    bar_compute();
+    if (cx.tid < C) mbar_arrive_cluster(mapa(smem_u32(cx.cbar), cx.tid));
+    wait_parity(smem_u32(cx.cbar), cx.cph, true, cx, p.status);
+    cx.cph ^= 1u;
+  }
+
+  // receive one exchange phase (XBYTES) on barrier `bar`
+  __device__ __forceinline__ static void exchange_wait(const JobParams& p, Ctx& cx, uint64_t* bar, uint32_t& parity) {
+    if (cx.tid == 0) mbar_arrive_expect_tx(bar, XBYTES);
+    wait_parity(smem_u32(bar), parity, true, cx, p.status);
+    parity ^= 1u;
+  }
+
+  // Send one block of M*Ec floats to every CTA r of the cluster: block
+  // src + r*src_stride lands in CTA r at dst + c*blk (c = this CTA), counted on
+  // r's barrier `rbar`.  The writers of src have executed fence_proxy_async()
+  // and a bar_compute() before this call.
+  __device__ __forceinline__ static void send_blocks(Ctx& cx, const float* src, int src_stride, const float* dst,
+                                                     uint64_t* rbar) {
+    if (cx.tid < C) {
+      const uint32_t r = (uint32_t)cx.tid;
+      bulk_s2c(mapa(smem_u32(dst + cx.c * S::blk), r), src + r * src_stride, (uint32_t)(MEc * 4),
+               mapa(smem_u32(rbar), r));
+    }
+  }
+
+  // ---------------------------------------------------------------- producer warp
+  __device__ __forceinline__ static void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
+    uint32_t q = 0;
+    for (int job = cid; job < p.n_jobs; job += ncl) {
+      const int s0 = min(job * S::G, p.samples - 1);
+      const uint8_t* Sl = p.S + (long long)(s0 / p.per_sched) * p.S_stride;
+      uint64_t valid = 0;
+      for (int t = 0; t < p.T; ++t) {
+        for (int b = 0; b < p.U; ++b) {
+          const int row = (p.S_rows == p.U) ? b : b / 3;
+          const bool vb = (valid >> b) & 1ull;
+          if (!(Sl[row * p.T + t] != 0 || (p.force && !vb))) continue;   // same rule as the compute warps
+          valid |= 1ull << b;
+          const int l = b / 3, u = b % 3;
+          for (int piece = 0; piece < 2; ++piece) {
+            const uint8_t* src =
+                p.wpack + (long long)cx.c * p.cta_stride + (long long)l * p.layer_stride + p.poff[u][piece];
+            const int ns = S::pNs(u, piece), k0 = S::pK0(u, piece), kps = S::pKps(u, piece);
+            const int ktb = S::pKtb(u, piece), hdr = S::pHdr(u, piece), nkt = S::pK(u, piece) / 16;
+            for (int s = 0; s < ns; ++s) {
+              const int kt0 = s == 0 ? 0 : k0 + (s - 1) * kps;
+              const int cnt = s == 0 ? k0 : min(kps, nkt - kt0);
+              const uint32_t off = s == 0 ? 0u : (uint32_t)(hdr + kt0 * ktb);
+              const uint32_t bytes = (uint32_t)((s == 0 ? hdr : 0) + cnt * ktb);
+              const uint32_t slot = q & (S::NSLOT - 1);
+              const uint32_t ph = (q / S::NSLOT) & 1u;
+              if (!mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
+                // the producer runs ahead of the compute warps: poll gently
+                const long long t0 = clock64();
+                while (!cx.dead && !mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
+                  __nanosleep(64);
+                  if (clock64() - t0 > WAIT_LIMIT) {
+                    atomicOr(p.status, ST_TIMEOUT);
+                    cx.dead = 1;
+                  }
+                }
+              }
+              mbar_arrive_expect_tx(&cx.full[slot], bytes);
+              bulk_g2s(cx.smem + p.sm.ring + slot * S::SLOT, src + off, bytes, &cx.full[slot]);
+              ++q;
+            }
+          }
+        }
+      }
+    }
+    // drain: every slab issued has landed before this CTA may exit (bounded waits)
+    const uint32_t first = q > (uint32_t)S::NSLOT ? q - S::NSLOT : 0u;
+    for (uint32_t k = first; k < q; ++k)
+      wait_parity(smem_u32(&cx.full[k & (S::NSLOT - 1)]), (k / S::NSLOT) & 1u, false, cx, p.status);
+  }
+
+  // ---------------------------------------------------------------- GEMMs over streamed slabs
+  // Piece (U, Q) arrives as NS slabs: slab 0 holds the header and k-tiles
+  // 0..K0-1, slab s >= 1 the next KPS k-tiles.  The slab boundaries are
+  // compile-time, so in the unrolled k-loop each warp waits for slab s at its
+  // first k-tile and releases it after its last one: the producer refills a
+  // slot as soon as every warp is past it, and a piece may span more slabs
+  // than the ring has slots.
+  template <int U, int Q>
+  __device__ __forceinline__ static constexpr bool slab_first(int kt) {
+    return kt >= S::pK0(U, Q) && (kt - S::pK0(U, Q)) % S::pKps(U, Q) == 0;
+  }
+  template <int U, int Q>
+  __device__ __forceinline__ static constexpr bool slab_last(int kt) {
+    return kt == S::pK(U, Q) / 16 - 1 || slab_first<U, Q>(kt + 1);
+  }
+
+  // bf16: warp w owns n-tiles w, w+8, ... (NTW of them)
+  template <int U, int Q>
+  __device__ __forceinline__ static void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda,
+                                                   const uint8_t* slab0,
+                                                   float (&acc)[MT][(S::pN(U, Q) / 8 + NCW - 1) / NCW][4]) {
+    constexpr int NT = S::pN(U, Q) / 8, NTW = (NT + NCW - 1) / NCW;
+    constexpr int NKT = S::pK(U, Q) / 16, K0 = S::pK0(U, Q), KPS = S::pKps(U, Q);
+    constexpr int HDR = S::pHdr(U, Q);
+    const uint8_t* sl = slab0 + HDR + cx.lane * 8;
+#pragma unroll
+    for (int m = 0; m < MT; ++m)
+#pragma unroll
+      for (int i = 0; i < NTW; ++i)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) acc[m][i][r] = 0.f;
+    const __nv_bfloat16* arow = A + (cx.lane & 15) * lda + (cx.lane >> 4) * 8;
+#pragma unroll
+    for (int kt = 0; kt < NKT; ++kt) {
+      if (slab_first<U, Q>(kt)) sl = ring_acquire(p, cx) + cx.lane * 8;
+      const int kk = kt < K0 ? kt : (kt - K0) % KPS;
+      uint32_t a[MT][4];
+#pragma unroll
+      for (int m = 0; m < MT; ++m) ldmatrix_x4(a[m], arow + m * 16 * lda + kt * 16);
+#pragma unroll
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        if (NT % NCW == 0 || nt < NT) {
+          const uint2 bf = *reinterpret_cast<const uint2*>(sl + (kk * NT + nt) * 256);
+#pragma unroll
+          for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], a[m], bf);
+        }
+      }
+      if (slab_last<U, Q>(kt)) ring_release(cx);
+    }
+  }
+
+  // fp32: one output per thread and slot i (M*N <= 16*NCT)
+  static constexpr int F32_MAXO = 16;
+  template <int U, int Q>
+  __device__ __forceinline__ static void gemm_f32(const JobParams& p, Ctx& cx, const float* A, int lda,
+                                                  const uint8_t* slab0, float (&acc)[F32_MAXO]) {
+    constexpr int N = S::pN(U, Q), NKT = S::pK(U, Q) / 16, K0 = S::pK0(U, Q), KPS = S::pKps(U, Q);
+    constexpr int HDR = S::pHdr(U, Q);
+    constexpr int NOUT = M * N;
+    constexpr int NO = (NOUT + NCT - 1) / NCT;
+    static_assert(NO <= F32_MAXO, "fp32 GEMM: at most 16 outputs per thread");
+    const float* sl = reinterpret_cast<const float*>(slab0 + HDR);
+#pragma unroll
+    for (int i = 0; i < F32_MAXO; ++i) acc[i] = 0.f;
+#pragma unroll
+    for (int kt = 0; kt < NKT; ++kt) {
+      if (slab_first<U, Q>(kt)) sl = reinterpret_cast<const float*>(ring_acquire(p, cx));
+      const int r0 = (kt < K0 ? kt : (kt - K0) % KPS) * 16;
+#pragma unroll 4
+      for (int k = 0; k < 16; ++k) {
+#pragma unroll
+        for (int i = 0; i < NO; ++i) {
+          const int o = cx.tid + i * NCT;
+          if (NOUT % NCT == 0 || o < NOUT)
+            acc[i] = fmaf(A[(o / N) * lda + kt * 16 + k], sl[(r0 + k) * N + (o % N)], acc[i]);
+        }
+      }
+      if (slab_last<U, Q>(kt)) ring_release(cx);
+    }
+  }
+
+  // ---------------------------------------------------------------- LayerNorm
+  // Rows m < M, half a warp per row, one pass for the mean and the second
+  // moment.  Row m is read from the gathered blocks (column col is in block
+  // col/Ec) and written to the A operand xln in type T.
+  __device__ __forceinline__ static void layernorm_rows(Ctx& cx, const float* blk, T* xln, const float* gam,
+                                                        const float* bet) {
+    constexpr int NV = E / 64;
+    const int half = cx.lane >> 4, hl = cx.lane & 15;
+#pragma unroll
+    for (int m0 = 0; m0 < M; m0 += 2 * NCW) {
+      const int m = m0 + cx.warp * 2 + half;
+      if (M % (2 * NCW) == 0 || m0 + cx.warp * 2 < M) {
+        float4 v[NV];
+        float s = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+          const int col = 4 * (hl + 16 * j);
+          v[j] = *reinterpret_cast<const float4*>(blk + (col >> S::lEc) * S::blk + (m << S::lEc) + (col & (Ec - 1)));
+          s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+          s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) {
+          s += __shfl_xor_sync(0xffffffffu, s, o);
+          s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+        }
+        const float mean = s * S::invE;
+        const float rstd = rsqrtf(fmaxf(s2 * S::invE - mean * mean, 0.f) + 1e-5f);
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+          const int col = 4 * (hl + 16 * j);
+          const float4 g = *reinterpret_cast<const float4*>(gam + col);
+          const float4 bb = *reinterpret_cast<const float4*>(bet + col);
+          const float y0 = (v[j].x - mean) * rstd * g.x + bb.x, y1 = (v[j].y - mean) * rstd * g.y + bb.y;
+          const float y2 = (v[j].z - mean) * rstd * g.z + bb.z, y3 = (v[j].w - mean) * rstd * g.w + bb.w;
+          T* dst = xln + m * S::lda + col;
+          if constexpr (BF) {
+            __nv_bfloat162 lo = __floats2bfloat162_rn(y0, y1), hi = __floats2bfloat162_rn(y2, y3);
+            uint2 pk;
+            pk.x = *reinterpret_cast<uint32_t*>(&lo);
+            pk.y = *reinterpret_cast<uint32_t*>(&hi);
+            *reinterpret_cast<uint2*>(dst) = pk;
+          } else {
+            *reinterpret_cast<float4*>(dst) = make_float4(y0, y1, y2, y3);
+          }
+        }
+      }
+    }
+  }
+
+  __device__ __forceinline__ static T* cache_ptr(const JobParams& p, Ctx& cx, int job, int b) {
+    if (p.sm.cs >= 0) return reinterpret_cast<T*>(cx.smem + p.sm.cs) + b * MEc;
+    return reinterpret_cast<T*>(p.cache) + ((long long)(job * p.U + b) * C + cx.c) * MEc;
+  }
+
+  // ---------------------------------------------------------------- first GEMM
+  // A = xln.  SA / CA: f32 rows of q|k|v (SA) or q (CA) + bias; FFN:
+  // T(gelu(. + bias)).  The output region aliases xln, so all warps finish
+  // their k-loop before any epilogue writes.
+  template <int U>
+  __device__ __forceinline__ static void gemm1(const JobParams& p, Ctx& cx, const uint8_t* slab0) {
+    constexpr int N = S::n1(U);
+    const float* bias = reinterpret_cast<const float*>(slab0) + 2 * E;
+    float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.xln);
+    T* hid = reinterpret_cast<T*>(cx.smem + p.sm.xln);
+    if constexpr (BF) {
+      constexpr int NT = N / 8, NTW = (NT + NCW - 1) / NCW;
+      float2 bv[NTW];
+#pragma unroll
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        bv[i] = (NT % NCW == 0 || nt < NT) ? *reinterpret_cast<const float2*>(bias + nt * 8 + 2 * (cx.lane & 3))
+                                            : make_float2(0.f, 0.f);
+      }
+      float acc[MT][NTW][4];
+      gemm_bf16<U, 0>(p, cx, reinterpret_cast<const __nv_bfloat16*>(cx.smem + p.sm.xln), S::lda, slab0, acc);
+      bar_compute();
+#pragma unroll
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        if (NT % NCW == 0 || nt < NT) {
+          const int n = nt * 8 + 2 * (cx.lane & 3);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
+              if (M % 16 == 0 || m < M) {
+                const float v0 = acc[mt][i][2 * h] + bv[i].x, v1 = acc[mt][i][2 * h + 1] + bv[i].y;
+                if constexpr (U == 2) {
+                  *reinterpret_cast<__nv_bfloat162*>(hid + m * S::ldh + n) =
+                      __floats2bfloat162_rn(gelu_erf(v0), gelu_erf(v1));
+                } else {
+                  *reinterpret_cast<float2*>(g1 + m * S::ldg1 + n) = make_float2(v0, v1);
+                }
+              }
+            }
+        }
+      }
+    } else {
+      constexpr int NOUT = M * N, NO = (NOUT + NCT - 1) / NCT;
+      float bv[F32_MAXO];
+#pragma unroll
+      for (int i = 0; i < F32_MAXO; ++i) {
+        const int o = cx.tid + i * NCT;
+        bv[i] = (i < NO && o < NOUT) ? bias[o % N] : 0.f;
+      }
+      float acc[F32_MAXO];
+      gemm_f32<U, 0>(p, cx, reinterpret_cast<const float*>(cx.smem + p.sm.xln), S::lda, slab0, acc);
+      bar_compute();
+#pragma unroll
+      for (int i = 0; i < NO; ++i) {
+        const int o = cx.tid + i * NCT;
+        if (o < NOUT) {
+          const int m = o / N, n = o % N;
+          const float v = acc[i] + bv[i];
+          if constexpr (U == 2)
+            hid[m * S::ldh + n] = from_f<T>(gelu_erf(v));
+          else
+            g1[m * S::ldg1 + n] = v;
+        }
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- second GEMM
+  // Partial sums over this CTA's K slice, staged in ablk in block layout
+  // (block r = columns r*Ec.. destined for CTA r).  Staging into ablk is safe
+  // block by block: CTA r's next gather writes only block r of ablk, and r can
+  // only send it after it has received this CTA's partial block r.
+  template <int U>
+  __device__ __forceinline__ static void gemm2(const JobParams& p, Ctx& cx) {
+    const T* A = reinterpret_cast<const T*>(cx.smem + (U == 2 ? p.sm.xln : p.sm.oc));
+    constexpr int lda = U == 2 ? S::ldh : S::ldo;
+    float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
+    if constexpr (BF) {
+      constexpr int NT = E / 8, NTW = (NT + NCW - 1) / NCW;
+      float acc[MT][NTW][4];
+      gemm_bf16<U, 1>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, ring_acquire(p, cx), acc);
+#pragma unroll
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        if (NT % NCW == 0 || nt < NT) {
+          const int n = nt * 8 + 2 * (cx.lane & 3);
+          float* dst = stage + (n >> S::lEc) * S::blk + (n & (Ec - 1));
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
+              if (M % 16 == 0 || m < M)
+                *reinterpret_cast<float2*>(dst + (m << S::lEc)) = make_float2(acc[mt][i][2 * h], acc[mt][i][2 * h + 1]);
+            }
+        }
+      }
+    } else {
+      constexpr int NOUT = M * E, NO = (NOUT + NCT - 1) / NCT;
+      float acc[F32_MAXO];
+      gemm_f32<U, 1>(p, cx, reinterpret_cast<const float*>(A), lda, ring_acquire(p, cx), acc);
+#pragma unroll
+      for (int i = 0; i < NO; ++i) {
+        const int o = cx.tid + i * NCT;
+        if (o < NOUT) {
+          const int m = o / E, n = o % E;
+          stage[(n >> S::lEc) * S::blk + (m << S::lEc) + (n & (Ec - 1))] = acc[i];
+        }
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- attention
+  // Scores: one (query row, key) pair per thread, softmax over groups of G
+  // lanes (G = keys rounded up to a power of two), probabilities to pb; then
+  // one output (row, dim of this CTA's slice) per thread.  SA: causal over the
+  // H tokens of the same sample (q, k of the CTA's head and v of its slice are
+  // rows of the first GEMM's output).  CA: the 1 + n_obs memory tokens in kvs.
+  template <int U>
+  __device__ __forceinline__ static void attention(const JobParams& p, Ctx& cx, const float* kvs) {
+    const float* g1 = reinterpret_cast<const float*>(cx.smem + p.sm.xln);
+    float* pb = reinterpret_cast<float*>(cx.smem + p.sm.pb);
+    T* oc = reinterpret_cast<T*>(cx.smem + p.sm.oc);
+    const float scale = rsqrtf((float)dh);
+    const int nk = U == 0 ? H : p.Cm;
+    int lG = 0;
+    while ((1 << lG) < nk) ++lG;
+    const int G = 1 << lG;
+    const int rows_per_pass = NCT >> lG;
+    for (int base = 0; base < M; base += rows_per_pass) {
+      const int m = base + (cx.tid >> lG), j = cx.tid & (G - 1);
+      float s = -INFINITY;
+      const bool live = m < M && j < nk;
+      if (live) {
+        const int i = m >> S::lH, qi = m & (H - 1);
+        if (U != 0 || j <= qi) {
+          const float4* q4 = reinterpret_cast<const float4*>(g1 + m * S::ldg1);
+          const float4* k4 = U == 0 ? reinterpret_cast<const float4*>(g1 + ((i << S::lH) + j) * S::ldg1 + dh)
+                                    : reinterpret_cast<const float4*>(kvs + (i * p.Cm + j) * S::kvw);
+          float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll
+          for (int e = 0; e < dh / 4; ++e) {
+            const float4 a = q4[e], b = k4[e];
+            d0 = fmaf(a.x, b.x, d0);
+            d1 = fmaf(a.y, b.y, d1);
+            d2 = fmaf(a.z, b.z, d2);
+            d3 = fmaf(a.w, b.w, d3);
+          }
+          s = ((d0 + d1) + (d2 + d3)) * scale;
+        }
+      }
+      const float mx = group_max_dyn(s, G);
+      const float ex = s == -INFINITY ? 0.f : __expf(s - mx);
+      const float sum = group_sum_dyn(ex, G);
+      if (live) pb[m * PLD + j] = ex * __frcp_rn(sum);
+    }
+    bar_compute();
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) {
+      const int o = cx.tid + k * NCT;
+      if (MEc % NCT == 0 || o < MEc) {
+        const int m = o >> S::lEc, e = o & (Ec - 1);
+        const int i = m >> S::lH, qi = m & (H - 1);
+        const float* prow = pb + m * PLD;
+        float a0 = 0.f, a1 = 0.f;
+        if constexpr (U == 0) {
+          const float* v = g1 + (i << S::lH) * S::ldg1 + 2 * dh + e;
+#pragma unroll
+          for (int j = 0; j < H; j += 2) {
+            if (j <= qi) a0 = fmaf(prow[j], v[j * S::ldg1], a0);
+            if (j + 1 <= qi) a1 = fmaf(prow[j + 1], v[(j + 1) * S::ldg1], a1);
+          }
+        } else {
+          const float* v = kvs + (i * p.Cm) * S::kvw + dh + e;
+          for (int j = 0; j < p.Cm; ++j) a0 = fmaf(prow[j], v[j * S::kvw], a0);
+        }
+        oc[m * S::ldo + e] = from_f<T>(a0 + a1);
+      }
+    }
+  }
+
+  // stage the memory tokens' keys (this CTA's head) and values (its slice) of
+  // layer l at step t into kvs (cp.async; waited before use)
+  __device__ __forceinline__ static void stage_kv(const JobParams& p, Ctx& cx, int l, int t, float* kvs) {
+    if (cx.kv_i >= 0) {
+      const float* src = cx.kv_base + (cx.kv_tok == 0 ? (long long)t * p.L * 2 * E : 0ll) + l * 2 * E + cx.kv_src;
+      cp_async16(kvs + cx.kv_dst, src);
+    }
+  }
+
+  // per-job part of the staging map (which sample's observation rows this thread copies)
+  __device__ __forceinline__ static void stage_kv_job(const JobParams& p, Ctx& cx, int sample0) {
+    if (cx.kv_i < 0) return;
+    const int s = min(sample0 + cx.kv_i, p.samples - 1);
+    cx.kv_base = cx.kv_tok == 0 ? p.kv_time
+                                : p.kv_obs + ((long long)(s % p.obs_mod) * p.n_obs + (cx.kv_tok - 1)) * p.L * 2 * E;
+  }
+
+  // ---------------------------------------------------------------- one refreshed unit (Eq. 1, (b,t) in S)
+  template <int U>
+  __device__ __forceinline__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0) {
+    const int l = b / 3;
+    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
+    float* ablk = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
+    float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
+    if constexpr (U == 1) {
+      if (p.kv_slots == 1) stage_kv(p, cx, l, t, kvs);
+      else kvs += l * S::G * p.Cm * S::kvw;
+    }
+    // exchange 1: every CTA receives every CTA's columns of a.  ablk is read by
+    // LayerNorm below; CTA r sends into it again only after this CTA's partial
+    // sums (sent after the first GEMM) reached r.
+    fence_proxy_async();
+    bar_compute();                     // ac final for this unit
+    send_blocks(cx, ac, 0, ablk, cx.xg);
+    exchange_wait(p, cx, cx.xg, cx.pg);
+    // slab 0 of piece 1: [gamma | beta | first bias | second-GEMM bias slice | k-tiles]
+    const uint8_t* s1 = ring_acquire(p, cx);
+    const float* hdr = reinterpret_cast<const float*>(s1);
+    float b2[EPT];
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) b2[k] = hdr[2 * E + S::n1(U) + ((cx.tid + k * NCT) & (Ec - 1))];
+    layernorm_rows(cx, ablk, reinterpret_cast<T*>(cx.smem + p.sm.xln), hdr, hdr + E);
+    bar_compute();
+    gemm1<U>(p, cx, s1);
+    if constexpr (U == 1) cp_async_wait_all();
+    bar_compute();
+    if constexpr (U != 2) {
+      attention<U>(p, cx, kvs);
+      bar_compute();
+    }
+    gemm2<U>(p, cx);
+    // exchange 2: block r of the staged partial sums goes to CTA r.  rs is read
+    // below; CTA r sends into it again only after this CTA's next gather.
+    fence_proxy_async();
+    bar_compute();
+    send_blocks(cx, ablk, S::blk, reinterpret_cast<const float*>(cx.smem + p.sm.rs), cx.xr);
+    exchange_wait(p, cx, cx.xr, cx.pr);
+    // finish this CTA's columns: r = sum of partials + bias; c_b <- r; a += r
+    const float* rs = reinterpret_cast<const float*>(cx.smem + p.sm.rs);
+    T* cache = cache_ptr(p, cx, job, b);
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) {
+      const int e = cx.tid + k * NCT;
+      if (MEc % NCT == 0 || e < MEc) {
+        float part[C];
+#pragma unroll
+        for (int cc = 0; cc < C; ++cc) part[cc] = rs[cc * S::blk + e];
+#pragma unroll
+        for (int w = C / 2; w > 0; w >>= 1)
+#pragma unroll
+          for (int cc = 0; cc < w; ++cc) part[cc] += part[cc + w];
+        const float r = part[0] + b2[k];
+        cache[e] = from_f<T>(r);
+        ac[e] += r;
+        if (p.trace) {
+          const int m = e >> S::lEc, j = e & (Ec - 1);
+          const int s = sample0 + (m >> S::lH);
+          if (s < p.samples)
+            p.trace[(((long long)t * p.U + b) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] = r;
+        }
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- skipped units b0..b1-1: a += c_b (in unit order)
+  __device__ __forceinline__ static void skip_run(const JobParams& p, Ctx& cx, int job, int b0, int b1, int t,
+                                                  int sample0, uint64_t valid) {
+    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
+    // units of the run whose cache holds a value (bit k = unit b0 + k)
+    const uint32_t live = (uint32_t)((valid >> b0) & ((1ull << (b1 - b0)) - 1ull));
+    const T* cb = cache_ptr(p, cx, job, b0);
+    const int cstride = p.sm.cs >= 0 ? MEc : C * MEc;
+#pragma unroll
+    for (int k = 0; k < EPT; ++k) {
+      const int e = cx.tid + k * NCT;
+      if (MEc % NCT == 0 || e < MEc) {
+        float cv[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) cv[q] = ((live >> q) & 1u) ? to_f<T>(cb[q * cstride + e]) : 0.f;
+        float a = ac[e];
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          if ((live >> q) & 1u) a += cv[q];
+        ac[e] = a;
+        if (p.trace) {
+          const int m = e >> S::lEc, j = e & (Ec - 1);
+          const int s = sample0 + (m >> S::lH);
+          if (s < p.samples) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              if (b0 + q < b1)
+                p.trace[(((long long)t * p.U + b0 + q) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] =
+                    cv[q];
+          }
+        }
+      }
+    }
+  }
+
+  // ---------------------------------------------------------------- output head + sampler step
+  __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t, const float4 tab0,
+                                                   const float4 tab1) {
+    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
+    float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
+    const float* z = reinterpret_cast<const float*>(cx.smem + p.sm.z);
+    const float* cst = reinterpret_cast<const float*>(cx.smem + p.sm.cst);
+    const float* lnf_g = cst + p.A * Ec + Ec + H * Ec;
+    const float* lnf_b = lnf_g + E;
+    const float* head_b = lnf_b + E;
+    const float* hw = p.headw_smem ? head_b + ((p.A + 3) & ~3) : p.vec + p.v_headw;
+    const float* hb;
+    if (p.head_sep) {
+      // double-buffered by step parity: source, landing blocks and barrier
+      const int par = t & 1;
+      float* src = reinterpret_cast<float*>(cx.smem + p.sm.hsrc) + par * MEc;
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) {
+        const int e = cx.tid + k * NCT;
+        if (MEc % NCT == 0 || e < MEc) src[e] = ac[e];
+      }
+      hb = reinterpret_cast<const float*>(cx.smem + p.sm.hblk) + par * C * S::blk;
+      fence_proxy_async();
+      bar_compute();
+      send_blocks(cx, src, 0, hb, cx.xh + par);
+      exchange_wait(p, cx, cx.xh + par, par ? cx.ph1 : cx.ph0);
+    } else {
+      hb = reinterpret_cast<const float*>(cx.smem + p.sm.ablk);
+      fence_proxy_async();
+      bar_compute();
+      send_blocks(cx, ac, 0, hb, cx.xg);
+      exchange_wait(p, cx, cx.xg, cx.pg);
+    }
+    cp_async_wait_all();
+    bar_compute();
+    const float inv_sa = tab0.x, s1 = tab0.y, cx0 = tab0.z, cxt = tab0.w, sig = tab1.x;
+    const float sab = tab1.y, sabp = tab1.z, s1p = tab1.w;
+    constexpr int NV = E / 64;
+    const int half = cx.lane >> 4, hl = cx.lane & 15;
+#pragma unroll
+    for (int m0 = 0; m0 < M; m0 += 2 * NCW) {
+      if (M % (2 * NCW) == 0 || m0 + cx.warp * 2 < M) {
+        const int m = m0 + cx.warp * 2 + half;
+        float4 v[NV];
+        float s = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+          const int col = 4 * (hl + 16 * j);
+          v[j] = *reinterpret_cast<const float4*>(hb + (col >> S::lEc) * S::blk + (m << S::lEc) + (col & (Ec - 1)));
+          s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+          s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) {
+          s += __shfl_xor_sync(0xffffffffu, s, o);
+          s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+        }
+        const float mean = s * S::invE;
+        const float rstd = rsqrtf(fmaxf(s2 * S::invE - mean * mean, 0.f) + 1e-5f);
+        // normalised values of this lane's columns, then one reduced dot per action dim
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+          const int col = 4 * (hl + 16 * j);
+          v[j].x = (v[j].x - mean) * rstd * lnf_g[col] + lnf_b[col];
+          v[j].y = (v[j].y - mean) * rstd * lnf_g[col + 1] + lnf_b[col + 1];
+          v[j].z = (v[j].z - mean) * rstd * lnf_g[col + 2] + lnf_b[col + 2];
+          v[j].w = (v[j].w - mean) * rstd * lnf_g[col + 3] + lnf_b[col + 3];
+        }
+        float eps = 0.f;
+        for (int a = 0; a < p.A; ++a) {
+          float part = 0.f;
+#pragma unroll
+          for (int j = 0; j < NV; ++j) {
+            const float* w = hw + 4 * (hl + 16 * j) * p.A + a;
+            part = fmaf(v[j].x, w[0], part);
+            part = fmaf(v[j].y, w[p.A], part);
+            part = fmaf(v[j].z, w[2 * p.A], part);
+            part = fmaf(v[j].w, w[3 * p.A], part);
+          }
+          const float e = group_sum<16>(part);
+          if (hl == a) eps = e + head_b[a];
+        }
+        if (hl < p.A) {
+          const float xv = x[m * p.A + hl];
+          float x0 = (xv - s1 * eps) * inv_sa;
+          x0 = fminf(1.0f, fmaxf(-1.0f, x0));
+          float xn;
+          if (p.sampler == 0) {
+            xn = cx0 * x0 + cxt * xv + sig * z[m * p.A + hl];
+          } else {
+            xn = sabp * x0 + s1p * ((xv - sab * x0) / s1);
+          }
+          x[m * p.A + hl] = xn;
+        }
+      }
+    }
+    if (!p.head_sep) csync(p, cx);                    // ablk is the next gather's landing zone
+    bar_compute();
+  }
+
+  // ---------------------------------------------------------------- the compute warps' job loop
+  __device__ __forceinline__ static void compute(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
+    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
+    float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
+    float* z = reinterpret_cast<float*>(cx.smem + p.sm.z);
+    uint64_t* sch = reinterpret_cast<uint64_t*>(cx.smem + p.sm.sch);
+    float* kvs = reinterpret_cast<float*>(cx.smem + p.sm.kvs);
+    const float* cst = reinterpret_cast<const float*>(cx.smem + p.sm.cst);
+    const float* c_inw = cst;
+    const float* c_inb = cst + p.A * Ec;
+    const float* c_pos = c_inb + Ec;
+    for (int job = cid; job < p.n_jobs; job += ncl) {
+      const int sample0 = job * S::G;
+      const int s_first = min(sample0, p.samples - 1);
+      const uint8_t* Sl = p.S + (long long)(s_first / p.per_sched) * p.S_stride;
+      // the job's lattice as one refresh mask per step, and the initial x
+      for (int t = cx.tid; t < p.T; t += NCT) {
+        uint64_t mask = 0;
+        for (int b = 0; b < p.U; ++b) {
+          const int row = (p.S_rows == p.U) ? b : b / 3;
+          if (Sl[row * p.T + t] != 0) mask |= 1ull << b;
+        }
+        sch[t] = mask;
+      }
+      for (int v = cx.tid; v < M * p.A; v += NCT) {
+        const int m = v / p.A;
+        const int s = min(sample0 + (m >> S::lH), p.samples - 1);
+        x[v] = p.noise[((long long)(s % p.obs_mod) * H + (m & (H - 1))) * p.A + (v % p.A)];
+      }
+      stage_kv_job(p, cx, sample0);
+      bar_compute();
+      uint64_t valid = 0;
+      for (int t = 0; t < p.T; ++t) {
+        const uint64_t refresh = sch[t] | (p.force ? ~valid : 0ull);
+        // sampler coefficients of this step (used at the head)
+        const float4 tab0 = *reinterpret_cast<const float4*>(p.stab + t * 8);
+        const float4 tab1 = *reinterpret_cast<const float4*>(p.stab + t * 8 + 4);
+        // stage z_t (DDPM) and, when every layer has a slot, the memory keys/values
+        // of this step's refreshed cross-attention units
+        if (p.sampler == 0) {
+          const int per = H * p.A / 4;
+          for (int v = cx.tid; v < S::G * per; v += NCT) {
+            const int i = v / per, w = v - i * per;
+            const int s = min(sample0 + i, p.samples - 1);
+            cp_async16(z + i * H * p.A + 4 * w,
+                       p.noise + ((long long)(1 + t) * p.obs_mod + (s % p.obs_mod)) * H * p.A + 4 * w);
+          }
+        }
+        if (p.kv_slots > 1)
+          for (int l = 0; l < p.L; ++l)
+            if ((refresh >> (3 * l + 1)) & 1ull) stage_kv(p, cx, l, t, kvs + l * S::G * p.Cm * S::kvw);
+        // input embedding into this CTA's columns
+#pragma unroll
+        for (int k = 0; k < EPT; ++k) {
+          const int e = cx.tid + k * NCT;
+          if (MEc % NCT == 0 || e < MEc) {
+            const int m = e >> S::lEc, j = e & (Ec - 1);
+            float acc = 0.f;
+            for (int a = 0; a < p.A; ++a) acc = fmaf(x[m * p.A + a], c_inw[a * Ec + j], acc);
+            ac[e] = acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j];
+          }
+        }
+        int b = 0;
+        while (b < p.U) {
+          if ((refresh >> b) & 1ull) {
+            valid |= 1ull << b;
+            const int u = b % 3;
+            if (u == 0) unit<0>(p, cx, job, b, t, sample0);
+            else if (u == 1) unit<1>(p, cx, job, b, t, sample0);
+            else unit<2>(p, cx, job, b, t, sample0);
+            ++b;
+          } else {
+            int b1 = b + 1;
+            while (b1 < p.U && b1 - b < 8 && !((refresh >> b1) & 1ull)) ++b1;
+            skip_run(p, cx, job, b, b1, t, sample0, valid);
+            b = b1;
+          }
+        }
+        head_step(p, cx, t, tab0, tab1);
+      }
+      // write the finished chunk
+      if (cx.c == 0) {
+        for (int v = cx.tid; v < M * p.A; v += NCT) {
+          const int s = sample0 + v / (H * p.A);
+          if (s < p.samples) p.out[(long long)sample0 * H * p.A + v] = x[v];
+        }
+      }
+      bar_compute();
+    }
+  }
+};
+
+template <typename T, class S>
+__global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant__ JobParams p) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  Ctx cx;
+  cx.smem = smem;
+  cx.tid = threadIdx.x;
+  cx.warp = threadIdx.x >> 5;
+  cx.lane = threadIdx.x & 31;
+  cx.c = (int)cluster_ctarank();
+  cx.full = reinterpret_cast<uint64_t*>(smem + p.sm.bars);
+  cx.empty = cx.full + S::NSLOT;
+  cx.cbar = cx.full + 2 * S::NSLOT;
+  cx.xg = cx.cbar + 1;
+  cx.xr = cx.cbar + 2;
+  cx.xh = cx.cbar + 3;
+  cx.q = 0;
+  cx.cph = cx.pg = cx.pr = cx.ph0 = cx.ph1 = 0;
+  cx.dead = 0;
+  {
+    // staging map: chunk v = tid over [G][1+n_obs][k chunks (dh/4) | v chunks (Ec/4)]
+    constexpr int kq = S::dh / 4, per_tok = kq + S::Ec / 4;
+    const int v = threadIdx.x;
+    cx.kv_i = -1;
+    cx.kv_base = nullptr;
+    if (v < S::G * p.Cm * per_tok) {
+      const int i = v / (p.Cm * per_tok);
+      const int rem = v - i * p.Cm * per_tok;
+      const int tok = rem / per_tok, w = rem - tok * per_tok;
+      const int head = (cx.c * S::Ec) / S::dh;
+      cx.kv_i = i;
+      cx.kv_tok = tok;
+      cx.kv_src = w < kq ? head * S::dh + 4 * w : S::E + cx.c * S::Ec + 4 * (w - kq);
+      cx.kv_dst = (i * p.Cm + tok) * S::kvw + (w < kq ? 4 * w : S::dh + 4 * (w - kq));
+    }
+  }
+  const uint32_t cid = cluster_idx(), ncl = cluster_count();
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S::NSLOT; ++i) {
+      mbar_init(&cx.full[i], 1);
+      mbar_init(&cx.empty[i], NCW);
+    }
+    mbar_init(cx.cbar, S::C);
+    mbar_init(cx.xg, 1);
+    mbar_init(cx.xr, 1);
+    mbar_init(cx.xh, 1);
+    mbar_init(cx.xh + 1, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // zero the operand and exchange buffers once: padded rows and columns must read as 0
+  for (int v = threadIdx.x; v < (p.sm.ac - p.sm.ablk) / 16; v += NTHREADS)
+    reinterpret_cast<float4*>(smem + p.sm.ablk)[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+  // per-kernel constants: in_w[:, cols], in_b[cols], pos[:, cols], lnf_g, lnf_b, head_b, head_w
+  {
+    float* cst = reinterpret_cast<float*>(smem + p.sm.cst);
+    const int c0 = cx.c * S::Ec;
+    for (int v = threadIdx.x; v < p.A * S::Ec; v += NTHREADS)
+      cst[v] = p.vec[p.v_inw + (v / S::Ec) * S::E + c0 + (v % S::Ec)];
+    float* d = cst + p.A * S::Ec;
+    for (int v = threadIdx.x; v < S::Ec; v += NTHREADS) d[v] = p.vec[p.v_inb + c0 + v];
+    d += S::Ec;
+    for (int v = threadIdx.x; v < S::H * S::Ec; v += NTHREADS)
+      d[v] = p.vec[p.v_pos + (v / S::Ec) * S::E + c0 + (v % S::Ec)];
+    d += S::H * S::Ec;
+    for (int v = threadIdx.x; v < S::E; v += NTHREADS) {
+      d[v] = p.vec[p.v_lnfg + v];
+      d[S::E + v] = p.vec[p.v_lnfb + v];
+    }
+    d += 2 * S::E;
+    for (int v = threadIdx.x; v < p.A; v += NTHREADS) d[v] = p.vec[p.v_headb + v];
+    d += (p.A + 3) & ~3;
+    if (p.headw_smem)
+      for (int v = threadIdx.x; v < S::E * p.A; v += NTHREADS) d[v] = p.vec[p.v_headw + v];
+  }
+  __syncthreads();
+  hw_cluster_sync();
+  const bool bad = p.sched_err != nullptr && *p.sched_err != 0;
+  if (!bad) {
+    if (cx.warp == NCW) {
+      if (cx.lane == 0) Loop<T, S>::producer(p, cx, cid, ncl);
+      __syncwarp();
+    } else {
+      Loop<T, S>::compute(p, cx, cid, ncl);
+    }
+  }
+  __syncwarp();
+  hw_cluster_sync();
+}
+
+// Host side of one shape: the plan must agree with the compile-time constants.
+template <typename T, class S>
+bool shape_matches(const JobParams& p) {
+  return p.E == S::E && p.dh == S::dh && p.H == S::H && p.C == S::C && p.g == S::G && p.M == S::M &&
+         p.Mp == S::Mp && p.blk == S::blk && p.lda == S::lda && p.ldg1 == S::ldg1 && p.kvw == S::kvw &&
+         p.ldh == S::ldh && p.ldo == S::ldo && p.kp_o == S::kp_o && p.kp_h == S::kp_h && p.nslot == S::NSLOT &&
+         p.slot_bytes == S::SLOT && p.hdr1[0] == S::hdr1(0) && p.hdr1[1] == S::hdr1(1) && p.hdr1[2] == S::hdr1(2) &&
+         (int)sizeof(T) == S::ES;
+}
+
+template <typename T, class S>
+cudaError_t shape_prepare(int smem_bytes, int* max_clusters) {
+  cudaError_t e = cudaFuncSetAttribute(job_kernel<T, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  if (e != cudaSuccess) return e;
+  if (S::C > 8) {
+    e = cudaFuncSetAttribute(job_kernel<T, S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S::C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(S::C, 1, 1);
+  cfg.blockDim = dim3(NTHREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem_bytes;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaOccupancyMaxActiveClusters(max_clusters, job_kernel<T, S>, &cfg);
+}
+
+template <typename T, class S>
+cudaError_t shape_launch(const JobParams& p, int n_clusters, cudaStream_t s) {
+  if (!shape_matches<T, S>(p)) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S::C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(n_clusters * S::C, 1, 1);
+  cfg.blockDim = dim3(NTHREADS, 1, 1);
+  cfg.dynamicSmemBytes = p.sm.total;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, job_kernel<T, S>, p);
+}
+
+}  // namespace evo
