@@ -318,7 +318,7 @@ def run_ours(args, world, rank, local):
         "roofline": roof,
         "e2e": {"value": chunks / total_e2e, "unit": "chunks/s", "h2d_bytes_per_step": bytes_in,
                 "d2h_bytes_per_step": int(h_out.numel() * 4)},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": binding.LAUNCHES_PER_DENOISE * args.steps,
         "clocks": headline["clocks"],
         "launch": ev.launch_info(),
     }

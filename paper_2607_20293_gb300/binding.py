@@ -24,6 +24,12 @@ _FIELDS = ["n_layer", "n_emb", "n_head", "horizon", "action_dim", "n_obs", "obs_
            "train_steps", "sampler", "dtype", "empty_cache", "cluster", "job_samples", "debug_sync"]
 
 
+# kernels one evo_denoise call launches: the observation tokens' embedding, the
+# three condition GEMVs (MLP E->4E, 4E->E, per-layer memory keys/values) and
+# the denoising-loop kernel
+LAUNCHES_PER_DENOISE = 5
+
+
 class EvoConfig(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int32) for f in _FIELDS]
 
