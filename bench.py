@@ -23,6 +23,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -85,7 +86,7 @@ class Clocks:
     def __init__(self, index: int):
         self.proc = None
         self.index = index
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        self.path = os.path.join(tempfile.gettempdir(), f"evo_bench_clocks_{os.getpid()}_{index}.csv")
 
     def start(self):
         try:
@@ -243,11 +244,12 @@ def run_ours(args, world, rank, local):
         clocks = Clocks(local) if frac == head_frac else None
         if clocks:
             clocks.start()
-        steps, kern = [], []
+        steps, kern, launches = [], [], 0
         for _ in range(args.steps):
             ms, kms = one(S)
             steps.append(ms)
             kern.append(kms)
+            launches += ev.last_call()["kernels"]
         torch.cuda.synchronize()
         if dist:
             tdist.barrier()
@@ -256,7 +258,8 @@ def run_ours(args, world, rank, local):
         fl = ev.flops(S)
         rec = {"chunks_per_s": n * 1000.0 / statistics.mean(steps), "p50_ms": statistics.median(steps),
                "kernel_ms_mean": statistics.mean(kern), "flops_per_chunk": fl, "ms": steps, "kernel_ms": kern,
-               "e2e_ms": e2e, "clocks": clk, "alg_bytes": algorithmic_bytes(cfg, S, n), "S": S}
+               "e2e_ms": e2e, "clocks": clk, "alg_bytes": algorithmic_bytes(cfg, S, n), "S": S,
+               "launches": launches, "path": ev.last_call()["path"]}
         sweep[frac] = rec
         if frac == head_frac:
             headline = rec
@@ -288,7 +291,8 @@ def run_ours(args, world, rank, local):
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": recorded_traffic(args.workload),
                 "peak_source": "measured HBM copy" if "hbm_gbs" in peaks else "fallback"}
-    roof["kernel"] = "evo::job_kernel"
+    roof["kernel"] = ("batch-wide sequence (tcgen05 GEMMs + row/attention kernels)" if headline["path"] == "wide"
+                      else "evo::job_kernel")
     roof["algorithmic_per_launch"] = headline["flops_per_chunk"] * n if big else headline["alg_bytes"]
     roof["kernel_ms"] = kern_ms
     bytes_in = (obs.nbytes + noise.nbytes)
@@ -318,9 +322,9 @@ def run_ours(args, world, rank, local):
         "roofline": roof,
         "e2e": {"value": chunks / total_e2e, "unit": "chunks/s", "h2d_bytes_per_step": bytes_in,
                 "d2h_bytes_per_step": int(h_out.numel() * 4)},
-        "gpu_launches": binding.LAUNCHES_PER_DENOISE * args.steps,
+        "gpu_launches": headline["launches"],
         "clocks": headline["clocks"],
-        "launch": ev.launch_info(),
+        "launch": dict(ev.launch_info(), path=headline["path"]),
     }
     return line, cfg
 

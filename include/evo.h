@@ -72,6 +72,9 @@ typedef struct evo_config {
   int32_t cluster;      /* CTAs that cooperate on one job; 0 = choose */
   int32_t job_samples;  /* samples per job (rows = job_samples * horizon); 0 = choose */
   int32_t debug_sync;   /* 1: synchronize after each call and return the device status */
+  int32_t wide_rows;    /* batch-wide tensor-core path for calls of at least this many action-token
+                           rows (samples x horizon); 0 = 1024; < 0 = never.  bf16 with n_emb 256 or
+                           512, head size 64, horizon dividing 128, at most 7 observation tokens */
 } evo_config;
 
 /* Number of float32 values in the weight blob for cfg (0 if cfg is invalid).
@@ -103,7 +106,9 @@ evo_status evo_destroy(evo_handle* h);
  *   S      [S_rows][T] uint8 lattice, host or device memory.  S_rows = 3L (unit rows
  *          b = 3l + {0 SA, 1 CA, 2 FFN}) or L (row l covers the three units of layer l).
  *          A host lattice is validated before launch; a device lattice is checked on the
- *          device (EVO_ERR_SCHEDULE in the status word, outputs untouched).
+ *          device (EVO_ERR_SCHEDULE in the status word, outputs untouched), except on
+ *          the batch-wide path, which copies it to the host (one synchronisation) and
+ *          returns EVO_ERR_SCHEDULE before any launch.
  *   out    device [N][H][A]             final actions (normalised space, after T steps)
  */
 evo_status evo_denoise(evo_handle* h, const float* obs, const float* noise,
@@ -181,6 +186,11 @@ evo_status evo_get_status(evo_handle* h);
  * clusters resident at once, dynamic shared memory per CTA (bytes). */
 evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* job_samples,
                                int32_t* max_clusters, int32_t* smem_bytes);
+
+/* How the handle's last call ran: path 0 = one cluster per job (the persistent
+ * denoising-loop kernel), 1 = batch-wide (step-synchronous over all samples,
+ * tensor-core GEMMs); kernels = kernel launches of that call. */
+evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels);
 
 const char* evo_status_string(evo_status s);
 

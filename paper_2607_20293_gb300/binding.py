@@ -21,13 +21,7 @@ DTYPES = {"fp32": 0, "bf16": 1}
 EMPTY = {"zero": 0, "force": 1}
 
 _FIELDS = ["n_layer", "n_emb", "n_head", "horizon", "action_dim", "n_obs", "obs_dim", "n_steps",
-           "train_steps", "sampler", "dtype", "empty_cache", "cluster", "job_samples", "debug_sync"]
-
-
-# kernels one evo_denoise call launches: the observation tokens' embedding, the
-# three condition GEMVs (MLP E->4E, 4E->E, per-layer memory keys/values) and
-# the denoising-loop kernel
-LAUNCHES_PER_DENOISE = 5
+           "train_steps", "sampler", "dtype", "empty_cache", "cluster", "job_samples", "debug_sync", "wide_rows"]
 
 
 class EvoConfig(ctypes.Structure):
@@ -67,6 +61,7 @@ def load() -> ctypes.CDLL:
         "evo_set_profile_events": (I32, [P, P, P]),
         "evo_get_launch_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(I32),
                                       ctypes.POINTER(I32)]),
+        "evo_get_last_call": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I64)]),
         "evo_status_string": (ctypes.c_char_p, [I32]),
     }
     for name, (res, args) in sig.items():
@@ -87,11 +82,11 @@ def _check(code: int, what: str):
 
 
 def make_config(cfg: dict, cluster: int = 0, job_samples: int = 0, empty: str = "zero",
-                debug_sync: bool = False) -> EvoConfig:
+                debug_sync: bool = False, wide_rows: int = 0) -> EvoConfig:
     return EvoConfig(cfg["n_layer"], cfg["n_emb"], cfg["n_head"], cfg["horizon"], cfg["action_dim"],
                      cfg["n_obs"], cfg["obs_dim"], cfg["n_steps"], cfg["train_steps"],
                      SAMPLERS[cfg["sampler"]], DTYPES[cfg["dtype"]], EMPTY[empty], cluster, job_samples,
-                     int(debug_sync))
+                     int(debug_sync), wide_rows)
 
 
 def weight_names(cfg: dict) -> list[str]:
@@ -155,10 +150,10 @@ class Evo:
     """One evo_handle: packed weights, caches and workspace on the current GPU."""
 
     def __init__(self, cfg: dict, weights: dict, max_batch: int, cluster: int = 0, job_samples: int = 0,
-                 empty: str = "zero", debug_sync: bool = False):
+                 empty: str = "zero", debug_sync: bool = False, wide_rows: int = 0):
         lib = load()
         self.cfg = dict(cfg)
-        self._c = make_config(cfg, cluster, job_samples, empty, debug_sync)
+        self._c = make_config(cfg, cluster, job_samples, empty, debug_sync, wide_rows)
         self._blob = pack_blob(cfg, weights)
         h = ctypes.c_void_p()
         _check(lib.evo_create(self._blob.ctypes.data, self._blob.size, ctypes.byref(self._c), max_batch,
@@ -181,6 +176,12 @@ class Evo:
         v = [ctypes.c_int32() for _ in range(4)]
         _check(load().evo_get_launch_info(self._h, *[ctypes.byref(x) for x in v]), "evo_get_launch_info")
         return dict(cluster=v[0].value, job_samples=v[1].value, max_clusters=v[2].value, smem_bytes=v[3].value)
+
+    def last_call(self) -> dict:
+        """path of the last call ("cluster" or "wide") and the kernels it launched"""
+        path, k = ctypes.c_int32(), ctypes.c_int64()
+        _check(load().evo_get_last_call(self._h, ctypes.byref(path), ctypes.byref(k)), "evo_get_last_call")
+        return dict(path="wide" if path.value == 1 else "cluster", kernels=k.value)
 
     def denoise(self, obs, noise, S, out=None, stream=None, trace=None):
         import torch

@@ -58,6 +58,11 @@ struct evo_handle {
   cudaStream_t last_stream = nullptr;
   cudaEvent_t prof_start = nullptr, prof_stop = nullptr;
   int woff[W_COUNT];
+  // batch-wide path (null when the configuration has none)
+  WideState* wide = nullptr;
+  long long wide_rows = 1024;
+  int last_path = 0;
+  long long last_kernels = 0;
 };
 
 namespace {
@@ -363,6 +368,7 @@ evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* j
 
 evo_status evo_destroy(evo_handle* h) {
   if (!h) return EVO_ERR_ARG;
+  wide_destroy(h->wide);
   cudaFree(h->wf32);
   cudaFree(h->woff_d);
   cudaFree(h->wpack);
@@ -586,6 +592,12 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   if (cudaMalloc(&h->pop_x, cap_samples * H * A * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMallocHost(&h->stage, h->sched_cap) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaEventCreateWithFlags(&h->stage_ev, cudaEventDisableTiming) != cudaSuccess) return fail(EVO_ERR_CUDA);
+  if (cfg->wide_rows >= 0 && wide_supported(cfg)) {
+    // every call's rows (population: (P+1) * N_obs samples) and lattices fit
+    const int ws = wide_create(&h->wide, cfg, weights, h->wf32, h->woff, (long long)max_batch * H, max_batch + 1);
+    if (ws == EVO_ERR_OOM || ws == EVO_ERR_CUDA) return fail((evo_status)ws);
+    if (cfg->wide_rows > 0) h->wide_rows = cfg->wide_rows;
+  }
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(EVO_ERR_CUDA);
 
   p.stab = h->stab;
@@ -637,6 +649,9 @@ evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int row
   return EVO_OK;
 }
 
+// kernels of the observation-condition path per call (embedding + three GEMVs)
+constexpr int COND_KERNELS = 4;
+
 cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, int shape = -1) {
   if (h->prof_start && h->prof_stop) {
     cudaError_t e = cudaEventRecord(h->prof_start, st);
@@ -644,6 +659,8 @@ cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, int 
   }
   cudaError_t e = launch_job(shape >= 0 ? shape : h->shape, p, std::min(p.n_jobs, h->max_clusters), st);
   if (e != cudaSuccess) return e;
+  h->last_path = 0;
+  h->last_kernels = COND_KERNELS + 1 + (p.sched_err ? 1 : 0);
   if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
   return cudaSuccess;
 }
@@ -655,12 +672,68 @@ evo_status finish(evo_handle* h, cudaStream_t st) {
   return EVO_OK;
 }
 
+// Stage n_sched lattices for the batch-wide path, which needs them on the host
+// as well: a device lattice is copied back (one synchronisation) and checked there.
+evo_status stage_wide(evo_handle* h, const uint8_t* S, int n_sched, int rows, bool add_ones, cudaStream_t st) {
+  const size_t bytes = (size_t)rows * h->T * n_sched;
+  std::vector<uint8_t> host;
+  if (is_device_ptr(S)) {
+    host.resize(bytes);
+    EVO_CUDA(cudaMemcpyAsync(host.data(), S, bytes, cudaMemcpyDeviceToHost, st));
+    EVO_CUDA(cudaStreamSynchronize(st));
+    S = host.data();
+  }
+  const int* err = nullptr;
+  return stage_schedules(h, S, n_sched, rows, add_ones, st, &err);   // host lattice: validated, cached
+}
+
+cudaError_t launch_wide(evo_handle* h, const float* noise, float* out, int samples, int per_sched, int n_sched,
+                        int S_rows, cudaStream_t st) {
+  WideCall c{};
+  c.noise = noise;
+  c.out = out;
+  c.kv_obs = h->kv_obs;
+  c.kv_time = h->kv_time;
+  c.stab = h->stab;
+  c.samples = samples;
+  c.per_sched = per_sched;
+  c.obs_mod = per_sched;
+  c.S_host = h->last_sched.data();
+  c.S_dev = h->sched;
+  c.n_sched = n_sched;
+  c.S_rows = S_rows;
+  c.status = h->status;
+  c.st = st;
+  if (h->prof_start && h->prof_stop) {
+    const cudaError_t e = cudaEventRecord(h->prof_start, st);
+    if (e != cudaSuccess) return e;
+  }
+  const cudaError_t e = wide_run(h->wide, c);
+  if (e != cudaSuccess) return e;
+  h->last_path = 1;
+  h->last_kernels = COND_KERNELS + wide_last_launches(h->wide);
+  if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
+  return cudaSuccess;
+}
+
+bool use_wide(const evo_handle* h, long long samples) {
+  return h->wide && samples * h->H >= h->wide_rows && samples * h->H <= wide_rows_capacity(h->wide);
+}
+
 evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int S_rows, int N, float* out,
                float* trace, void* stream) {
   if (!h || !obs || !noise || !S || !out) return EVO_ERR_ARG;
   if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
   if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (!trace && use_wide(h, N)) {
+    const evo_status s = stage_wide(h, S, 1, S_rows, false, st);
+    if (s != EVO_OK) return s;
+    EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
+                             h->cond_scratch, h->kv_obs, st));
+    EVO_CUDA(launch_wide(h, noise, out, N, N, 1, S_rows, st));
+    return finish(h, st);
+  }
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
@@ -773,6 +846,19 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   if (samples > h->max_batch) return EVO_ERR_SHAPE;
   if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int HA = h->H * h->A;
+  if (use_wide(h, samples)) {
+    const evo_status s = stage_wide(h, S_pop, P, S_rows, true, st);
+    if (s != EVO_OK) return s;
+    EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
+                             h->cond_scratch, h->kv_obs, st));
+    EVO_CUDA(launch_wide(h, noise, h->pop_x, (int)samples, N_obs, P + 1, S_rows, st));
+    EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
+    h->last_kernels += 1;
+    if (out_actions)
+      EVO_CUDA(cudaMemcpyAsync(out_actions, h->pop_x, (size_t)P * N_obs * HA * 4, cudaMemcpyDeviceToDevice, st));
+    return finish(h, st);
+  }
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S_pop, P, S_rows, true, st, &err);
   if (s != EVO_OK) return s;
@@ -811,8 +897,8 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   p.out = h->pop_x;
   p.trace = nullptr;
   EVO_CUDA(launch_loop(h, p, st, shape));
-  const int HA = h->H * h->A;
   EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
+  h->last_kernels += 1;
   if (out_actions)
     EVO_CUDA(cudaMemcpyAsync(out_actions, h->pop_x, (size_t)P * N_obs * HA * 4, cudaMemcpyDeviceToDevice, st));
   return finish(h, st);
@@ -822,6 +908,13 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
   if (!h || (start == nullptr) != (stop == nullptr)) return EVO_ERR_ARG;
   h->prof_start = reinterpret_cast<cudaEvent_t>(start);
   h->prof_stop = reinterpret_cast<cudaEvent_t>(stop);
+  return EVO_OK;
+}
+
+evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels) {
+  if (!h) return EVO_ERR_ARG;
+  if (path) *path = h->last_path;
+  if (kernels) *kernels = h->last_kernels;
   return EVO_OK;
 }
 

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
+#include "evo.h"
+
 namespace evo {
 
 constexpr int NCW = 8;              // compute warps per CTA
@@ -100,6 +102,29 @@ cudaError_t launch_obs_cond(const float* wf32, const int* woff_dev, const int* w
                             int n_obs, int D, int L, int E, float* scratch, float* kv_obs, cudaStream_t s);
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s);
 cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev, cudaStream_t s);
+
+// batch-wide path (evo_wide.cu)
+struct WideState;
+struct WideCall {
+  const float* noise;             // [n_noise][obs_mod][H][A]
+  float* out;                     // [samples][H][A]: running x, final actions
+  const float* kv_obs;            // [obs_mod][n_obs][L][2E]
+  const float* kv_time;           // [T][L][2E]
+  const float* stab;              // [T][8]
+  int samples, per_sched, obs_mod;
+  const uint8_t* S_host;          // [n_sched][S_rows][T], validated
+  const uint8_t* S_dev;           // the same lattices on the device
+  int n_sched, S_rows;
+  int* status;
+  cudaStream_t st;
+};
+bool wide_supported(const evo_config* c);
+int wide_create(WideState** out, const evo_config* c, const float* weights, const float* wf32_dev, const int* woff,
+                long long max_rows, int max_sched);   // evo_status
+void wide_destroy(WideState* w);
+long long wide_rows_capacity(const WideState* w);
+long long wide_last_launches(const WideState* w);
+cudaError_t wide_run(WideState* w, const WideCall& c);
 
 // offsets (in floats) of the named tensors inside the float32 weight blob
 enum WOff {

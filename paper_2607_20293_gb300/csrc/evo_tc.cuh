@@ -1,0 +1,301 @@
+// Tensor-core GEMM of the batch-wide path: C[rows][N] = A[rows][K] . B[N][K]^T
+// on the fifth-generation tensor cores (tcgen05), bf16 operands, fp32
+// accumulation in tensor memory, with the epilogues the denoiser needs fused.
+//
+// One CTA computes one BM x BN tile:
+//   * warp 0, one lane: TMA producer.  Tiles of A (BM x 64) and B (BN x 64)
+//     land in a ring of STAGES shared-memory stages with the 128-byte swizzle
+//     (cp.async.bulk.tensor + mbarrier transaction counts);
+//   * warp 1, one lane: MMA issuer.  Four tcgen05.mma (K = 16 each) per stage
+//     into one TMEM accumulator of BN columns; tcgen05.commit frees the stage
+//     when the MMAs that read it are done, and signals the epilogue at the end;
+//   * all four warps: epilogue.  Warp w owns TMEM lanes (= tile rows)
+//     32w..32w+31 and reads 32 columns at a time with tcgen05.ld.
+// BM = 128, BN = 128 and three stages (97 KB of shared memory, 128 TMEM
+// columns) let two CTAs share an SM, so one CTA's epilogue overlaps the other's
+// main loop.
+//
+// Every wait on an mbarrier is bounded: on expiry the thread records
+// ST_TIMEOUT in the status word and carries on, so the kernel always ends.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include "evo_internal.h"
+
+namespace evo {
+namespace tc {
+
+constexpr int BM = 128, BN = 128, BK = 64, STAGES = 3;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 128;   // alignment slack, stages, barriers
+constexpr long long TC_WAIT_LIMIT = 1ll << 26;                  // polls before a wait gives up
+
+enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2 };
+
+struct GemmArgs {
+  int K;                      // multiple of BK
+  int b_row0;                 // first row of B (its tensor map spans every layer's matrices)
+  const float* bias;          // [N] fp32
+  __nv_bfloat16* out;         // EPI_BF16 / EPI_GELU_BF16: out[row * ldo + n]
+  int ldo;
+  float* resid;               // EPI_RESID: residual stream [rows][ldr] fp32, += r
+  __nv_bfloat16* cache;       // EPI_RESID: unit cache [rows][ldr], <- bf16(r)
+  int ldr;
+  int rows;                   // real rows; rows >= this are padding
+  // refresh gate (null: every row refreshes): row -> sample row / H -> lattice
+  // (sample / per_sched); refresh = S[lattice * S_stride + srow * T + t]
+  const uint8_t* S;
+  long long S_stride;
+  int srow, T, t, H, per_sched, force;
+  int* status;
+};
+
+// ---------------------------------------------------------------- PTX wrappers
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init1(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// bounded wait for the phase of `parity` to complete
+__device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, int* status) {
+  const uint32_t a = su32(bar);
+  if (mbar_test(a, parity)) return;
+  for (long long i = 0; i < TC_WAIT_LIMIT; ++i) {
+    if (mbar_test(a, parity)) return;
+    if (i > 64) __nanosleep(32);
+  }
+  atomicOr(status, ST_TIMEOUT);
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(su32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(su32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major operand in 128-byte-swizzled rows
+// (8-row groups 1024 bytes apart), the layout a SWIZZLE_128B TMA box of 64
+// bf16 columns produces.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);      // start address
+  d |= (uint64_t)1 << 16;                         // leading byte offset (unused with this swizzle)
+  d |= (uint64_t)(1024 >> 4) << 32;               // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;                         // descriptor version
+  d |= (uint64_t)2 << 61;                         // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, M = BM, N = BN.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          tmem_d),
+      "l"(a), "l"(b), "r"(IDESC), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(su32(bar))
+               : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ bool row_refreshes(const GemmArgs& g, int row) {
+  if (row >= g.rows) return false;
+  if (!g.S) return true;
+  if (g.force && g.t == 0) return true;
+  const int sample = row / g.H;
+  return g.S[(long long)(sample / g.per_sched) * g.S_stride + (long long)g.srow * g.T + g.t] != 0;
+}
+
+__device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
+
+// ---------------------------------------------------------------- the kernel
+template <int MODE>
+__global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                                                      const __grid_constant__ CUtensorMap tmB, const GemmArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // a tile none of whose rows refresh has nothing to do (uniform over the CTA)
+  if (g.S) {
+    const int r = m0 + lane * 4;   // 128 rows, 4 per lane: any refreshing row keeps the tile
+    const bool any = row_refreshes(g, r) || row_refreshes(g, r + 1) || row_refreshes(g, r + 2) ||
+                     row_refreshes(g, r + 3);
+    if (!__any_sync(0xffffffffu, any)) return;
+  } else if (m0 >= g.rows) {
+    return;
+  }
+
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* accb = empty + STAGES;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  if (warp == 0) tmem_alloc(tslot, BN);
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init1(&full[s], 1);
+      mbar_init1(&empty[s], 1);
+    }
+    mbar_init1(accb, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const int KB = g.K / BK;
+
+  if (warp == 0 && lane == 0) {
+    // producer
+    for (int kb = 0; kb < KB; ++kb) {
+      const int s = kb % STAGES;
+      if (kb >= STAGES) mbar_wait(&empty[s], (uint32_t)((kb / STAGES) - 1) & 1u, g.status);
+      uint8_t* sa = smem + s * STAGE_BYTES;
+      mbar_expect_tx(&full[s], STAGE_BYTES);
+      tma_load_2d(sa, &tmA, kb * BK, m0, &full[s]);
+      tma_load_2d(sa + A_BYTES, &tmB, kb * BK, g.b_row0 + n0, &full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer
+    for (int kb = 0; kb < KB; ++kb) {
+      const int s = kb % STAGES;
+      mbar_wait(&full[s], (uint32_t)(kb / STAGES) & 1u, g.status);
+      tc_fence_after();
+      const uint32_t sa = su32(smem + s * STAGE_BYTES);
+      const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+#pragma unroll
+      for (int k = 0; k < BK / 16; ++k)   // +32 bytes along K = +2 in the encoded start address
+        mma_f16(tmem, da + 2 * k, db + 2 * k, (kb | k) != 0);
+      mma_commit(&empty[s]);
+    }
+    mma_commit(accb);
+  }
+  __syncwarp();
+  mbar_wait(accb, 0, g.status);
+  tc_fence_after();
+
+  // epilogue: thread = one row, 32 columns per TMEM load
+  const int row = m0 + warp * 32 + lane;
+  const bool live = MODE == EPI_RESID ? row_refreshes(g, row) : row < g.rows;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    float v[32];
+    tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(c * 32), v);
+    const int n = n0 + c * 32;
+    if (!live) continue;
+    const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 bb = __ldg(b4 + q);
+      v[4 * q] += bb.x;
+      v[4 * q + 1] += bb.y;
+      v[4 * q + 2] += bb.z;
+      v[4 * q + 3] += bb.w;
+    }
+    if constexpr (MODE == EPI_RESID) {
+      float4* a4 = reinterpret_cast<float4*>(g.resid + (long long)row * g.ldr + n);
+      uint4* c4 = reinterpret_cast<uint4*>(g.cache + (long long)row * g.ldr + n);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint4 pk;
+        uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
+          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        c4[q] = pk;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 a = a4[q];
+        a.x += v[4 * q];
+        a.y += v[4 * q + 1];
+        a.z += v[4 * q + 2];
+        a.w += v[4 * q + 3];
+        a4[q] = a;
+      }
+    } else {
+      if constexpr (MODE == EPI_GELU_BF16) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
+      }
+      uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint4 pk;
+        uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
+          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+        }
+        o4[q] = pk;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, BN);
+}
+
+}  // namespace tc
+}  // namespace evo

@@ -1,0 +1,781 @@
+// The batch-wide path: every sample of a call advances through the T-step
+// loop together, one lattice cell (b, t) at a time, so the projections and the
+// MLP of a refreshed unit are dense GEMMs over all N*H action-token rows on the
+// tensor cores (evo_tc.cuh).  Used for large batches, where re-streaming each
+// unit's weights per sample (the cluster kernel) would waste the chip.
+//
+// Per call:
+//   first_kernel      for every lattice and unit, the first step that refreshes it
+//   init_kernel       x <- noise[0]; a <- x W_in + b_in + P_pos
+//   for t in 0..T-1:
+//     for every unit b that some lattice refreshes at t (Eq. 1, (b,t) in S):
+//       prep_kernel   rows: a += c_k for the units k since the previous prep that
+//                     the row's lattice skipped (a cache that was never written
+//                     holds zero: skipped); then LN_b(a) -> xln for refreshing rows
+//       SA:  GEMM xln W_qkv (bf16 out) -> sa_attn_kernel -> GEMM attn W_o (+= a, -> c_b)
+//       CA:  GEMM xln W_q -> ca_attn_kernel (memory tokens) -> GEMM attn W_o (+= a, -> c_b)
+//       FFN: GEMM xln W_1 (GELU, bf16 out) -> GEMM h W_2 (+= a, -> c_b)
+//     head_kernel     pending skips, LN_f, eps = . W_head + b_head, sampler step
+//                     (DDPM / DDIM), next step's input embedding
+// A tile of rows none of whose lattices refresh the unit is skipped inside the
+// GEMM; the residual epilogue touches only refreshing rows.  Rows of one
+// lattice are contiguous (samples are ordered by lattice), so with the batch
+// sizes this path serves a 128-row tile rarely mixes lattices.
+
+#include <cuda.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <vector>
+
+#include "evo_internal.h"
+#include "evo_tc.cuh"
+
+namespace evo {
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 matrix [rows][K], K contiguous, read in boxes of 64 x box_rows with the
+// 128-byte swizzle
+bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+uint16_t bf16_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7f800000u) == 0x7f800000u) return (uint16_t)(u >> 16);
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+// ---------------------------------------------------------------- lattice access on the device
+struct Lat {
+  const uint8_t* S;     // [n_sched][S_rows][T]
+  long long stride;     // bytes per lattice
+  const int* first;     // [n_sched][U]: first step that refreshes the unit (T: never)
+  int S_rows, U, T, H, per_sched, force;
+};
+
+__device__ __forceinline__ bool lat_refresh(const Lat& L, int sample, int b, int t) {
+  if (L.force && t == 0) return true;
+  const int r = L.S_rows == L.U ? b : b / 3;
+  return L.S[(long long)(sample / L.per_sched) * L.stride + (long long)r * L.T + t] != 0;
+}
+
+// the unit's cache holds a value at step t (it was refreshed at an earlier step)
+__device__ __forceinline__ bool lat_valid(const Lat& L, int sample, int b, int t) {
+  return L.first[(sample / L.per_sched) * L.U + b] < t;
+}
+
+__global__ void first_kernel(Lat L, int n_sched, int* first) {
+  const int s = blockIdx.x;
+  for (int b = threadIdx.x; b < L.U; b += blockDim.x) {
+    int f = L.T;
+    if (L.force) {
+      f = 0;
+    } else {
+      const int r = L.S_rows == L.U ? b : b / 3;
+      const uint8_t* row = L.S + (long long)s * L.stride + (long long)r * L.T;
+      for (int t = 0; t < L.T; ++t)
+        if (row[t]) {
+          f = t;
+          break;
+        }
+    }
+    first[s * L.U + b] = f;
+  }
+  (void)n_sched;
+}
+
+// ---------------------------------------------------------------- row kernels (one warp per row)
+struct RowArgs {
+  Lat lat;
+  int rows, E, A, t;
+  float* a;                       // [rows][E]
+  const __nv_bfloat16* cache;     // [U][rmax][E]
+  long long cache_unit;           // elements per unit
+  int lo, b;                      // pending skips over units [lo, b); b < U: LayerNorm of unit b
+  const float* gamma;
+  const float* beta;
+  __nv_bfloat16* xln;             // [rows][E]
+  // head / embedding
+  float* x;                       // [samples][H][A] (= rows x A)
+  const float* noise;             // [n_noise][obs_mod][H][A]
+  int obs_mod;
+  const float* stab;              // [T][8]
+  int sampler;
+  const float* lnf_g;
+  const float* lnf_b;
+  const float* head_w;            // [E][A]
+  const float* head_b;            // [A]
+  const float* in_w;              // [A][E]
+  const float* in_b;              // [E]
+  const float* pos;               // [H][E]
+};
+
+template <int NV>
+__device__ __forceinline__ void load_row(const float* src, int lane, float4 (&v)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) v[j] = *reinterpret_cast<const float4*>(src + 4 * lane + 128 * j);
+}
+
+template <int NV>
+__device__ __forceinline__ void store_row(float* dst, int lane, const float4 (&v)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) *reinterpret_cast<float4*>(dst + 4 * lane + 128 * j) = v[j];
+}
+
+__device__ __forceinline__ float warp_sum(float s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  return s;
+}
+
+// a += c_k for the pending units this row's lattice skipped (and that hold a value)
+template <int NV>
+__device__ __forceinline__ bool pending_skips(const RowArgs& p, int row, int sample, int lane, float4 (&v)[NV]) {
+  bool dirty = false;
+  for (int k = p.lo; k < p.b; ++k) {
+    if (lat_refresh(p.lat, sample, k, p.t) || !lat_valid(p.lat, sample, k, p.t)) continue;
+    const __nv_bfloat16* c = p.cache + k * p.cache_unit + (long long)row * p.E;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const uint2 raw = *reinterpret_cast<const uint2*>(c + 4 * lane + 128 * j);
+      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&raw.x);
+      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&raw.y);
+      v[j].x += __low2float(lo);
+      v[j].y += __high2float(lo);
+      v[j].z += __low2float(hi);
+      v[j].w += __high2float(hi);
+    }
+    dirty = true;
+  }
+  return dirty;
+}
+
+template <int NV>
+__device__ __forceinline__ void layer_norm(float4 (&v)[NV], const float* g, const float* bb, int lane, float invE) {
+  float s = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+    s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
+  }
+  s = warp_sum(s);
+  s2 = warp_sum(s2);
+  const float mean = s * invE;
+  const float rstd = rsqrtf(fmaxf(s2 * invE - mean * mean, 0.f) + 1e-5f);
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int col = 4 * lane + 128 * j;
+    const float4 gg = *reinterpret_cast<const float4*>(g + col);
+    const float4 b4 = *reinterpret_cast<const float4*>(bb + col);
+    v[j].x = (v[j].x - mean) * rstd * gg.x + b4.x;
+    v[j].y = (v[j].y - mean) * rstd * gg.y + b4.y;
+    v[j].z = (v[j].z - mean) * rstd * gg.z + b4.z;
+    v[j].w = (v[j].w - mean) * rstd * gg.w + b4.w;
+  }
+}
+
+template <int NV>
+__global__ void __launch_bounds__(256) prep_kernel(const RowArgs p) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.rows) return;
+  const int sample = row / p.lat.H;
+  const bool ln = lat_refresh(p.lat, sample, p.b, p.t);
+  float4 v[NV];
+  float* arow = p.a + (long long)row * p.E;
+  load_row<NV>(arow, lane, v);
+  if (pending_skips<NV>(p, row, sample, lane, v)) store_row<NV>(arow, lane, v);
+  if (!ln) return;
+  layer_norm<NV>(v, p.gamma, p.beta, lane, 1.f / (float)p.E);
+  __nv_bfloat16* dst = p.xln + (long long)row * p.E;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    __nv_bfloat162 lo = __floats2bfloat162_rn(v[j].x, v[j].y), hi = __floats2bfloat162_rn(v[j].z, v[j].w);
+    uint2 pk;
+    pk.x = *reinterpret_cast<uint32_t*>(&lo);
+    pk.y = *reinterpret_cast<uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(dst + 4 * lane + 128 * j) = pk;
+  }
+}
+
+// a <- sum_a x[a] W_in[a] + b_in + P_pos[token] for this row
+template <int NV>
+__device__ __forceinline__ void embed_row(const RowArgs& p, int row, int lane, float xa_lane) {
+  const int tok = row % p.lat.H;
+  float4 v[NV];
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int col = 4 * lane + 128 * j;
+    const float4 b4 = *reinterpret_cast<const float4*>(p.in_b + col);
+    const float4 p4 = *reinterpret_cast<const float4*>(p.pos + (long long)tok * p.E + col);
+    v[j] = make_float4(b4.x + p4.x, b4.y + p4.y, b4.z + p4.z, b4.w + p4.w);
+  }
+  float acc[NV][4];
+#pragma unroll
+  for (int j = 0; j < NV; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+  for (int a = 0; a < p.A; ++a) {
+    const float xa = __shfl_sync(0xffffffffu, xa_lane, a);
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const float4 w = *reinterpret_cast<const float4*>(p.in_w + (long long)a * p.E + 4 * lane + 128 * j);
+      acc[j][0] = fmaf(xa, w.x, acc[j][0]);
+      acc[j][1] = fmaf(xa, w.y, acc[j][1]);
+      acc[j][2] = fmaf(xa, w.z, acc[j][2]);
+      acc[j][3] = fmaf(xa, w.w, acc[j][3]);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    v[j].x += acc[j][0];
+    v[j].y += acc[j][1];
+    v[j].z += acc[j][2];
+    v[j].w += acc[j][3];
+  }
+  store_row<NV>(p.a + (long long)row * p.E, lane, v);
+}
+
+template <int NV>
+__global__ void __launch_bounds__(256) init_kernel(const RowArgs p) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.rows) return;
+  const int H = p.lat.H, sample = row / H, tok = row % H;
+  float xv = 0.f;
+  if (lane < p.A) {
+    xv = p.noise[((long long)(sample % p.obs_mod) * H + tok) * p.A + lane];
+    p.x[(long long)row * p.A + lane] = xv;
+  }
+  embed_row<NV>(p, row, lane, xv);
+}
+
+template <int NV>
+__global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.rows) return;
+  const int H = p.lat.H, sample = row / H, tok = row % H, t = p.t;
+  float4 v[NV];
+  load_row<NV>(p.a + (long long)row * p.E, lane, v);
+  pending_skips<NV>(p, row, sample, lane, v);        // a is rebuilt from x for the next step
+  layer_norm<NV>(v, p.lnf_g, p.lnf_b, lane, 1.f / (float)p.E);
+  float eps = 0.f;
+  for (int a = 0; a < p.A; ++a) {
+    float part = 0.f;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const float* w = p.head_w + (long long)(4 * lane + 128 * j) * p.A + a;
+      part = fmaf(v[j].x, w[0], part);
+      part = fmaf(v[j].y, w[p.A], part);
+      part = fmaf(v[j].z, w[2 * p.A], part);
+      part = fmaf(v[j].w, w[3 * p.A], part);
+    }
+    part = warp_sum(part);
+    if (lane == a) eps = part + p.head_b[a];
+  }
+  float xn = 0.f;
+  if (lane < p.A) {
+    const float* tb = p.stab + t * 8;
+    const float inv_sa = tb[0], s1 = tb[1], cx0 = tb[2], cxt = tb[3], sig = tb[4], sab = tb[5], sabp = tb[6],
+                s1p = tb[7];
+    const float xv = p.x[(long long)row * p.A + lane];
+    float x0 = (xv - s1 * eps) * inv_sa;
+    x0 = fminf(1.0f, fmaxf(-1.0f, x0));
+    if (p.sampler == 0) {
+      const float z = p.noise[(((long long)(1 + t) * p.obs_mod + (sample % p.obs_mod)) * H + tok) * p.A + lane];
+      xn = cx0 * x0 + cxt * xv + sig * z;
+    } else {
+      xn = sabp * x0 + s1p * ((xv - sab * x0) / s1);
+    }
+    p.x[(long long)row * p.A + lane] = xn;
+  }
+  if (t + 1 < p.lat.T) embed_row<NV>(p, row, lane, xn);
+}
+
+// ---------------------------------------------------------------- attention
+struct AttnArgs {
+  Lat lat;
+  int b, t, l, L, E, nh, dh, rows, samples, n_obs, obs_mod;
+  const __nv_bfloat16* qkv;       // SA: [rows][3E] (q | k | v); CA: [rows][E] (q)
+  __nv_bfloat16* att;             // [rows][E]
+  const float* kv_time;           // [T][L][2E]
+  const float* kv_obs;            // [obs_mod][n_obs][L][2E]
+  float scale;
+};
+
+// causal self-attention of one (sample, head) over its H action tokens
+__global__ void __launch_bounds__(128) sa_attn_kernel(const AttnArgs p) {
+  const int s = blockIdx.x, h = blockIdx.y;
+  if (!lat_refresh(p.lat, s, p.b, p.t)) return;
+  extern __shared__ float sm[];
+  const int H = p.lat.H, dh = p.dh, ld = dh + 1, E = p.E;
+  float* q = sm;
+  float* k = q + H * ld;
+  float* v = k + H * ld;
+  float* pr = v + H * ld;   // [H][H + 1]
+  const __nv_bfloat16* base = p.qkv + (long long)s * H * 3 * E + h * dh;
+  for (int idx = threadIdx.x; idx < H * dh / 2; idx += blockDim.x) {
+    const int i = idx / (dh / 2), d = 2 * (idx % (dh / 2));
+    const __nv_bfloat16* r = base + (long long)i * 3 * E + d;
+    const float2 fq = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r));
+    const float2 fk = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r + E));
+    const float2 fv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r + 2 * E));
+    q[i * ld + d] = fq.x;
+    q[i * ld + d + 1] = fq.y;
+    k[i * ld + d] = fk.x;
+    k[i * ld + d + 1] = fk.y;
+    v[i * ld + d] = fv.x;
+    v[i * ld + d + 1] = fv.y;
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < H * H; idx += blockDim.x) {
+    const int i = idx / H, j = idx % H;
+    float sc = -INFINITY;
+    if (j <= i) {
+      float d0 = 0.f, d1 = 0.f;
+      for (int e = 0; e < dh; e += 2) {
+        d0 = fmaf(q[i * ld + e], k[j * ld + e], d0);
+        d1 = fmaf(q[i * ld + e + 1], k[j * ld + e + 1], d1);
+      }
+      sc = (d0 + d1) * p.scale;
+    }
+    pr[i * (H + 1) + j] = sc;
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = warp; i < H; i += blockDim.x >> 5) {
+    const float x = lane < H ? pr[i * (H + 1) + lane] : -INFINITY;
+    float mx = x;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    const float ex = x == -INFINITY ? 0.f : __expf(x - mx);
+    const float sum = warp_sum(ex);
+    if (lane < H) pr[i * (H + 1) + lane] = ex / sum;
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < H * dh; idx += blockDim.x) {
+    const int i = idx / dh, d = idx % dh;
+    float o = 0.f;
+    for (int j = 0; j <= i; ++j) o = fmaf(pr[i * (H + 1) + j], v[j * ld + d], o);
+    p.att[((long long)s * H + i) * E + h * dh + d] = __float2bfloat16_rn(o);
+  }
+}
+
+// cross-attention of one (row, head) to the 1 + n_obs memory tokens
+template <int DH>
+__global__ void __launch_bounds__(128) ca_attn_kernel(const AttnArgs p) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int row = idx / p.nh, h = idx % p.nh;
+  if (row >= p.rows) return;
+  const int sample = row / p.lat.H;
+  if (!lat_refresh(p.lat, sample, p.b, p.t)) return;
+  const int E = p.E, Cm = 1 + p.n_obs;
+  float q[DH];
+  const __nv_bfloat16* qr = p.qkv + (long long)row * E + h * DH;
+#pragma unroll
+  for (int d = 0; d < DH; d += 2) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(qr + d));
+    q[d] = f.x;
+    q[d + 1] = f.y;
+  }
+  constexpr int MAXC = 8;
+  float sc[MAXC];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j) {
+    sc[j] = -INFINITY;
+    if (j < Cm) {
+      const float* kr = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
+                               : p.kv_obs + (((long long)(sample % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
+      kr += h * DH;
+      float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll
+      for (int d = 0; d < DH; d += 4) {
+        const float4 kk = *reinterpret_cast<const float4*>(kr + d);
+        d0 = fmaf(q[d], kk.x, d0);
+        d1 = fmaf(q[d + 1], kk.y, d1);
+        d2 = fmaf(q[d + 2], kk.z, d2);
+        d3 = fmaf(q[d + 3], kk.w, d3);
+      }
+      sc[j] = ((d0 + d1) + (d2 + d3)) * p.scale;
+      mx = fmaxf(mx, sc[j]);
+    }
+  }
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j) {
+    sc[j] = j < Cm ? __expf(sc[j] - mx) : 0.f;
+    sum += sc[j];
+  }
+  const float inv = 1.f / sum;
+#pragma unroll
+  for (int d = 0; d < DH; ++d) q[d] = 0.f;
+#pragma unroll
+  for (int j = 0; j < MAXC; ++j) {
+    if (j < Cm) {
+      const float* vr = (j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
+                                : p.kv_obs + (((long long)(sample % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E) +
+                        E + h * DH;
+      const float w = sc[j] * inv;
+#pragma unroll
+      for (int d = 0; d < DH; d += 4) {
+        const float4 vv = *reinterpret_cast<const float4*>(vr + d);
+        q[d] = fmaf(w, vv.x, q[d]);
+        q[d + 1] = fmaf(w, vv.y, q[d + 1]);
+        q[d + 2] = fmaf(w, vv.z, q[d + 2]);
+        q[d + 3] = fmaf(w, vv.w, q[d + 3]);
+      }
+    }
+  }
+  __nv_bfloat16* o = p.att + (long long)row * E + h * DH;
+#pragma unroll
+  for (int d = 0; d < DH; d += 2) *reinterpret_cast<__nv_bfloat162*>(o + d) = __floats2bfloat162_rn(q[d], q[d + 1]);
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- state
+struct WideState {
+  int L = 0, E = 0, nh = 0, dh = 0, H = 0, A = 0, n_obs = 0, T = 0, U = 0, sampler = 0, force = 0;
+  long long rmax = 0;     // rows the buffers hold (multiple of BM)
+  int max_sched = 0;
+  const float* wf32 = nullptr;
+  int woff[W_COUNT];
+  __nv_bfloat16* wt_e = nullptr;    // [L * 10E][E]: per layer W_qkv^T | W_o^T | W_q^T | W_o'^T | W_1^T
+  __nv_bfloat16* wt_4e = nullptr;   // [L * E][4E]: per layer W_2^T
+  __nv_bfloat16* xln = nullptr;     // [rmax][E]
+  __nv_bfloat16* qkv = nullptr;     // [rmax][3E]
+  __nv_bfloat16* att = nullptr;     // [rmax][E]
+  __nv_bfloat16* hid = nullptr;     // [rmax][4E]
+  __nv_bfloat16* cache = nullptr;   // [U][rmax][E]
+  float* a = nullptr;               // [rmax][E]
+  int* first = nullptr;             // [max_sched][U]
+  CUtensorMap mA_xln, mA_att, mA_hid, mB_e, mB_4e;
+  std::vector<uint8_t> any;         // [U][T] scratch: some lattice refreshes (b, t)
+  long long launches = 0;
+};
+
+namespace {
+
+const float* wl(const WideState* w, int l, int id) {
+  return w->wf32 + w->woff[W_LAYER0] + (long long)l * w->woff[W_LAYER_STRIDE] + w->woff[id];
+}
+
+template <int MODE>
+cudaError_t gemm(const CUtensorMap& ma, const CUtensorMap& mb, const tc::GemmArgs& g, int rows_p, int N,
+                 cudaStream_t st) {
+  tc::gemm_kernel<MODE><<<dim3(rows_p / tc::BM, N / tc::BN), 128, tc::SMEM_BYTES, st>>>(ma, mb, g);
+  return cudaGetLastError();
+}
+
+template <int NV>
+cudaError_t launch_rows(int which, const RowArgs& p, cudaStream_t st) {
+  const int blocks = (p.rows + 7) / 8;
+  if (which == 0) init_kernel<NV><<<blocks, 256, 0, st>>>(p);
+  else if (which == 1) prep_kernel<NV><<<blocks, 256, 0, st>>>(p);
+  else head_kernel<NV><<<blocks, 256, 0, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t rows_kernel(int which, const RowArgs& p, cudaStream_t st) {
+  switch (p.E / 128) {
+    case 2: return launch_rows<2>(which, p, st);
+    case 4: return launch_rows<4>(which, p, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+bool wide_supported(const evo_config* c) {
+  const int E = c->n_emb, dh = E / c->n_head;
+  return c->dtype == EVO_DTYPE_BF16 && (E == 256 || E == 512) && dh == 64 && c->horizon <= 32 &&
+         128 % c->horizon == 0 && c->action_dim <= 32 && 1 + c->n_obs <= 8 && encode_fn() != nullptr;
+}
+
+int wide_create(WideState** out, const evo_config* c, const float* weights, const float* wf32_dev, const int* woff,
+                long long max_rows, int max_sched) {
+  *out = nullptr;
+  if (!wide_supported(c)) return EVO_ERR_UNSUPPORTED;
+  WideState* w = new WideState();
+  w->L = c->n_layer;
+  w->E = c->n_emb;
+  w->nh = c->n_head;
+  w->dh = w->E / w->nh;
+  w->H = c->horizon;
+  w->A = c->action_dim;
+  w->n_obs = c->n_obs;
+  w->T = c->n_steps;
+  w->U = 3 * c->n_layer;
+  w->sampler = c->sampler;
+  w->force = c->empty_cache == EVO_EMPTY_FORCE;
+  w->rmax = (max_rows + tc::BM - 1) / tc::BM * tc::BM;
+  w->max_sched = max_sched;
+  w->wf32 = wf32_dev;
+  std::memcpy(w->woff, woff, sizeof(w->woff));
+  w->any.resize((size_t)w->U * w->T);
+  const int E = w->E, L = w->L;
+  const long long R = w->rmax;
+  auto fail = [&](int s) {
+    wide_destroy(w);
+    return s;
+  };
+  // weights, transposed to [N][K] (K contiguous) in bf16
+  {
+    std::vector<uint16_t> te((size_t)L * 10 * E * E), t4((size_t)L * E * 4 * E);
+    auto WLh = [&](int l, int id) { return weights + woff[W_LAYER0] + (size_t)l * woff[W_LAYER_STRIDE] + woff[id]; };
+    for (int l = 0; l < L; ++l) {
+      uint16_t* d = te.data() + (size_t)l * 10 * E * E;
+      const float* wqkv = WLh(l, WL_SA_WQKV);
+      const float* wo = WLh(l, WL_SA_WO);
+      const float* wq = WLh(l, WL_CA_WQ);
+      const float* wo2 = WLh(l, WL_CA_WO);
+      const float* w1 = WLh(l, WL_FF_W1);
+      const float* w2 = WLh(l, WL_FF_W2);
+      for (int k = 0; k < E; ++k) {
+        for (int n = 0; n < 3 * E; ++n) d[(size_t)n * E + k] = bf16_bits(wqkv[(size_t)k * 3 * E + n]);
+        for (int n = 0; n < E; ++n) {
+          d[(size_t)(3 * E + n) * E + k] = bf16_bits(wo[(size_t)k * E + n]);
+          d[(size_t)(4 * E + n) * E + k] = bf16_bits(wq[(size_t)k * E + n]);
+          d[(size_t)(5 * E + n) * E + k] = bf16_bits(wo2[(size_t)k * E + n]);
+        }
+        for (int n = 0; n < 4 * E; ++n) d[(size_t)(6 * E + n) * E + k] = bf16_bits(w1[(size_t)k * 4 * E + n]);
+      }
+      uint16_t* d4 = t4.data() + (size_t)l * E * 4 * E;
+      for (int k = 0; k < 4 * E; ++k)
+        for (int n = 0; n < E; ++n) d4[(size_t)n * 4 * E + k] = bf16_bits(w2[(size_t)k * E + n]);
+    }
+    if (cudaMalloc(&w->wt_e, te.size() * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMalloc(&w->wt_4e, t4.size() * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMemcpy(w->wt_e, te.data(), te.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess) return fail(EVO_ERR_CUDA);
+    if (cudaMemcpy(w->wt_4e, t4.data(), t4.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(EVO_ERR_CUDA);
+  }
+  if (cudaMalloc(&w->xln, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->qkv, R * 3 * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->att, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->hid, R * 4 * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->cache, (size_t)w->U * R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->a, R * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->first, (size_t)max_sched * w->U * sizeof(int)) != cudaSuccess) return fail(EVO_ERR_OOM);
+  // operand rows that no call writes (padding up to a tile) read as zero
+  cudaMemset(w->xln, 0, R * E * 2);
+  cudaMemset(w->att, 0, R * E * 2);
+  cudaMemset(w->hid, 0, R * 4 * E * 2);
+  if (!make_map(&w->mA_xln, w->xln, R, E, tc::BM) || !make_map(&w->mA_att, w->att, R, E, tc::BM) ||
+      !make_map(&w->mA_hid, w->hid, R, 4 * E, tc::BM) || !make_map(&w->mB_e, w->wt_e, (long long)L * 10 * E, E, tc::BN) ||
+      !make_map(&w->mB_4e, w->wt_4e, (long long)L * E, 4 * E, tc::BN))
+    return fail(EVO_ERR_CUDA);
+  if (cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tc::SMEM_BYTES) != cudaSuccess ||
+      cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_GELU_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tc::SMEM_BYTES) != cudaSuccess ||
+      cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           tc::SMEM_BYTES) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(EVO_ERR_CUDA);
+  *out = w;
+  return EVO_OK;
+}
+
+void wide_destroy(WideState* w) {
+  if (!w) return;
+  cudaFree(w->wt_e);
+  cudaFree(w->wt_4e);
+  cudaFree(w->xln);
+  cudaFree(w->qkv);
+  cudaFree(w->att);
+  cudaFree(w->hid);
+  cudaFree(w->cache);
+  cudaFree(w->a);
+  cudaFree(w->first);
+  delete w;
+}
+
+long long wide_rows_capacity(const WideState* w) { return w ? w->rmax : 0; }
+long long wide_last_launches(const WideState* w) { return w ? w->launches : 0; }
+
+cudaError_t wide_run(WideState* w, const WideCall& c) {
+  const int E = w->E, L = w->L, U = w->U, T = w->T, H = w->H;
+  const long long R = (long long)c.samples * H;
+  if (R > w->rmax || c.n_sched > w->max_sched) return cudaErrorInvalidValue;
+  const int Rp = (int)((R + tc::BM - 1) / tc::BM * tc::BM);
+  cudaStream_t st = c.st;
+  long long n = 0;
+  cudaError_t e;
+#define WCK(x)                    \
+  do {                            \
+    e = (x);                      \
+    if (e != cudaSuccess) return e; \
+    ++n;                          \
+  } while (0)
+
+  // which cells some lattice refreshes (host copy of the lattices)
+  const long long one = (long long)c.S_rows * T;
+  for (int b = 0; b < U; ++b)
+    for (int t = 0; t < T; ++t) {
+      const int r = c.S_rows == U ? b : b / 3;
+      bool any = w->force && t == 0;
+      for (int s = 0; s < c.n_sched && !any; ++s) any = c.S_host[s * one + (long long)r * T + t] != 0;
+      w->any[(size_t)b * T + t] = any;
+    }
+
+  Lat lat;
+  lat.S = c.S_dev;
+  lat.stride = one;
+  lat.first = w->first;
+  lat.S_rows = c.S_rows;
+  lat.U = U;
+  lat.T = T;
+  lat.H = H;
+  lat.per_sched = c.per_sched;
+  lat.force = w->force;
+  first_kernel<<<c.n_sched, 64, 0, st>>>(lat, c.n_sched, w->first);
+  WCK(cudaGetLastError());
+
+  RowArgs rp{};
+  rp.lat = lat;
+  rp.rows = (int)R;
+  rp.E = E;
+  rp.A = w->A;
+  rp.a = w->a;
+  rp.cache = w->cache;
+  rp.cache_unit = w->rmax * E;
+  rp.xln = w->xln;
+  rp.x = c.out;
+  rp.noise = c.noise;
+  rp.obs_mod = c.obs_mod;
+  rp.stab = c.stab;
+  rp.sampler = w->sampler;
+  rp.lnf_g = w->wf32 + w->woff[W_LNF_G];
+  rp.lnf_b = w->wf32 + w->woff[W_LNF_B];
+  rp.head_w = w->wf32 + w->woff[W_HEAD_W];
+  rp.head_b = w->wf32 + w->woff[W_HEAD_B];
+  rp.in_w = w->wf32 + w->woff[W_IN_W];
+  rp.in_b = w->wf32 + w->woff[W_IN_B];
+  rp.pos = w->wf32 + w->woff[W_POS];
+  WCK(rows_kernel(0, rp, st));
+
+  tc::GemmArgs g{};
+  g.rows = (int)R;
+  g.S = c.S_dev;
+  g.S_stride = one;
+  g.T = T;
+  g.H = H;
+  g.per_sched = c.per_sched;
+  g.force = w->force;
+  g.status = c.status;
+  g.ldr = E;
+  g.resid = w->a;
+
+  AttnArgs ap{};
+  ap.lat = lat;
+  ap.L = L;
+  ap.E = E;
+  ap.nh = w->nh;
+  ap.dh = w->dh;
+  ap.rows = (int)R;
+  ap.samples = c.samples;
+  ap.n_obs = w->n_obs;
+  ap.obs_mod = c.obs_mod;
+  ap.att = w->att;
+  ap.kv_time = c.kv_time;
+  ap.kv_obs = c.kv_obs;
+  ap.scale = 1.f / std::sqrt((float)w->dh);
+  const size_t sa_smem = (size_t)(3 * H * (w->dh + 1) + H * (H + 1)) * sizeof(float);
+
+  for (int t = 0; t < T; ++t) {
+    int lo = 0;
+    rp.t = t;
+    g.t = t;
+    ap.t = t;
+    for (int b = 0; b < U; ++b) {
+      if (!w->any[(size_t)b * T + t]) continue;
+      const int l = b / 3, u = b % 3;
+      static const int ln_g[3] = {WL_LN1G, WL_LN2G, WL_LN3G}, ln_b[3] = {WL_LN1B, WL_LN2B, WL_LN3B};
+      rp.lo = lo;
+      rp.b = b;
+      rp.gamma = wl(w, l, ln_g[u]);
+      rp.beta = wl(w, l, ln_b[u]);
+      WCK(rows_kernel(1, rp, st));
+      lo = b;
+      g.srow = c.S_rows == U ? b : b / 3;
+      g.cache = w->cache + (long long)b * w->rmax * E;
+      ap.b = b;
+      ap.l = l;
+      const int rowE = l * 10 * E;
+      if (u == 0) {
+        g.K = E;
+        g.b_row0 = rowE;
+        g.bias = wl(w, l, WL_SA_BQKV);
+        g.out = w->qkv;
+        g.ldo = 3 * E;
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, st));
+        ap.qkv = w->qkv;
+        sa_attn_kernel<<<dim3(c.samples, w->nh), 128, sa_smem, st>>>(ap);
+        WCK(cudaGetLastError());
+        g.b_row0 = rowE + 3 * E;
+        g.bias = wl(w, l, WL_SA_BO);
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, st));
+      } else if (u == 1) {
+        g.K = E;
+        g.b_row0 = rowE + 4 * E;
+        g.bias = wl(w, l, WL_CA_BQ);
+        g.out = w->qkv;
+        g.ldo = E;
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, st));
+        ap.qkv = w->qkv;
+        ca_attn_kernel<64><<<(int)((R * w->nh + 127) / 128), 128, 0, st>>>(ap);
+        WCK(cudaGetLastError());
+        g.b_row0 = rowE + 5 * E;
+        g.bias = wl(w, l, WL_CA_BO);
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, st));
+      } else {
+        g.K = E;
+        g.b_row0 = rowE + 6 * E;
+        g.bias = wl(w, l, WL_FF_B1);
+        g.out = w->hid;
+        g.ldo = 4 * E;
+        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, st));
+        g.K = 4 * E;
+        g.b_row0 = l * E;
+        g.bias = wl(w, l, WL_FF_B2);
+        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, st));
+      }
+    }
+    rp.lo = lo;
+    rp.b = U;
+    WCK(rows_kernel(2, rp, st));
+  }
+#undef WCK
+  w->launches = n;
+  return cudaSuccess;
+}
+
+}  // namespace evo

@@ -172,10 +172,12 @@ def test_odd_batch_with_two_samples_per_job(torch, B):
 
 # ------------------------------------------------------------------ batched configs at full size
 
-def test_manip_batch64_heterogeneous(torch, B):
-    cfg, W, obs, noise, ev, d_obs, d_noise = setup("manip", 64, torch, B)
+@pytest.mark.parametrize("path", ["wide", "cluster"])
+def test_manip_batch64_heterogeneous(torch, B, path):
+    cfg, W, obs, noise, ev, d_obs, d_noise = setup("manip", 64, torch, B, wide_rows=0 if path == "wide" else -1)
     S = synth.heterogeneous_schedule(24, 100, 4)
     got = ev.denoise(d_obs, d_noise, S).cpu().numpy()
+    assert ev.last_call()["path"] == path
     idx = [0, 17, 63]
     check(got[idx], oracle_subset(W, cfg, obs, noise, S, idx), TOL["bf16"], "manip")
     assert np.all(np.isfinite(got)) and np.all(np.abs(got) <= 1.5)
@@ -187,22 +189,27 @@ def test_scaleup(torch, B, n, frac):
     cfg, W, obs, noise, ev, d_obs, d_noise = setup(name, n, torch, B)
     S = synth.bernoulli_schedule(36, 100, frac, 7)
     got = ev.denoise(d_obs, d_noise, S).cpu().numpy()
+    assert ev.last_call()["path"] == "wide"
     idx = [0, n - 1]
     check(got[idx], oracle_subset(W, cfg, obs, noise, S, idx), TOL["bf16"], name)
 
 
-def test_population_64x16(torch, B):
+@pytest.mark.parametrize("path", ["wide", "cluster"])
+def test_population_64x16(torch, B, path):
     cfg = synth.config("population")
     W = synth.make_weights(cfg, 0)
     P, N = cfg["n_candidates"], cfg["batch"]
     obs, noise = synth.make_obs(cfg, N, 1), synth.make_noise(cfg, N, 2)
     pop = synth.guided_population(synth.dissimilarity_map(8, 100, 5), P, 6)
-    ev = B.Evo(cfg, W, (P + 1) * N)
+    # the reference chunks below (N samples) must take the population's path
+    ev = B.Evo(cfg, W, (P + 1) * N, wide_rows=N * cfg["horizon"] if path == "wide" else -1)
     x, dev = ev.population(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(), pop)
+    assert ev.last_call()["path"] == path
     x, dev = x.cpu().numpy(), dev.cpu().numpy()
     # deviation is consistent with the returned actions and the all-refresh reference
     full = ev.denoise(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(),
                       np.ones((24, 100), np.uint8)).cpu().numpy()
+    assert ev.last_call()["path"] == path
     host_dev = np.linalg.norm((x - full[None]).reshape(P, N, -1), axis=2).mean(1)
     assert np.allclose(dev, host_dev, rtol=1e-4, atol=1e-5)
     # sampled chunks against the oracle, including the reference
