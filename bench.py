@@ -198,6 +198,8 @@ def run_ours(args, world, rank, local):
     build.build()
     binding.load()
     name, fracs, head_frac, kind = WORKLOADS[args.workload]
+    if args.fractions:
+        fracs, head_frac = args.fractions, args.fractions[0]
     cfg = synth.config(name)
     n = cfg["batch"]
     W = synth.make_weights(cfg, 0)
@@ -337,9 +339,13 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="pusht", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fractions", type=float, nargs="*", default=None,
+                    help="refresh fractions to sweep (default: the workload's; the headline is the first)")
     args = ap.parse_args()
     world, rank, local = dist_env()
     name, fracs, head_frac, kind = WORKLOADS[args.workload]
+    if args.fractions:
+        head_frac = args.fractions[0]
 
     if args.impl == "reference":
         if rank != 0:

@@ -74,7 +74,8 @@ typedef struct evo_config {
   int32_t debug_sync;   /* 1: synchronize after each call and return the device status */
   int32_t wide_rows;    /* batch-wide tensor-core path for calls of at least this many action-token
                            rows (samples x horizon); 0 = 1024; < 0 = never.  bf16 with n_emb 256 or
-                           512, head size 64, horizon dividing 128, at most 7 observation tokens */
+                           512, head size 64, horizon 16 or 32, action dim <= 16, at most 7
+                           observation tokens */
 } evo_config;
 
 /* Number of float32 values in the weight blob for cfg (0 if cfg is invalid).

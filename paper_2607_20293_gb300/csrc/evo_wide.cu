@@ -140,16 +140,53 @@ struct RowArgs {
   const float* pos;               // [H][E]
 };
 
+// Row layout of the warp-per-row kernels: lane owns columns
+// [256 j + 8 lane, 256 j + 8 lane + 8) for j < NV = E / 256, so a row of the
+// fp32 stream is two float4 per lane and chunk, a bf16 cache row one uint4.
 template <int NV>
-__device__ __forceinline__ void load_row(const float* src, int lane, float4 (&v)[NV]) {
+struct RowV {
+  float v[NV][8];
+};
+
+template <int NV>
+__device__ __forceinline__ void load_row(const float* src, int lane, RowV<NV>& r) {
 #pragma unroll
-  for (int j = 0; j < NV; ++j) v[j] = *reinterpret_cast<const float4*>(src + 4 * lane + 128 * j);
+  for (int j = 0; j < NV; ++j) {
+    const float4* s4 = reinterpret_cast<const float4*>(src + 256 * j + 8 * lane);
+    const float4 a = s4[0], b = s4[1];
+    r.v[j][0] = a.x; r.v[j][1] = a.y; r.v[j][2] = a.z; r.v[j][3] = a.w;
+    r.v[j][4] = b.x; r.v[j][5] = b.y; r.v[j][6] = b.z; r.v[j][7] = b.w;
+  }
 }
 
 template <int NV>
-__device__ __forceinline__ void store_row(float* dst, int lane, const float4 (&v)[NV]) {
+__device__ __forceinline__ void store_row(float* dst, int lane, const RowV<NV>& r) {
 #pragma unroll
-  for (int j = 0; j < NV; ++j) *reinterpret_cast<float4*>(dst + 4 * lane + 128 * j) = v[j];
+  for (int j = 0; j < NV; ++j) {
+    float4* d4 = reinterpret_cast<float4*>(dst + 256 * j + 8 * lane);
+    d4[0] = make_float4(r.v[j][0], r.v[j][1], r.v[j][2], r.v[j][3]);
+    d4[1] = make_float4(r.v[j][4], r.v[j][5], r.v[j][6], r.v[j][7]);
+  }
+}
+
+__device__ __forceinline__ void add_bf16x8(float* v, uint4 raw) {
+  const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+    v[2 * i] += f.x;
+    v[2 * i + 1] += f.y;
+  }
+}
+
+__device__ __forceinline__ uint4 pack_bf16x8(const float* v) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    w[i] = *reinterpret_cast<uint32_t*>(&h);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 __device__ __forceinline__ float warp_sum(float s) {
@@ -158,49 +195,65 @@ __device__ __forceinline__ float warp_sum(float s) {
   return s;
 }
 
-// a += c_k for the pending units this row's lattice skipped (and that hold a value)
+// a += c_k for the pending units [lo, b) this row's lattice skipped and that
+// hold a value; the cache rows of up to four units are in flight at once
 template <int NV>
-__device__ __forceinline__ bool pending_skips(const RowArgs& p, int row, int sample, int lane, float4 (&v)[NV]) {
-  bool dirty = false;
-  for (int k = p.lo; k < p.b; ++k) {
-    if (lat_refresh(p.lat, sample, k, p.t) || !lat_valid(p.lat, sample, k, p.t)) continue;
-    const __nv_bfloat16* c = p.cache + k * p.cache_unit + (long long)row * p.E;
+__device__ __forceinline__ bool pending_skips(const RowArgs& p, int row, int sample, int lane, RowV<NV>& r) {
+  uint64_t m = 0;
+  for (int k = p.lo; k < p.b; ++k)
+    if (!lat_refresh(p.lat, sample, k, p.t) && lat_valid(p.lat, sample, k, p.t)) m |= 1ull << k;
+  if (!m) return false;
+  const __nv_bfloat16* base = p.cache + (long long)row * p.E + 8 * lane;
+  while (m) {
+    int ks[4];
+    int nk = 0;
 #pragma unroll
-    for (int j = 0; j < NV; ++j) {
-      const uint2 raw = *reinterpret_cast<const uint2*>(c + 4 * lane + 128 * j);
-      const __nv_bfloat162 lo = *reinterpret_cast<const __nv_bfloat162*>(&raw.x);
-      const __nv_bfloat162 hi = *reinterpret_cast<const __nv_bfloat162*>(&raw.y);
-      v[j].x += __low2float(lo);
-      v[j].y += __high2float(lo);
-      v[j].z += __low2float(hi);
-      v[j].w += __high2float(hi);
+    for (int q = 0; q < 4; ++q) {
+      ks[q] = m ? __ffsll((long long)m) - 1 : -1;
+      if (m) {
+        m &= m - 1;
+        ++nk;
+      }
     }
-    dirty = true;
+    uint4 raw[4][NV];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int j = 0; j < NV; ++j)
+        raw[q][j] = ks[q] >= 0 ? *reinterpret_cast<const uint4*>(base + ks[q] * p.cache_unit + 256 * j)
+                               : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      if (q < nk)
+#pragma unroll
+        for (int j = 0; j < NV; ++j) add_bf16x8(r.v[j], raw[q][j]);
   }
-  return dirty;
+  return true;
 }
 
 template <int NV>
-__device__ __forceinline__ void layer_norm(float4 (&v)[NV], const float* g, const float* bb, int lane, float invE) {
+__device__ __forceinline__ void layer_norm(RowV<NV>& r, const float* g, const float* bb, int lane, float invE) {
   float s = 0.f, s2 = 0.f;
 #pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
-    s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
-  }
+  for (int j = 0; j < NV; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      s += r.v[j][i];
+      s2 += r.v[j][i] * r.v[j][i];
+    }
   s = warp_sum(s);
   s2 = warp_sum(s2);
   const float mean = s * invE;
   const float rstd = rsqrtf(fmaxf(s2 * invE - mean * mean, 0.f) + 1e-5f);
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
-    const int col = 4 * lane + 128 * j;
-    const float4 gg = *reinterpret_cast<const float4*>(g + col);
-    const float4 b4 = *reinterpret_cast<const float4*>(bb + col);
-    v[j].x = (v[j].x - mean) * rstd * gg.x + b4.x;
-    v[j].y = (v[j].y - mean) * rstd * gg.y + b4.y;
-    v[j].z = (v[j].z - mean) * rstd * gg.z + b4.z;
-    v[j].w = (v[j].w - mean) * rstd * gg.w + b4.w;
+    const int col = 256 * j + 8 * lane;
+    const float4 g0 = *reinterpret_cast<const float4*>(g + col), g1 = *reinterpret_cast<const float4*>(g + col + 4);
+    const float4 b0 = *reinterpret_cast<const float4*>(bb + col), b1 = *reinterpret_cast<const float4*>(bb + col + 4);
+    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) r.v[j][i] = (r.v[j][i] - mean) * rstd * gg[i] + bv[i];
   }
 }
 
@@ -210,57 +263,43 @@ __global__ void __launch_bounds__(256) prep_kernel(const RowArgs p) {
   if (row >= p.rows) return;
   const int sample = row / p.lat.H;
   const bool ln = lat_refresh(p.lat, sample, p.b, p.t);
-  float4 v[NV];
+  RowV<NV> r;
   float* arow = p.a + (long long)row * p.E;
-  load_row<NV>(arow, lane, v);
-  if (pending_skips<NV>(p, row, sample, lane, v)) store_row<NV>(arow, lane, v);
+  load_row<NV>(arow, lane, r);
+  if (pending_skips<NV>(p, row, sample, lane, r)) store_row<NV>(arow, lane, r);
   if (!ln) return;
-  layer_norm<NV>(v, p.gamma, p.beta, lane, 1.f / (float)p.E);
-  __nv_bfloat16* dst = p.xln + (long long)row * p.E;
+  layer_norm<NV>(r, p.gamma, p.beta, lane, 1.f / (float)p.E);
+  __nv_bfloat16* dst = p.xln + (long long)row * p.E + 8 * lane;
 #pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    __nv_bfloat162 lo = __floats2bfloat162_rn(v[j].x, v[j].y), hi = __floats2bfloat162_rn(v[j].z, v[j].w);
-    uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&lo);
-    pk.y = *reinterpret_cast<uint32_t*>(&hi);
-    *reinterpret_cast<uint2*>(dst + 4 * lane + 128 * j) = pk;
-  }
+  for (int j = 0; j < NV; ++j) *reinterpret_cast<uint4*>(dst + 256 * j) = pack_bf16x8(r.v[j]);
 }
 
 // a <- sum_a x[a] W_in[a] + b_in + P_pos[token] for this row
 template <int NV>
 __device__ __forceinline__ void embed_row(const RowArgs& p, int row, int lane, float xa_lane) {
   const int tok = row % p.lat.H;
-  float4 v[NV];
+  RowV<NV> r;
+  load_row<NV>(p.pos + (long long)tok * p.E, lane, r);
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
-    const int col = 4 * lane + 128 * j;
-    const float4 b4 = *reinterpret_cast<const float4*>(p.in_b + col);
-    const float4 p4 = *reinterpret_cast<const float4*>(p.pos + (long long)tok * p.E + col);
-    v[j] = make_float4(b4.x + p4.x, b4.y + p4.y, b4.z + p4.z, b4.w + p4.w);
+    const int col = 256 * j + 8 * lane;
+    const float4 b0 = *reinterpret_cast<const float4*>(p.in_b + col), b1 = *reinterpret_cast<const float4*>(p.in_b + col + 4);
+    r.v[j][0] += b0.x; r.v[j][1] += b0.y; r.v[j][2] += b0.z; r.v[j][3] += b0.w;
+    r.v[j][4] += b1.x; r.v[j][5] += b1.y; r.v[j][6] += b1.z; r.v[j][7] += b1.w;
   }
-  float acc[NV][4];
-#pragma unroll
-  for (int j = 0; j < NV; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
   for (int a = 0; a < p.A; ++a) {
     const float xa = __shfl_sync(0xffffffffu, xa_lane, a);
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
-      const float4 w = *reinterpret_cast<const float4*>(p.in_w + (long long)a * p.E + 4 * lane + 128 * j);
-      acc[j][0] = fmaf(xa, w.x, acc[j][0]);
-      acc[j][1] = fmaf(xa, w.y, acc[j][1]);
-      acc[j][2] = fmaf(xa, w.z, acc[j][2]);
-      acc[j][3] = fmaf(xa, w.w, acc[j][3]);
+      const float* w = p.in_w + (long long)a * p.E + 256 * j + 8 * lane;
+      const float4 w0 = *reinterpret_cast<const float4*>(w), w1 = *reinterpret_cast<const float4*>(w + 4);
+      r.v[j][0] = fmaf(xa, w0.x, r.v[j][0]); r.v[j][1] = fmaf(xa, w0.y, r.v[j][1]);
+      r.v[j][2] = fmaf(xa, w0.z, r.v[j][2]); r.v[j][3] = fmaf(xa, w0.w, r.v[j][3]);
+      r.v[j][4] = fmaf(xa, w1.x, r.v[j][4]); r.v[j][5] = fmaf(xa, w1.y, r.v[j][5]);
+      r.v[j][6] = fmaf(xa, w1.z, r.v[j][6]); r.v[j][7] = fmaf(xa, w1.w, r.v[j][7]);
     }
   }
-#pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    v[j].x += acc[j][0];
-    v[j].y += acc[j][1];
-    v[j].z += acc[j][2];
-    v[j].w += acc[j][3];
-  }
-  store_row<NV>(p.a + (long long)row * p.E, lane, v);
+  store_row<NV>(p.a + (long long)row * p.E, lane, r);
 }
 
 template <int NV>
@@ -276,44 +315,55 @@ __global__ void __launch_bounds__(256) init_kernel(const RowArgs p) {
   embed_row<NV>(p, row, lane, xv);
 }
 
+constexpr int MAXA = 16;
+
 template <int NV>
 __global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.rows) return;
-  const int H = p.lat.H, sample = row / H, tok = row % H, t = p.t;
-  float4 v[NV];
-  load_row<NV>(p.a + (long long)row * p.E, lane, v);
-  pending_skips<NV>(p, row, sample, lane, v);        // a is rebuilt from x for the next step
-  layer_norm<NV>(v, p.lnf_g, p.lnf_b, lane, 1.f / (float)p.E);
-  float eps = 0.f;
-  for (int a = 0; a < p.A; ++a) {
-    float part = 0.f;
+  const int H = p.lat.H, sample = row / H, tok = row % H, t = p.t, A = p.A;
+  RowV<NV> r;
+  load_row<NV>(p.a + (long long)row * p.E, lane, r);
+  pending_skips<NV>(p, row, sample, lane, r);        // a is rebuilt from x for the next step
+  layer_norm<NV>(r, p.lnf_g, p.lnf_b, lane, 1.f / (float)p.E);
+  // eps[a] = sum_e v[e] W_head[e][a]: this lane's 8 columns per chunk are 8
+  // consecutive rows of W_head, then one reduction per action dimension
+  float part[MAXA];
 #pragma unroll
-    for (int j = 0; j < NV; ++j) {
-      const float* w = p.head_w + (long long)(4 * lane + 128 * j) * p.A + a;
-      part = fmaf(v[j].x, w[0], part);
-      part = fmaf(v[j].y, w[p.A], part);
-      part = fmaf(v[j].z, w[2 * p.A], part);
-      part = fmaf(v[j].w, w[3 * p.A], part);
+  for (int a = 0; a < MAXA; ++a) part[a] = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float* w = p.head_w + (long long)(256 * j + 8 * lane + i) * A;
+      const float v = r.v[j][i];
+#pragma unroll
+      for (int a = 0; a < MAXA; ++a)
+        if (a < A) part[a] = fmaf(v, w[a], part[a]);
     }
-    part = warp_sum(part);
-    if (lane == a) eps = part + p.head_b[a];
+  float eps = 0.f;
+#pragma unroll
+  for (int a = 0; a < MAXA; ++a) {
+    if (a < A) {
+      const float e = warp_sum(part[a]);
+      if (lane == a) eps = e + p.head_b[a];
+    }
   }
   float xn = 0.f;
-  if (lane < p.A) {
+  if (lane < A) {
     const float* tb = p.stab + t * 8;
     const float inv_sa = tb[0], s1 = tb[1], cx0 = tb[2], cxt = tb[3], sig = tb[4], sab = tb[5], sabp = tb[6],
                 s1p = tb[7];
-    const float xv = p.x[(long long)row * p.A + lane];
+    const float xv = p.x[(long long)row * A + lane];
     float x0 = (xv - s1 * eps) * inv_sa;
     x0 = fminf(1.0f, fmaxf(-1.0f, x0));
     if (p.sampler == 0) {
-      const float z = p.noise[(((long long)(1 + t) * p.obs_mod + (sample % p.obs_mod)) * H + tok) * p.A + lane];
+      const float z = p.noise[(((long long)(1 + t) * p.obs_mod + (sample % p.obs_mod)) * H + tok) * A + lane];
       xn = cx0 * x0 + cxt * xv + sig * z;
     } else {
       xn = sabp * x0 + s1p * ((xv - sab * x0) / s1);
     }
-    p.x[(long long)row * p.A + lane] = xn;
+    p.x[(long long)row * A + lane] = xn;
   }
   if (t + 1 < p.lat.T) embed_row<NV>(p, row, lane, xn);
 }
@@ -329,80 +379,192 @@ struct AttnArgs {
   float scale;
 };
 
-// causal self-attention of one (sample, head) over its H action tokens
-__global__ void __launch_bounds__(128) sa_attn_kernel(const AttnArgs p) {
-  const int s = blockIdx.x, h = blockIdx.y;
-  if (!lat_refresh(p.lat, s, p.b, p.t)) return;
-  extern __shared__ float sm[];
-  const int H = p.lat.H, dh = p.dh, ld = dh + 1, E = p.E;
-  float* q = sm;
-  float* k = q + H * ld;
-  float* v = k + H * ld;
-  float* pr = v + H * ld;   // [H][H + 1]
-  const __nv_bfloat16* base = p.qkv + (long long)s * H * 3 * E + h * dh;
-  for (int idx = threadIdx.x; idx < H * dh / 2; idx += blockDim.x) {
-    const int i = idx / (dh / 2), d = 2 * (idx % (dh / 2));
-    const __nv_bfloat16* r = base + (long long)i * 3 * E + d;
-    const float2 fq = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r));
-    const float2 fk = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r + E));
-    const float2 fv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(r + 2 * E));
-    q[i * ld + d] = fq.x;
-    q[i * ld + d + 1] = fq.y;
-    k[i * ld + d] = fk.x;
-    k[i * ld + d + 1] = fk.y;
-    v[i * ld + d] = fv.x;
-    v[i * ld + d + 1] = fv.y;
-  }
-  __syncthreads();
-  for (int idx = threadIdx.x; idx < H * H; idx += blockDim.x) {
-    const int i = idx / H, j = idx % H;
-    float sc = -INFINITY;
-    if (j <= i) {
-      float d0 = 0.f, d1 = 0.f;
-      for (int e = 0; e < dh; e += 2) {
-        d0 = fmaf(q[i * ld + e], k[j * ld + e], d0);
-        d1 = fmaf(q[i * ld + e + 1], k[j * ld + e + 1], d1);
-      }
-      sc = (d0 + d1) * p.scale;
-    }
-    pr[i * (H + 1) + j] = sc;
-  }
-  __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = warp; i < H; i += blockDim.x >> 5) {
-    const float x = lane < H ? pr[i * (H + 1) + lane] : -INFINITY;
-    float mx = x;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    const float ex = x == -INFINITY ? 0.f : __expf(x - mx);
-    const float sum = warp_sum(ex);
-    if (lane < H) pr[i * (H + 1) + lane] = ex / sum;
-  }
-  __syncthreads();
-  for (int idx = threadIdx.x; idx < H * dh; idx += blockDim.x) {
-    const int i = idx / dh, d = idx % dh;
-    float o = 0.f;
-    for (int j = 0; j <= i; ++j) o = fmaf(pr[i * (H + 1) + j], v[j * ld + d], o);
-    p.att[((long long)s * H + i) * E + h * dh + d] = __float2bfloat16_rn(o);
-  }
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(tc::su32(p)));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(tc::su32(p)));
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack2(float x, float y) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  return *reinterpret_cast<uint32_t*>(&h);
 }
 
-// cross-attention of one (row, head) to the 1 + n_obs memory tokens
-template <int DH>
-__global__ void __launch_bounds__(128) ca_attn_kernel(const AttnArgs p) {
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  const int row = idx / p.nh, h = idx % p.nh;
-  if (row >= p.rows) return;
-  const int sample = row / p.lat.H;
-  if (!lat_refresh(p.lat, sample, p.b, p.t)) return;
-  const int E = p.E, Cm = 1 + p.n_obs;
-  float q[DH];
-  const __nv_bfloat16* qr = p.qkv + (long long)row * E + h * DH;
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tc::su32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+constexpr int SA_DH = 64, SA_LDS = SA_DH + 8;   // head size; shared row stride (bf16), conflict-free ldmatrix
+constexpr int SA_WARPS = 4;
+
+// Causal self-attention of one (sample, head) per warp on the tensor cores
+// (mma.sync m16n8k16, bf16 in, fp32 accumulate): S = Q K^T over the H action
+// tokens, masked softmax on the accumulators, O = P V with P taken straight
+// from the score registers.
+template <int MT>   // H = 16 MT
+__global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p) {
+  constexpr int H = 16 * MT, NKT = H / 8;
+  const int s = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y * SA_WARPS + warp;
+  if (!lat_refresh(p.lat, s, p.b, p.t)) return;
+  extern __shared__ __align__(16) uint8_t sa_smem[];
+  __nv_bfloat16* sq = reinterpret_cast<__nv_bfloat16*>(sa_smem) + warp * 3 * H * SA_LDS;
+  __nv_bfloat16* sk = sq + H * SA_LDS;
+  __nv_bfloat16* sv = sk + H * SA_LDS;
+  if (h >= p.nh) return;
+  const int E = p.E;
+  const __nv_bfloat16* base = p.qkv + (long long)s * H * 3 * E + h * SA_DH;
+  for (int c = lane; c < H * 24; c += 32) {          // per token: q, k, v rows of 8 x 16 bytes
+    const int i = c / 24, rem = c - i * 24, which = rem >> 3, ch = rem & 7;
+    cp_async16(sq + which * H * SA_LDS + i * SA_LDS + ch * 8, base + (long long)i * 3 * E + which * E + ch * 8);
+  }
+  cp_async_wait_all();
+  __syncwarp();
+  const int g = lane >> 2, tq = lane & 3;
+  float sc[MT][NKT][4];
 #pragma unroll
-  for (int d = 0; d < DH; d += 2) {
-    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(qr + d));
-    q[d] = f.x;
-    q[d + 1] = f.y;
+  for (int m = 0; m < MT; ++m)
+#pragma unroll
+    for (int n = 0; n < NKT; ++n) sc[m][n][0] = sc[m][n][1] = sc[m][n][2] = sc[m][n][3] = 0.f;
+#pragma unroll
+  for (int k2 = 0; k2 < SA_DH / 32; ++k2) {           // 32 head dims = two k-steps per pass
+    uint32_t a0[MT][4], a1[MT][4];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      const __nv_bfloat16* qa = sq + (m * 16 + (lane & 15)) * SA_LDS + k2 * 32 + (lane >> 4) * 8;
+      ldsm_x4(a0[m], qa);
+      ldsm_x4(a1[m], qa + 16);
+    }
+#pragma unroll
+    for (int n = 0; n < NKT; ++n) {
+      uint32_t b[4];
+      ldsm_x4(b, sk + (n * 8 + (lane & 7)) * SA_LDS + k2 * 32 + (lane >> 3) * 8);
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        mma16816(sc[m][n], a0[m], b[0], b[1]);
+        mma16816(sc[m][n], a1[m], b[2], b[3]);
+      }
+    }
+  }
+  // causal mask, softmax over keys (rows g and g + 8 of each m-tile)
+  float inv[MT][2];
+#pragma unroll
+  for (int m = 0; m < MT; ++m) {
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int n = 0; n < NKT; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int row = m * 16 + g + (e >> 1) * 8, col = n * 8 + 2 * tq + (e & 1);
+        const float v = col <= row ? sc[m][n][e] * p.scale : -INFINITY;
+        sc[m][n][e] = v;
+        mx[e >> 1] = fmaxf(mx[e >> 1], v);
+      }
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      mx[hh] = fmaxf(mx[hh], __shfl_xor_sync(0xffffffffu, mx[hh], 1));
+      mx[hh] = fmaxf(mx[hh], __shfl_xor_sync(0xffffffffu, mx[hh], 2));
+    }
+    float sum[2] = {0.f, 0.f};
+#pragma unroll
+    for (int n = 0; n < NKT; ++n)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float v = sc[m][n][e] == -INFINITY ? 0.f : __expf(sc[m][n][e] - mx[e >> 1]);
+        sc[m][n][e] = v;
+        sum[e >> 1] += v;
+      }
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      sum[hh] += __shfl_xor_sync(0xffffffffu, sum[hh], 1);
+      sum[hh] += __shfl_xor_sync(0xffffffffu, sum[hh], 2);
+      inv[m][hh] = 1.f / sum[hh];
+    }
+  }
+  // O = P V
+  float o[MT][SA_DH / 8][4];
+#pragma unroll
+  for (int m = 0; m < MT; ++m)
+#pragma unroll
+    for (int n = 0; n < SA_DH / 8; ++n) o[m][n][0] = o[m][n][1] = o[m][n][2] = o[m][n][3] = 0.f;
+#pragma unroll
+  for (int kk = 0; kk < H / 16; ++kk) {
+    uint32_t a[MT][4];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      a[m][0] = pack2(sc[m][2 * kk][0], sc[m][2 * kk][1]);
+      a[m][1] = pack2(sc[m][2 * kk][2], sc[m][2 * kk][3]);
+      a[m][2] = pack2(sc[m][2 * kk + 1][0], sc[m][2 * kk + 1][1]);
+      a[m][3] = pack2(sc[m][2 * kk + 1][2], sc[m][2 * kk + 1][3]);
+    }
+#pragma unroll
+    for (int n2 = 0; n2 < SA_DH / 16; ++n2) {
+      uint32_t b[4];
+      ldsm_x4_t(b, sv + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * SA_LDS + n2 * 16 + (lane >> 4) * 8);
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        mma16816(o[m][2 * n2], a[m], b[0], b[1]);
+        mma16816(o[m][2 * n2 + 1], a[m], b[2], b[3]);
+      }
+    }
+  }
+#pragma unroll
+  for (int m = 0; m < MT; ++m)
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      __nv_bfloat16* dst = p.att + ((long long)s * H + m * 16 + g + hh * 8) * E + h * SA_DH + 2 * tq;
+#pragma unroll
+      for (int n = 0; n < SA_DH / 8; ++n)
+        *reinterpret_cast<uint32_t*>(dst + n * 8) =
+            pack2(o[m][n][2 * hh] * inv[m][hh], o[m][n][2 * hh + 1] * inv[m][hh]);
+    }
+}
+
+// Cross-attention to the 1 + n_obs memory tokens: a block per sample with
+// every head's memory keys/values staged in shared memory, a warp per head, a
+// lane per action token (row).
+template <int DH>
+__global__ void __launch_bounds__(256) ca_attn_kernel(const AttnArgs p) {
+  const int s = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (!lat_refresh(p.lat, s, p.b, p.t)) return;
+  extern __shared__ __align__(16) float kv[];      // [Cm][2E]
+  const int E = p.E, Cm = 1 + p.n_obs;
+  for (int v = threadIdx.x; v < Cm * E / 2; v += blockDim.x) {
+    const int j = v / (E / 2), c = v - j * (E / 2);
+    const float* src = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
+                              : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
+    reinterpret_cast<float4*>(kv + j * 2 * E)[c] = reinterpret_cast<const float4*>(src)[c];
+  }
+  __syncthreads();
+  const int H = p.lat.H;
+  if (warp >= p.nh || lane >= H) return;
+  const int h = warp, row = s * H + lane;
+  float q[DH];
+  const uint4* qr = reinterpret_cast<const uint4*>(p.qkv + (long long)row * E + h * DH);
+#pragma unroll
+  for (int c = 0; c < DH / 8; ++c) {
+    const uint4 raw = qr[c];
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+      q[8 * c + 2 * i] = f.x;
+      q[8 * c + 2 * i + 1] = f.y;
+    }
   }
   constexpr int MAXC = 8;
   float sc[MAXC];
@@ -411,19 +573,14 @@ __global__ void __launch_bounds__(128) ca_attn_kernel(const AttnArgs p) {
   for (int j = 0; j < MAXC; ++j) {
     sc[j] = -INFINITY;
     if (j < Cm) {
-      const float* kr = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
-                               : p.kv_obs + (((long long)(sample % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
-      kr += h * DH;
-      float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+      const float* kr = kv + j * 2 * E + h * DH;
+      float d0 = 0.f, d1 = 0.f;
 #pragma unroll
-      for (int d = 0; d < DH; d += 4) {
-        const float4 kk = *reinterpret_cast<const float4*>(kr + d);
-        d0 = fmaf(q[d], kk.x, d0);
-        d1 = fmaf(q[d + 1], kk.y, d1);
-        d2 = fmaf(q[d + 2], kk.z, d2);
-        d3 = fmaf(q[d + 3], kk.w, d3);
+      for (int d = 0; d < DH; d += 2) {
+        d0 = fmaf(q[d], kr[d], d0);
+        d1 = fmaf(q[d + 1], kr[d + 1], d1);
       }
-      sc[j] = ((d0 + d1) + (d2 + d3)) * p.scale;
+      sc[j] = (d0 + d1) * p.scale;
       mx = fmaxf(mx, sc[j]);
     }
   }
@@ -439,24 +596,18 @@ __global__ void __launch_bounds__(128) ca_attn_kernel(const AttnArgs p) {
 #pragma unroll
   for (int j = 0; j < MAXC; ++j) {
     if (j < Cm) {
-      const float* vr = (j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
-                                : p.kv_obs + (((long long)(sample % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E) +
-                        E + h * DH;
+      const float* vr = kv + j * 2 * E + E + h * DH;
       const float w = sc[j] * inv;
 #pragma unroll
-      for (int d = 0; d < DH; d += 4) {
-        const float4 vv = *reinterpret_cast<const float4*>(vr + d);
-        q[d] = fmaf(w, vv.x, q[d]);
-        q[d + 1] = fmaf(w, vv.y, q[d + 1]);
-        q[d + 2] = fmaf(w, vv.z, q[d + 2]);
-        q[d + 3] = fmaf(w, vv.w, q[d + 3]);
-      }
+      for (int d = 0; d < DH; ++d) q[d] = fmaf(w, vr[d], q[d]);
     }
   }
-  __nv_bfloat16* o = p.att + (long long)row * E + h * DH;
+  uint4* o = reinterpret_cast<uint4*>(p.att + (long long)row * E + h * DH);
 #pragma unroll
-  for (int d = 0; d < DH; d += 2) *reinterpret_cast<__nv_bfloat162*>(o + d) = __floats2bfloat162_rn(q[d], q[d + 1]);
+  for (int c = 0; c < DH / 8; ++c) o[c] = pack_bf16x8(q + 8 * c);
 }
+
+size_t sa_smem_bytes(int H) { return (size_t)SA_WARPS * 3 * H * SA_LDS * sizeof(__nv_bfloat16); }
 
 }  // namespace
 
@@ -504,9 +655,9 @@ cudaError_t launch_rows(int which, const RowArgs& p, cudaStream_t st) {
 }
 
 cudaError_t rows_kernel(int which, const RowArgs& p, cudaStream_t st) {
-  switch (p.E / 128) {
+  switch (p.E / 256) {
+    case 1: return launch_rows<1>(which, p, st);
     case 2: return launch_rows<2>(which, p, st);
-    case 4: return launch_rows<4>(which, p, st);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -515,8 +666,9 @@ cudaError_t rows_kernel(int which, const RowArgs& p, cudaStream_t st) {
 
 bool wide_supported(const evo_config* c) {
   const int E = c->n_emb, dh = E / c->n_head;
-  return c->dtype == EVO_DTYPE_BF16 && (E == 256 || E == 512) && dh == 64 && c->horizon <= 32 &&
-         128 % c->horizon == 0 && c->action_dim <= 32 && 1 + c->n_obs <= 8 && encode_fn() != nullptr;
+  return c->dtype == EVO_DTYPE_BF16 && (E == 256 || E == 512) && dh == 64 && (c->horizon == 16 || c->horizon == 32) &&
+         c->action_dim <= MAXA && c->n_head <= 8 && 1 + c->n_obs <= 8 && 3 * c->n_layer <= 64 &&
+         encode_fn() != nullptr;
 }
 
 int wide_create(WideState** out, const evo_config* c, const float* weights, const float* wf32_dev, const int* woff,
@@ -598,6 +750,11 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
                            tc::SMEM_BYTES) != cudaSuccess ||
       cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            tc::SMEM_BYTES) != cudaSuccess)
+    return fail(EVO_ERR_CUDA);
+  if (cudaFuncSetAttribute(sa_attn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(16)) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(sa_attn_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(32)) !=
+          cudaSuccess)
     return fail(EVO_ERR_CUDA);
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(EVO_ERR_CUDA);
   *out = w;
@@ -708,7 +865,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   ap.kv_time = c.kv_time;
   ap.kv_obs = c.kv_obs;
   ap.scale = 1.f / std::sqrt((float)w->dh);
-  const size_t sa_smem = (size_t)(3 * H * (w->dh + 1) + H * (H + 1)) * sizeof(float);
+  const size_t sa_smem = sa_smem_bytes(H);
+  const size_t ca_smem = (size_t)(1 + w->n_obs) * 2 * E * sizeof(float);
 
   for (int t = 0; t < T; ++t) {
     int lo = 0;
@@ -738,7 +896,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.ldo = 3 * E;
         WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, st));
         ap.qkv = w->qkv;
-        sa_attn_kernel<<<dim3(c.samples, w->nh), 128, sa_smem, st>>>(ap);
+        if (H == 32) sa_attn_kernel<2><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
+        else sa_attn_kernel<1><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 3 * E;
         g.bias = wl(w, l, WL_SA_BO);
@@ -751,7 +910,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.ldo = E;
         WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, st));
         ap.qkv = w->qkv;
-        ca_attn_kernel<64><<<(int)((R * w->nh + 127) / 128), 128, 0, st>>>(ap);
+        ca_attn_kernel<64><<<c.samples, 32 * w->nh, ca_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 5 * E;
         g.bias = wl(w, l, WL_CA_BO);
