@@ -2,18 +2,20 @@
 // on the fifth-generation tensor cores (tcgen05), bf16 operands, fp32
 // accumulation in tensor memory, with the epilogues the denoiser needs fused.
 //
-// One CTA computes one BM x BN tile:
+// Persistent: a CTA per SM walks the BM x BN output tiles (m-major, so
+// consecutive tiles reuse the same rows of A from L2), warp-specialised:
 //   * warp 0, one lane: TMA producer.  Tiles of A (BM x 64) and B (BN x 64)
-//     land in a ring of STAGES shared-memory stages with the 128-byte swizzle
+//     land in a ring of shared-memory stages with the 128-byte swizzle
 //     (cp.async.bulk.tensor + mbarrier transaction counts);
 //   * warp 1, one lane: MMA issuer.  Four tcgen05.mma (K = 16 each) per stage
-//     into one TMEM accumulator of BN columns; tcgen05.commit frees the stage
-//     when the MMAs that read it are done, and signals the epilogue at the end;
-//   * all four warps: epilogue.  Warp w owns TMEM lanes (= tile rows)
-//     32w..32w+31 and reads 32 columns at a time with tcgen05.ld.
-// BM = 128, BN = 128 and three stages (97 KB of shared memory, 128 TMEM
-// columns) let two CTAs share an SM, so one CTA's epilogue overlaps the other's
-// main loop.
+//     into one of two TMEM accumulators of BN columns; tcgen05.commit frees a
+//     stage when the MMAs that read it are done, and hands a finished
+//     accumulator to the epilogue;
+//   * warps 2-5: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
+//     quadrant 32 (w % 4) .. +31, 32 columns at a time (tcgen05.ld), applies
+//     bias / GELU / residual-and-cache, stores, and releases the accumulator.
+// With two accumulators the epilogue of one tile overlaps the main loop of the
+// next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
 // Every wait on an mbarrier is bounded: on expiry the thread records
 // ST_TIMEOUT in the status word and carries on, so the kernel always ends.
@@ -28,12 +30,23 @@
 namespace evo {
 namespace tc {
 
-constexpr int BM = 128, BN = 128, BK = 64, STAGES = 3;
+constexpr int BM = 128, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 128;   // alignment slack, stages, barriers
+constexpr int NTHREADS_GEMM = 192;                              // producer, MMA, four epilogue warps
 constexpr long long TC_WAIT_LIMIT = 1ll << 26;                  // polls before a wait gives up
+
+template <int BN>
+struct TileCfg {
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;   // alignment slack, stages, barriers
+  static constexpr int TMEM_COLS = 2 * BN;                                // two accumulators
+  // instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+  // K-major, M = BM, N = BN
+  static constexpr uint32_t IDESC =
+      (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+};
 
 enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2 };
 
@@ -83,6 +96,10 @@ __device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, int* s
   atomicOr(status, ST_TIMEOUT);
 }
 
+__device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(bar)) : "memory");
+}
+
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes) : "memory");
 }
@@ -121,15 +138,11 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
-// K-major, M = BM, N = BN.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-
-__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t accumulate) {
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
           tmem_d),
-      "l"(a), "l"(b), "r"(IDESC), "r"(accumulate)
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 
@@ -164,36 +177,98 @@ __device__ __forceinline__ bool row_refreshes(const GemmArgs& g, int row) {
 
 __device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
 
-// ---------------------------------------------------------------- the kernel
+// does any row of the tile starting at m0 refresh?  (the same answer in every role)
+__device__ __forceinline__ bool tile_live(const GemmArgs& g, int m0) {
+  if (m0 >= g.rows) return false;
+  if (!g.S || (g.force && g.t == 0)) return true;
+  const int last = min(m0 + BM, g.rows) - 1;
+  for (int s = m0 / g.H; s <= last / g.H; ++s)
+    if (g.S[(long long)(s / g.per_sched) * g.S_stride + (long long)g.srow * g.T + g.t] != 0) return true;
+  return false;
+}
+
 template <int MODE>
-__global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmA,
-                                                      const __grid_constant__ CUtensorMap tmB, const GemmArgs g) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n, float (&v)[32]) {
+  const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 bb = __ldg(b4 + q);
+    v[4 * q] += bb.x;
+    v[4 * q + 1] += bb.y;
+    v[4 * q + 2] += bb.z;
+    v[4 * q + 3] += bb.w;
+  }
+  if constexpr (MODE == EPI_RESID) {
+    float4* a4 = reinterpret_cast<float4*>(g.resid + (long long)row * g.ldr + n);
+    uint4* c4 = reinterpret_cast<uint4*>(g.cache + (long long)row * g.ldr + n);
+    float4 av[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) av[q] = a4[q];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 pk;
+      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
+        pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+      }
+      c4[q] = pk;
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      av[q].x += v[4 * q];
+      av[q].y += v[4 * q + 1];
+      av[q].z += v[4 * q + 2];
+      av[q].w += v[4 * q + 3];
+      a4[q] = av[q];
+    }
+  } else {
+    if constexpr (MODE == EPI_GELU_BF16) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
+    }
+    uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint4 pk;
+      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
+        pw[j] = *reinterpret_cast<uint32_t*>(&h2);
+      }
+      o4[q] = pk;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- the kernel
+// Tiles: m_tiles x n_tiles, tile i -> (i / n_tiles, i % n_tiles); CTA c takes
+// tiles c, c + gridDim.x, ...
+template <int MODE, int BN>
+__global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                                                                const __grid_constant__ CUtensorMap tmB,
+                                                                const GemmArgs g, int m_tiles, int n_tiles) {
+  using C = TileCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // a tile none of whose rows refresh has nothing to do (uniform over the CTA)
-  if (g.S) {
-    const int r = m0 + lane * 4;   // 128 rows, 4 per lane: any refreshing row keeps the tile
-    const bool any = row_refreshes(g, r) || row_refreshes(g, r + 1) || row_refreshes(g, r + 2) ||
-                     row_refreshes(g, r + 3);
-    if (!__any_sync(0xffffffffu, any)) return;
-  } else if (m0 >= g.rows) {
-    return;
-  }
-
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-  uint64_t* empty = full + STAGES;
-  uint64_t* accb = empty + STAGES;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
-  if (warp == 0) tmem_alloc(tslot, BN);
-  if (threadIdx.x == 32) {
-    for (int s = 0; s < STAGES; ++s) {
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;     // [2]: accumulator ready for the epilogue
+  uint64_t* tempty = tfull + 2;            // [2]: accumulator drained by the epilogue
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tempty + 2);
+  if (warp == 1) tmem_alloc(tslot, C::TMEM_COLS);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
       mbar_init1(&full[s], 1);
       mbar_init1(&empty[s], 1);
     }
-    mbar_init1(accb, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init1(&tfull[a], 1);
+      mbar_init1(&tempty[a], 4);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -201,100 +276,76 @@ __global__ void __launch_bounds__(128, 1) gemm_kernel(const __grid_constant__ CU
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const int KB = g.K / BK;
+  const int KB = g.K / BK, total = m_tiles * n_tiles;
 
-  if (warp == 0 && lane == 0) {
-    // producer
-    for (int kb = 0; kb < KB; ++kb) {
-      const int s = kb % STAGES;
-      if (kb >= STAGES) mbar_wait(&empty[s], (uint32_t)((kb / STAGES) - 1) & 1u, g.status);
-      uint8_t* sa = smem + s * STAGE_BYTES;
-      mbar_expect_tx(&full[s], STAGE_BYTES);
-      tma_load_2d(sa, &tmA, kb * BK, m0, &full[s]);
-      tma_load_2d(sa + A_BYTES, &tmB, kb * BK, g.b_row0 + n0, &full[s]);
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t q = 0;
+      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+        if (!tile_live(g, m0)) continue;
+        for (int kb = 0; kb < KB; ++kb, ++q) {
+          const int s = q % C::STAGES;
+          mbar_wait(&empty[s], ((q / C::STAGES) & 1u) ^ 1u, g.status);
+          uint8_t* sa = smem + s * C::STAGE_BYTES;
+          mbar_expect_tx(&full[s], C::STAGE_BYTES);
+          tma_load_2d(sa, &tmA, kb * BK, m0, &full[s]);
+          tma_load_2d(sa + A_BYTES, &tmB, kb * BK, g.b_row0 + n0, &full[s]);
+        }
+      }
     }
-  } else if (warp == 1 && lane == 0) {
-    // MMA issuer
-    for (int kb = 0; kb < KB; ++kb) {
-      const int s = kb % STAGES;
-      mbar_wait(&full[s], (uint32_t)(kb / STAGES) & 1u, g.status);
-      tc_fence_after();
-      const uint32_t sa = su32(smem + s * STAGE_BYTES);
-      const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t q = 0, it = 0;
+      for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+        if (!tile_live(g, (tile / n_tiles) * BM)) continue;
+        const uint32_t acc = it & 1u;
+        mbar_wait(&tempty[acc], ((it >> 1) & 1u) ^ 1u, g.status);
+        tc_fence_after();
+        const uint32_t d = tmem + acc * BN;
+        for (int kb = 0; kb < KB; ++kb, ++q) {
+          const int s = q % C::STAGES;
+          mbar_wait(&full[s], (q / C::STAGES) & 1u, g.status);
+          tc_fence_after();
+          const uint32_t sa = su32(smem + s * C::STAGE_BYTES);
+          const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
 #pragma unroll
-      for (int k = 0; k < BK / 16; ++k)   // +32 bytes along K = +2 in the encoded start address
-        mma_f16(tmem, da + 2 * k, db + 2 * k, (kb | k) != 0);
-      mma_commit(&empty[s]);
+          for (int k = 0; k < BK / 16; ++k)   // +32 bytes along K = +2 in the encoded start address
+            mma_f16(d, da + 2 * k, db + 2 * k, C::IDESC, (kb | k) != 0);
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&tfull[acc]);
+        ++it;
+      }
     }
-    mma_commit(accb);
+  } else {
+    // epilogue warps: TMEM lane quadrant (warp % 4) = tile rows 32 (warp % 4) ..
+    const int quad = warp & 3;
+    uint32_t it = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
+      const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
+      if (!tile_live(g, m0)) continue;
+      const uint32_t acc = it & 1u;
+      mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status);
+      tc_fence_after();
+      const int row = m0 + quad * 32 + lane;
+      const bool live = MODE == EPI_RESID ? row_refreshes(g, row) : row < g.rows;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
+        if (live) epilogue_chunk<MODE>(g, row, n0 + c * 32, v);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive1(&tempty[acc]);
+      ++it;
+    }
   }
   __syncwarp();
-  mbar_wait(accb, 0, g.status);
-  tc_fence_after();
-
-  // epilogue: thread = one row, 32 columns per TMEM load
-  const int row = m0 + warp * 32 + lane;
-  const bool live = MODE == EPI_RESID ? row_refreshes(g, row) : row < g.rows;
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    float v[32];
-    tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(c * 32), v);
-    const int n = n0 + c * 32;
-    if (!live) continue;
-    const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const float4 bb = __ldg(b4 + q);
-      v[4 * q] += bb.x;
-      v[4 * q + 1] += bb.y;
-      v[4 * q + 2] += bb.z;
-      v[4 * q + 3] += bb.w;
-    }
-    if constexpr (MODE == EPI_RESID) {
-      float4* a4 = reinterpret_cast<float4*>(g.resid + (long long)row * g.ldr + n);
-      uint4* c4 = reinterpret_cast<uint4*>(g.cache + (long long)row * g.ldr + n);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint4 pk;
-        uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
-          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-        c4[q] = pk;
-      }
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        float4 a = a4[q];
-        a.x += v[4 * q];
-        a.y += v[4 * q + 1];
-        a.z += v[4 * q + 2];
-        a.w += v[4 * q + 3];
-        a4[q] = a;
-      }
-    } else {
-      if constexpr (MODE == EPI_GELU_BF16) {
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
-      }
-      uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        uint4 pk;
-        uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
-          pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-        }
-        o4[q] = pk;
-      }
-    }
-  }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, BN);
+  if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
 }
 
 }  // namespace tc

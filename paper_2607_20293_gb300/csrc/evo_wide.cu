@@ -612,6 +612,11 @@ size_t sa_smem_bytes(int H) { return (size_t)SA_WARPS * 3 * H * SA_LDS * sizeof(
 }  // namespace
 
 // ---------------------------------------------------------------- state
+// B operands: one tensor map per weight matrix and tile width
+struct BMaps {
+  CUtensorMap n128, n256;
+};
+
 struct WideState {
   int L = 0, E = 0, nh = 0, dh = 0, H = 0, A = 0, n_obs = 0, T = 0, U = 0, sampler = 0, force = 0;
   long long rmax = 0;     // rows the buffers hold (multiple of BM)
@@ -627,7 +632,9 @@ struct WideState {
   __nv_bfloat16* cache = nullptr;   // [U][rmax][E]
   float* a = nullptr;               // [rmax][E]
   int* first = nullptr;             // [max_sched][U]
-  CUtensorMap mA_xln, mA_att, mA_hid, mB_e, mB_4e;
+  CUtensorMap mA_xln, mA_att, mA_hid;
+  BMaps mB_e, mB_4e;
+  int num_sms = 0;
   std::vector<uint8_t> any;         // [U][T] scratch: some lattice refreshes (b, t)
   long long launches = 0;
 };
@@ -639,10 +646,25 @@ const float* wl(const WideState* w, int l, int id) {
 }
 
 template <int MODE>
-cudaError_t gemm(const CUtensorMap& ma, const CUtensorMap& mb, const tc::GemmArgs& g, int rows_p, int N,
+cudaError_t gemm(const CUtensorMap& ma, const BMaps& mb, const tc::GemmArgs& g, int rows_p, int N, int num_sms,
                  cudaStream_t st) {
-  tc::gemm_kernel<MODE><<<dim3(rows_p / tc::BM, N / tc::BN), 128, tc::SMEM_BYTES, st>>>(ma, mb, g);
+  const int m_tiles = rows_p / tc::BM;
+  if (N % 256 == 0 && m_tiles * (N / 256) >= num_sms) {
+    const int total = m_tiles * (N / 256);
+    tc::gemm_kernel<MODE, 256><<<std::min(total, num_sms), tc::NTHREADS_GEMM, tc::TileCfg<256>::SMEM_BYTES, st>>>(
+        ma, mb.n256, g, m_tiles, N / 256);
+  } else {
+    const int total = m_tiles * (N / 128);
+    tc::gemm_kernel<MODE, 128><<<std::min(total, num_sms), tc::NTHREADS_GEMM, tc::TileCfg<128>::SMEM_BYTES, st>>>(
+        ma, mb.n128, g, m_tiles, N / 128);
+  }
   return cudaGetLastError();
+}
+
+template <int MODE, int BN>
+cudaError_t gemm_attr() {
+  return cudaFuncSetAttribute(tc::gemm_kernel<MODE, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              tc::TileCfg<BN>::SMEM_BYTES);
 }
 
 template <int NV>
@@ -741,16 +763,22 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
   cudaMemset(w->att, 0, R * E * 2);
   cudaMemset(w->hid, 0, R * 4 * E * 2);
   if (!make_map(&w->mA_xln, w->xln, R, E, tc::BM) || !make_map(&w->mA_att, w->att, R, E, tc::BM) ||
-      !make_map(&w->mA_hid, w->hid, R, 4 * E, tc::BM) || !make_map(&w->mB_e, w->wt_e, (long long)L * 10 * E, E, tc::BN) ||
-      !make_map(&w->mB_4e, w->wt_4e, (long long)L * E, 4 * E, tc::BN))
+      !make_map(&w->mA_hid, w->hid, R, 4 * E, tc::BM) ||
+      !make_map(&w->mB_e.n128, w->wt_e, (long long)L * 10 * E, E, 128) ||
+      !make_map(&w->mB_e.n256, w->wt_e, (long long)L * 10 * E, E, 256) ||
+      !make_map(&w->mB_4e.n128, w->wt_4e, (long long)L * E, 4 * E, 128) ||
+      !make_map(&w->mB_4e.n256, w->wt_4e, (long long)L * E, 4 * E, 256))
     return fail(EVO_ERR_CUDA);
-  if (cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           tc::SMEM_BYTES) != cudaSuccess ||
-      cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_GELU_BF16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           tc::SMEM_BYTES) != cudaSuccess ||
-      cudaFuncSetAttribute(tc::gemm_kernel<tc::EPI_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           tc::SMEM_BYTES) != cudaSuccess)
+  if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
+      gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
+      gemm_attr<tc::EPI_RESID, 128>() != cudaSuccess || gemm_attr<tc::EPI_RESID, 256>() != cudaSuccess)
     return fail(EVO_ERR_CUDA);
+  {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&w->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || w->num_sms <= 0)
+      return fail(EVO_ERR_CUDA);
+  }
   if (cudaFuncSetAttribute(sa_attn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(16)) !=
           cudaSuccess ||
       cudaFuncSetAttribute(sa_attn_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(32)) !=
@@ -894,38 +922,38 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.bias = wl(w, l, WL_SA_BQKV);
         g.out = w->qkv;
         g.ldo = 3 * E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, st));
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, st));
         ap.qkv = w->qkv;
         if (H == 32) sa_attn_kernel<2><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
         else sa_attn_kernel<1><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 3 * E;
         g.bias = wl(w, l, WL_SA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, st));
       } else if (u == 1) {
         g.K = E;
         g.b_row0 = rowE + 4 * E;
         g.bias = wl(w, l, WL_CA_BQ);
         g.out = w->qkv;
         g.ldo = E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, st));
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, st));
         ap.qkv = w->qkv;
         ca_attn_kernel<64><<<c.samples, 32 * w->nh, ca_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 5 * E;
         g.bias = wl(w, l, WL_CA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, st));
       } else {
         g.K = E;
         g.b_row0 = rowE + 6 * E;
         g.bias = wl(w, l, WL_FF_B1);
         g.out = w->hid;
         g.ldo = 4 * E;
-        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, st));
+        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, st));
         g.K = 4 * E;
         g.b_row0 = l * E;
         g.bias = wl(w, l, WL_FF_B2);
-        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, st));
       }
     }
     rp.lo = lo;
