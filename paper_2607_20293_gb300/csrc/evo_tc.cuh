@@ -11,9 +11,10 @@
 //     into one of two TMEM accumulators of BN columns; tcgen05.commit frees a
 //     stage when the MMAs that read it are done, and hands a finished
 //     accumulator to the epilogue;
-//   * warps 2-5: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
-//     quadrant 32 (w % 4) .. +31, 32 columns at a time (tcgen05.ld), applies
-//     bias / GELU / residual-and-cache, stores, and releases the accumulator.
+//   * warps 2-9: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
+//     quadrant 32 (w % 4) .. +31 and one half of the tile's columns, 32 at a
+//     time (tcgen05.ld), applies bias / GELU / residual-and-cache, stores, and
+//     releases the accumulator.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
 // next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
@@ -32,7 +33,8 @@ namespace tc {
 
 constexpr int BM = 128, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int NTHREADS_GEMM = 192;                              // producer, MMA, four epilogue warps
+constexpr int EPI_WARPS = 8;                                    // two per TMEM lane quadrant
+constexpr int NTHREADS_GEMM = 32 * (2 + EPI_WARPS);             // producer, MMA, epilogue warps
 constexpr long long TC_WAIT_LIMIT = 1ll << 26;                  // polls before a wait gives up
 
 template <int BN>
@@ -267,7 +269,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init1(&tfull[a], 1);
-      mbar_init1(&tempty[a], 4);
+      mbar_init1(&tempty[a], EPI_WARPS);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -319,8 +321,9 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       }
     }
   } else {
-    // epilogue warps: TMEM lane quadrant (warp % 4) = tile rows 32 (warp % 4) ..
-    const int quad = warp & 3;
+    // epilogue warps: TMEM lane quadrant (warp % 4) = tile rows 32 (warp % 4) ..,
+    // column half (warp - 2) / 4
+    const int quad = warp & 3, half = (warp - 2) >> 2;
     uint32_t it = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
@@ -331,7 +334,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       const int row = m0 + quad * 32 + lane;
       const bool live = MODE == EPI_RESID ? row_refreshes(g, row) : row < g.rows;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
         float v[32];
         tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
         if (live) epilogue_chunk<MODE>(g, row, n0 + c * 32, v);

@@ -12,8 +12,8 @@
 //       prep_kernel   rows: a += c_k for the units k since the previous prep that
 //                     the row's lattice skipped (a cache that was never written
 //                     holds zero: skipped); then LN_b(a) -> xln for refreshing rows
-//       SA:  GEMM xln W_qkv (bf16 out) -> sa_attn_kernel -> GEMM attn W_o (+= a, -> c_b)
-//       CA:  GEMM xln W_q -> ca_attn_kernel (memory tokens) -> GEMM attn W_o (+= a, -> c_b)
+//       SA:  GEMM xln W_qkv (bf16 out) -> attention (causal) -> GEMM attn W_o (+= a, -> c_b)
+//       CA:  GEMM xln W_q -> attention (memory tokens) -> GEMM attn W_o (+= a, -> c_b)
 //       FFN: GEMM xln W_1 (GELU, bf16 out) -> GEMM h W_2 (+= a, -> c_b)
 //     head_kernel     pending skips, LN_f, eps = . W_head + b_head, sampler step
 //                     (DDPM / DDIM), next step's input embedding
@@ -133,7 +133,7 @@ struct RowArgs {
   int sampler;
   const float* lnf_g;
   const float* lnf_b;
-  const float* head_w;            // [E][A]
+  const float* head_wt;           // [A][E] (W_head transposed)
   const float* head_b;            // [A]
   const float* in_w;              // [A][E]
   const float* in_b;              // [E]
@@ -326,28 +326,27 @@ __global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
   load_row<NV>(p.a + (long long)row * p.E, lane, r);
   pending_skips<NV>(p, row, sample, lane, r);        // a is rebuilt from x for the next step
   layer_norm<NV>(r, p.lnf_g, p.lnf_b, lane, 1.f / (float)p.E);
-  // eps[a] = sum_e v[e] W_head[e][a]: this lane's 8 columns per chunk are 8
-  // consecutive rows of W_head, then one reduction per action dimension
-  float part[MAXA];
-#pragma unroll
-  for (int a = 0; a < MAXA; ++a) part[a] = 0.f;
-#pragma unroll
-  for (int j = 0; j < NV; ++j)
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float* w = p.head_w + (long long)(256 * j + 8 * lane + i) * A;
-      const float v = r.v[j][i];
-#pragma unroll
-      for (int a = 0; a < MAXA; ++a)
-        if (a < A) part[a] = fmaf(v, w[a], part[a]);
-    }
+  // eps[a] = sum_e v[e] W_head[e][a] over this lane's columns (coalesced rows
+  // of W_head^T), then one reduction per action dimension
   float eps = 0.f;
+  for (int a = 0; a < A; ++a) {
+    const float* w = p.head_wt + (long long)a * p.E + 8 * lane;
+    float part = 0.f;
 #pragma unroll
-  for (int a = 0; a < MAXA; ++a) {
-    if (a < A) {
-      const float e = warp_sum(part[a]);
-      if (lane == a) eps = e + p.head_b[a];
+    for (int j = 0; j < NV; ++j) {
+      const float4 w0 = *reinterpret_cast<const float4*>(w + 256 * j);
+      const float4 w1 = *reinterpret_cast<const float4*>(w + 256 * j + 4);
+      part = fmaf(r.v[j][0], w0.x, part);
+      part = fmaf(r.v[j][1], w0.y, part);
+      part = fmaf(r.v[j][2], w0.z, part);
+      part = fmaf(r.v[j][3], w0.w, part);
+      part = fmaf(r.v[j][4], w1.x, part);
+      part = fmaf(r.v[j][5], w1.y, part);
+      part = fmaf(r.v[j][6], w1.z, part);
+      part = fmaf(r.v[j][7], w1.w, part);
     }
+    part = warp_sum(part);
+    if (lane == a) eps = part + p.head_b[a];
   }
   float xn = 0.f;
   if (lane < A) {
@@ -411,26 +410,52 @@ __device__ __forceinline__ void cp_async_wait_all() {
 constexpr int SA_DH = 64, SA_LDS = SA_DH + 8;   // head size; shared row stride (bf16), conflict-free ldmatrix
 constexpr int SA_WARPS = 4;
 
-// Causal self-attention of one (sample, head) per warp on the tensor cores
-// (mma.sync m16n8k16, bf16 in, fp32 accumulate): S = Q K^T over the H action
-// tokens, masked softmax on the accumulators, O = P V with P taken straight
-// from the score registers.
-template <int MT>   // H = 16 MT
-__global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p) {
-  constexpr int H = 16 * MT, NKT = H / 8;
+// Attention of one (sample, head) per warp on the tensor cores (mma.sync
+// m16n8k16, bf16 in, fp32 accumulate): S = Q K^T, masked softmax on the
+// accumulators, O = P V with P taken straight from the score registers.
+//   self  (CROSS = false): causal over the H action tokens; q, k, v are the
+//         sample's rows of the fused projection [rows][3E];
+//   cross (CROSS = true):  over the 1 + n_obs memory tokens (padded to 16 with
+//         masked keys); q [rows][E], keys/values of the memory tokens (the
+//         timestep token of step t and the sample's observation tokens, fp32,
+//         rounded to bf16 here).
+template <int MT, bool CROSS>   // H = 16 MT
+__global__ void __launch_bounds__(SA_WARPS * 32) attn_mma_kernel(const AttnArgs p) {
+  constexpr int H = 16 * MT, NK = CROSS ? 16 : H, NKT = NK / 8;
   const int s = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y * SA_WARPS + warp;
   if (!lat_refresh(p.lat, s, p.b, p.t)) return;
   extern __shared__ __align__(16) uint8_t sa_smem[];
-  __nv_bfloat16* sq = reinterpret_cast<__nv_bfloat16*>(sa_smem) + warp * 3 * H * SA_LDS;
+  __nv_bfloat16* sq = reinterpret_cast<__nv_bfloat16*>(sa_smem) + warp * (H + 2 * NK) * SA_LDS;
   __nv_bfloat16* sk = sq + H * SA_LDS;
-  __nv_bfloat16* sv = sk + H * SA_LDS;
+  __nv_bfloat16* sv = sk + NK * SA_LDS;
   if (h >= p.nh) return;
   const int E = p.E;
-  const __nv_bfloat16* base = p.qkv + (long long)s * H * 3 * E + h * SA_DH;
-  for (int c = lane; c < H * 24; c += 32) {          // per token: q, k, v rows of 8 x 16 bytes
-    const int i = c / 24, rem = c - i * 24, which = rem >> 3, ch = rem & 7;
-    cp_async16(sq + which * H * SA_LDS + i * SA_LDS + ch * 8, base + (long long)i * 3 * E + which * E + ch * 8);
+  if constexpr (!CROSS) {
+    const __nv_bfloat16* base = p.qkv + (long long)s * H * 3 * E + h * SA_DH;
+    for (int c = lane; c < H * 24; c += 32) {          // per token: q, k, v rows of 8 x 16 bytes
+      const int i = c / 24, rem = c - i * 24, which = rem >> 3, ch = rem & 7;
+      cp_async16(sq + which * H * SA_LDS + i * SA_LDS + ch * 8, base + (long long)i * 3 * E + which * E + ch * 8);
+    }
+  } else {
+    const __nv_bfloat16* base = p.qkv + (long long)s * H * E + h * SA_DH;
+    for (int c = lane; c < H * 8; c += 32) {
+      const int i = c >> 3, ch = c & 7;
+      cp_async16(sq + i * SA_LDS + ch * 8, base + (long long)i * E + ch * 8);
+    }
+    const int Cm = 1 + p.n_obs;
+    for (int c = lane; c < NK * SA_DH / 2; c += 32) {   // pairs of head dims of every (padded) key
+      const int j = c / (SA_DH / 2), d = 2 * (c % (SA_DH / 2));
+      float2 kk = make_float2(0.f, 0.f), vv = make_float2(0.f, 0.f);
+      if (j < Cm) {
+        const float* src = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
+                                  : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
+        kk = *reinterpret_cast<const float2*>(src + h * SA_DH + d);
+        vv = *reinterpret_cast<const float2*>(src + E + h * SA_DH + d);
+      }
+      *reinterpret_cast<__nv_bfloat162*>(sk + j * SA_LDS + d) = __floats2bfloat162_rn(kk.x, kk.y);
+      *reinterpret_cast<__nv_bfloat162*>(sv + j * SA_LDS + d) = __floats2bfloat162_rn(vv.x, vv.y);
+    }
   }
   cp_async_wait_all();
   __syncwarp();
@@ -460,7 +485,8 @@ __global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p
       }
     }
   }
-  // causal mask, softmax over keys (rows g and g + 8 of each m-tile)
+  // mask, softmax over keys (rows g and g + 8 of each m-tile)
+  const int nkeys = CROSS ? 1 + p.n_obs : H;
   float inv[MT][2];
 #pragma unroll
   for (int m = 0; m < MT; ++m) {
@@ -470,7 +496,8 @@ __global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int row = m * 16 + g + (e >> 1) * 8, col = n * 8 + 2 * tq + (e & 1);
-        const float v = col <= row ? sc[m][n][e] * p.scale : -INFINITY;
+        const bool keep = CROSS ? col < nkeys : col <= row;
+        const float v = keep ? sc[m][n][e] * p.scale : -INFINITY;
         sc[m][n][e] = v;
         mx[e >> 1] = fmaxf(mx[e >> 1], v);
       }
@@ -502,7 +529,7 @@ __global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p
 #pragma unroll
     for (int n = 0; n < SA_DH / 8; ++n) o[m][n][0] = o[m][n][1] = o[m][n][2] = o[m][n][3] = 0.f;
 #pragma unroll
-  for (int kk = 0; kk < H / 16; ++kk) {
+  for (int kk = 0; kk < NK / 16; ++kk) {
     uint32_t a[MT][4];
 #pragma unroll
     for (int m = 0; m < MT; ++m) {
@@ -534,80 +561,15 @@ __global__ void __launch_bounds__(SA_WARPS * 32) sa_attn_kernel(const AttnArgs p
     }
 }
 
-// Cross-attention to the 1 + n_obs memory tokens: a block per sample with
-// every head's memory keys/values staged in shared memory, a warp per head, a
-// lane per action token (row).
-template <int DH>
-__global__ void __launch_bounds__(256) ca_attn_kernel(const AttnArgs p) {
-  const int s = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (!lat_refresh(p.lat, s, p.b, p.t)) return;
-  extern __shared__ __align__(16) float kv[];      // [Cm][2E]
-  const int E = p.E, Cm = 1 + p.n_obs;
-  for (int v = threadIdx.x; v < Cm * E / 2; v += blockDim.x) {
-    const int j = v / (E / 2), c = v - j * (E / 2);
-    const float* src = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
-                              : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
-    reinterpret_cast<float4*>(kv + j * 2 * E)[c] = reinterpret_cast<const float4*>(src)[c];
-  }
-  __syncthreads();
-  const int H = p.lat.H;
-  if (warp >= p.nh || lane >= H) return;
-  const int h = warp, row = s * H + lane;
-  float q[DH];
-  const uint4* qr = reinterpret_cast<const uint4*>(p.qkv + (long long)row * E + h * DH);
-#pragma unroll
-  for (int c = 0; c < DH / 8; ++c) {
-    const uint4 raw = qr[c];
-    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
-      q[8 * c + 2 * i] = f.x;
-      q[8 * c + 2 * i + 1] = f.y;
-    }
-  }
-  constexpr int MAXC = 8;
-  float sc[MAXC];
-  float mx = -INFINITY;
-#pragma unroll
-  for (int j = 0; j < MAXC; ++j) {
-    sc[j] = -INFINITY;
-    if (j < Cm) {
-      const float* kr = kv + j * 2 * E + h * DH;
-      float d0 = 0.f, d1 = 0.f;
-#pragma unroll
-      for (int d = 0; d < DH; d += 2) {
-        d0 = fmaf(q[d], kr[d], d0);
-        d1 = fmaf(q[d + 1], kr[d + 1], d1);
-      }
-      sc[j] = (d0 + d1) * p.scale;
-      mx = fmaxf(mx, sc[j]);
-    }
-  }
-  float sum = 0.f;
-#pragma unroll
-  for (int j = 0; j < MAXC; ++j) {
-    sc[j] = j < Cm ? __expf(sc[j] - mx) : 0.f;
-    sum += sc[j];
-  }
-  const float inv = 1.f / sum;
-#pragma unroll
-  for (int d = 0; d < DH; ++d) q[d] = 0.f;
-#pragma unroll
-  for (int j = 0; j < MAXC; ++j) {
-    if (j < Cm) {
-      const float* vr = kv + j * 2 * E + E + h * DH;
-      const float w = sc[j] * inv;
-#pragma unroll
-      for (int d = 0; d < DH; ++d) q[d] = fmaf(w, vr[d], q[d]);
-    }
-  }
-  uint4* o = reinterpret_cast<uint4*>(p.att + (long long)row * E + h * DH);
-#pragma unroll
-  for (int c = 0; c < DH / 8; ++c) o[c] = pack_bf16x8(q + 8 * c);
+size_t attn_smem_bytes(int H, bool cross) {
+  return (size_t)SA_WARPS * (H + 2 * (cross ? 16 : H)) * SA_LDS * sizeof(__nv_bfloat16);
 }
 
-size_t sa_smem_bytes(int H) { return (size_t)SA_WARPS * 3 * H * SA_LDS * sizeof(__nv_bfloat16); }
+template <int MT, bool CROSS>
+cudaError_t attn_attr() {
+  return cudaFuncSetAttribute(attn_mma_kernel<MT, CROSS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)attn_smem_bytes(16 * MT, CROSS));
+}
 
 }  // namespace
 
@@ -631,6 +593,7 @@ struct WideState {
   __nv_bfloat16* hid = nullptr;     // [rmax][4E]
   __nv_bfloat16* cache = nullptr;   // [U][rmax][E]
   float* a = nullptr;               // [rmax][E]
+  float* head_wt = nullptr;         // [A][E]
   int* first = nullptr;             // [max_sched][U]
   CUtensorMap mA_xln, mA_att, mA_hid;
   BMaps mB_e, mB_4e;
@@ -751,6 +714,15 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     if (cudaMemcpy(w->wt_4e, t4.data(), t4.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(EVO_ERR_CUDA);
   }
+  {
+    std::vector<float> ht((size_t)w->A * E);
+    const float* hw = weights + woff[W_HEAD_W];
+    for (int e = 0; e < E; ++e)
+      for (int a = 0; a < w->A; ++a) ht[(size_t)a * E + e] = hw[(size_t)e * w->A + a];
+    if (cudaMalloc(&w->head_wt, ht.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMemcpy(w->head_wt, ht.data(), ht.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(EVO_ERR_CUDA);
+  }
   if (cudaMalloc(&w->xln, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMalloc(&w->qkv, R * 3 * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMalloc(&w->att, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
@@ -779,10 +751,8 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
         cudaDeviceGetAttribute(&w->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || w->num_sms <= 0)
       return fail(EVO_ERR_CUDA);
   }
-  if (cudaFuncSetAttribute(sa_attn_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(16)) !=
-          cudaSuccess ||
-      cudaFuncSetAttribute(sa_attn_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sa_smem_bytes(32)) !=
-          cudaSuccess)
+  if (attn_attr<1, false>() != cudaSuccess || attn_attr<2, false>() != cudaSuccess ||
+      attn_attr<1, true>() != cudaSuccess || attn_attr<2, true>() != cudaSuccess)
     return fail(EVO_ERR_CUDA);
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(EVO_ERR_CUDA);
   *out = w;
@@ -800,6 +770,7 @@ void wide_destroy(WideState* w) {
   cudaFree(w->cache);
   cudaFree(w->a);
   cudaFree(w->first);
+  cudaFree(w->head_wt);
   delete w;
 }
 
@@ -860,7 +831,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   rp.sampler = w->sampler;
   rp.lnf_g = w->wf32 + w->woff[W_LNF_G];
   rp.lnf_b = w->wf32 + w->woff[W_LNF_B];
-  rp.head_w = w->wf32 + w->woff[W_HEAD_W];
+  rp.head_wt = w->head_wt;
   rp.head_b = w->wf32 + w->woff[W_HEAD_B];
   rp.in_w = w->wf32 + w->woff[W_IN_W];
   rp.in_b = w->wf32 + w->woff[W_IN_B];
@@ -893,8 +864,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   ap.kv_time = c.kv_time;
   ap.kv_obs = c.kv_obs;
   ap.scale = 1.f / std::sqrt((float)w->dh);
-  const size_t sa_smem = sa_smem_bytes(H);
-  const size_t ca_smem = (size_t)(1 + w->n_obs) * 2 * E * sizeof(float);
+  const size_t sa_smem = attn_smem_bytes(H, false), ca_smem = attn_smem_bytes(H, true);
+  const dim3 attn_grid(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS);
 
   for (int t = 0; t < T; ++t) {
     int lo = 0;
@@ -924,8 +895,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.ldo = 3 * E;
         WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, st));
         ap.qkv = w->qkv;
-        if (H == 32) sa_attn_kernel<2><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
-        else sa_attn_kernel<1><<<dim3(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS), SA_WARPS * 32, sa_smem, st>>>(ap);
+        if (H == 32) attn_mma_kernel<2, false><<<attn_grid, SA_WARPS * 32, sa_smem, st>>>(ap);
+        else attn_mma_kernel<1, false><<<attn_grid, SA_WARPS * 32, sa_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 3 * E;
         g.bias = wl(w, l, WL_SA_BO);
@@ -938,7 +909,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.ldo = E;
         WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, st));
         ap.qkv = w->qkv;
-        ca_attn_kernel<64><<<c.samples, 32 * w->nh, ca_smem, st>>>(ap);
+        if (H == 32) attn_mma_kernel<2, true><<<attn_grid, SA_WARPS * 32, ca_smem, st>>>(ap);
+        else attn_mma_kernel<1, true><<<attn_grid, SA_WARPS * 32, ca_smem, st>>>(ap);
         WCK(cudaGetLastError());
         g.b_row0 = rowE + 5 * E;
         g.bias = wl(w, l, WL_CA_BO);
