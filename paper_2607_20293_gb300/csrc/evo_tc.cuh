@@ -124,6 +124,12 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
+// Programmatic dependent launch: let the next kernel of the stream start its
+// launch now; wait until the previous kernel has finished and its writes are
+// visible (a no-op for kernels launched without the attribute).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -277,6 +283,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();                              // A, the residual stream and the lattice come from earlier kernels
   const uint32_t tmem = *tslot;
   const int KB = g.K / BK, total = m_tiles * n_tiles;
 
@@ -346,6 +353,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
     }
   }
   __syncwarp();
+  pdl_trigger();                           // the next kernel may launch while this one drains
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);

@@ -95,6 +95,8 @@ __device__ __forceinline__ bool lat_valid(const Lat& L, int sample, int b, int t
 }
 
 __global__ void first_kernel(Lat L, int n_sched, int* first) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
   const int s = blockIdx.x;
   for (int b = threadIdx.x; b < L.U; b += blockDim.x) {
     int f = L.T;
@@ -259,6 +261,8 @@ __device__ __forceinline__ void layer_norm(RowV<NV>& r, const float* g, const fl
 
 template <int NV>
 __global__ void __launch_bounds__(256) prep_kernel(const RowArgs p) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.rows) return;
   const int sample = row / p.lat.H;
@@ -304,6 +308,8 @@ __device__ __forceinline__ void embed_row(const RowArgs& p, int row, int lane, f
 
 template <int NV>
 __global__ void __launch_bounds__(256) init_kernel(const RowArgs p) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.rows) return;
   const int H = p.lat.H, sample = row / H, tok = row % H;
@@ -319,6 +325,8 @@ constexpr int MAXA = 16;
 
 template <int NV>
 __global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.rows) return;
   const int H = p.lat.H, sample = row / H, tok = row % H, t = p.t, A = p.A;
@@ -421,6 +429,8 @@ constexpr int SA_WARPS = 4;
 //         rounded to bf16 here).
 template <int MT, bool CROSS>   // H = 16 MT
 __global__ void __launch_bounds__(SA_WARPS * 32) attn_mma_kernel(const AttnArgs p) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
   constexpr int H = 16 * MT, NK = CROSS ? 16 : H, NKT = NK / 8;
   const int s = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y * SA_WARPS + warp;
@@ -608,20 +618,40 @@ const float* wl(const WideState* w, int l, int id) {
   return w->wf32 + w->woff[W_LAYER0] + (long long)l * w->woff[W_LAYER_STRIDE] + w->woff[id];
 }
 
+constexpr long long PDL_MAX_ROWS = 32768;
+
+// Launch with programmatic stream serialization: the kernel may begin while
+// its predecessor finishes (every kernel of this path waits for it with
+// griddepcontrol.wait before touching global data).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(bool pdl, void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
 template <int MODE>
 cudaError_t gemm(const CUtensorMap& ma, const BMaps& mb, const tc::GemmArgs& g, int rows_p, int N, int num_sms,
-                 cudaStream_t st) {
+                 bool pdl, cudaStream_t st) {
   const int m_tiles = rows_p / tc::BM;
   if (N % 256 == 0 && m_tiles * (N / 256) >= num_sms) {
     const int total = m_tiles * (N / 256);
-    tc::gemm_kernel<MODE, 256><<<std::min(total, num_sms), tc::NTHREADS_GEMM, tc::TileCfg<256>::SMEM_BYTES, st>>>(
-        ma, mb.n256, g, m_tiles, N / 256);
+    return launch_pdl(pdl, tc::gemm_kernel<MODE, 256>, dim3(std::min(total, num_sms)), dim3(tc::NTHREADS_GEMM),
+                      tc::TileCfg<256>::SMEM_BYTES, st, ma, mb.n256, g, m_tiles, N / 256);
   } else {
     const int total = m_tiles * (N / 128);
-    tc::gemm_kernel<MODE, 128><<<std::min(total, num_sms), tc::NTHREADS_GEMM, tc::TileCfg<128>::SMEM_BYTES, st>>>(
-        ma, mb.n128, g, m_tiles, N / 128);
+    return launch_pdl(pdl, tc::gemm_kernel<MODE, 128>, dim3(std::min(total, num_sms)), dim3(tc::NTHREADS_GEMM),
+                      tc::TileCfg<128>::SMEM_BYTES, st, ma, mb.n128, g, m_tiles, N / 128);
   }
-  return cudaGetLastError();
 }
 
 template <int MODE, int BN>
@@ -631,18 +661,17 @@ cudaError_t gemm_attr() {
 }
 
 template <int NV>
-cudaError_t launch_rows(int which, const RowArgs& p, cudaStream_t st) {
+cudaError_t launch_rows(int which, const RowArgs& p, bool pdl, cudaStream_t st) {
   const int blocks = (p.rows + 7) / 8;
-  if (which == 0) init_kernel<NV><<<blocks, 256, 0, st>>>(p);
-  else if (which == 1) prep_kernel<NV><<<blocks, 256, 0, st>>>(p);
-  else head_kernel<NV><<<blocks, 256, 0, st>>>(p);
-  return cudaGetLastError();
+  if (which == 0) return launch_pdl(pdl, init_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
+  if (which == 1) return launch_pdl(pdl, prep_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
+  return launch_pdl(pdl, head_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
 }
 
-cudaError_t rows_kernel(int which, const RowArgs& p, cudaStream_t st) {
+cudaError_t rows_kernel(int which, const RowArgs& p, bool pdl, cudaStream_t st) {
   switch (p.E / 256) {
-    case 1: return launch_rows<1>(which, p, st);
-    case 2: return launch_rows<2>(which, p, st);
+    case 1: return launch_rows<1>(which, p, pdl, st);
+    case 2: return launch_rows<2>(which, p, pdl, st);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -783,6 +812,9 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   if (R > w->rmax || c.n_sched > w->max_sched) return cudaErrorInvalidValue;
   const int Rp = (int)((R + tc::BM - 1) / tc::BM * tc::BM);
   cudaStream_t st = c.st;
+  // programmatic dependent launch hides the kernel-to-kernel gap where the
+  // kernels are short; on the largest batches it measured slower, so it is off
+  const bool pdl = R < PDL_MAX_ROWS;
   long long n = 0;
   cudaError_t e;
 #define WCK(x)                    \
@@ -812,8 +844,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   lat.H = H;
   lat.per_sched = c.per_sched;
   lat.force = w->force;
-  first_kernel<<<c.n_sched, 64, 0, st>>>(lat, c.n_sched, w->first);
-  WCK(cudaGetLastError());
+  WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first));
 
   RowArgs rp{};
   rp.lat = lat;
@@ -836,7 +867,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   rp.in_w = w->wf32 + w->woff[W_IN_W];
   rp.in_b = w->wf32 + w->woff[W_IN_B];
   rp.pos = w->wf32 + w->woff[W_POS];
-  WCK(rows_kernel(0, rp, st));
+  WCK(rows_kernel(0, rp, pdl, st));
 
   tc::GemmArgs g{};
   g.rows = (int)R;
@@ -880,7 +911,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
       rp.b = b;
       rp.gamma = wl(w, l, ln_g[u]);
       rp.beta = wl(w, l, ln_b[u]);
-      WCK(rows_kernel(1, rp, st));
+      WCK(rows_kernel(1, rp, pdl, st));
       lo = b;
       g.srow = c.S_rows == U ? b : b / 3;
       g.cache = w->cache + (long long)b * w->rmax * E;
@@ -893,44 +924,42 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
         g.bias = wl(w, l, WL_SA_BQKV);
         g.out = w->qkv;
         g.ldo = 3 * E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, st));
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, pdl, st));
         ap.qkv = w->qkv;
-        if (H == 32) attn_mma_kernel<2, false><<<attn_grid, SA_WARPS * 32, sa_smem, st>>>(ap);
-        else attn_mma_kernel<1, false><<<attn_grid, SA_WARPS * 32, sa_smem, st>>>(ap);
-        WCK(cudaGetLastError());
+        WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, false> : attn_mma_kernel<1, false>, attn_grid,
+                       dim3(SA_WARPS * 32), sa_smem, st, ap));
         g.b_row0 = rowE + 3 * E;
         g.bias = wl(w, l, WL_SA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
       } else if (u == 1) {
         g.K = E;
         g.b_row0 = rowE + 4 * E;
         g.bias = wl(w, l, WL_CA_BQ);
         g.out = w->qkv;
         g.ldo = E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, st));
+        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
         ap.qkv = w->qkv;
-        if (H == 32) attn_mma_kernel<2, true><<<attn_grid, SA_WARPS * 32, ca_smem, st>>>(ap);
-        else attn_mma_kernel<1, true><<<attn_grid, SA_WARPS * 32, ca_smem, st>>>(ap);
-        WCK(cudaGetLastError());
+        WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, true> : attn_mma_kernel<1, true>, attn_grid,
+                       dim3(SA_WARPS * 32), ca_smem, st, ap));
         g.b_row0 = rowE + 5 * E;
         g.bias = wl(w, l, WL_CA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
       } else {
         g.K = E;
         g.b_row0 = rowE + 6 * E;
         g.bias = wl(w, l, WL_FF_B1);
         g.out = w->hid;
         g.ldo = 4 * E;
-        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, st));
+        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, pdl, st));
         g.K = 4 * E;
         g.b_row0 = l * E;
         g.bias = wl(w, l, WL_FF_B2);
-        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, st));
+        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, pdl, st));
       }
     }
     rp.lo = lo;
     rp.b = U;
-    WCK(rows_kernel(2, rp, st));
+    WCK(rows_kernel(2, rp, pdl, st));
   }
 #undef WCK
   w->launches = n;
