@@ -193,6 +193,11 @@ evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* j
  * tensor-core GEMMs); kernels = kernel launches of that call. */
 evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels);
 
+/* The cudaError_t of the most recent CUDA runtime failure behind an
+ * EVO_ERR_CUDA on the calling thread (0 if none): the detail a caller needs to
+ * tell, for instance, a launch-configuration error from a device fault. */
+int32_t evo_last_cuda_error(void);
+
 const char* evo_status_string(evo_status s);
 
 #ifdef __cplusplus

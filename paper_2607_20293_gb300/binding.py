@@ -31,7 +31,10 @@ class EvoConfig(ctypes.Structure):
 class EvoError(RuntimeError):
     def __init__(self, code: int, what: str):
         self.code = code
-        super().__init__(f"{what}: {status_string(code)} ({code})")
+        detail = ""
+        if code == ERR_CUDA and _lib is not None:
+            detail = f", CUDA error {_lib.evo_last_cuda_error()}"
+        super().__init__(f"{what}: {status_string(code)} ({code}{detail})")
 
 
 _lib = None
@@ -62,6 +65,7 @@ def load() -> ctypes.CDLL:
         "evo_get_launch_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(I32),
                                       ctypes.POINTER(I32)]),
         "evo_get_last_call": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I64)]),
+        "evo_last_cuda_error": (I32, []),
         "evo_status_string": (ctypes.c_char_p, [I32]),
     }
     for name, (res, args) in sig.items():

@@ -67,10 +67,16 @@ struct evo_handle {
 
 namespace {
 
+// CUDA runtime error of the most recent failed call on this thread
+thread_local int g_last_cuda_error = 0;
+
 #define EVO_CUDA(x)                                   \
   do {                                                \
     cudaError_t _e = (x);                             \
-    if (_e != cudaSuccess) return EVO_ERR_CUDA;       \
+    if (_e != cudaSuccess) {                          \
+      g_last_cuda_error = (int)_e;                    \
+      return EVO_ERR_CUDA;                            \
+    }                                                 \
   } while (0)
 
 bool config_ok(const evo_config* c) {
@@ -276,6 +282,7 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   p.invE = 1.0f / (float)E;
   if (p.Cm > 32 || p.M * p.Ec > 4 * NCT) return -1;
   if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
+  if (es == 2 && p.Cm > 16) return -1;                      // tensor-core attention pads memory keys to 16
   if (es == 2) {
     if (p.Mp > 32) return -1;
   } else {
@@ -667,7 +674,7 @@ cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, int 
 
 evo_status finish(evo_handle* h, cudaStream_t st) {
   h->last_stream = st;
-  if (cudaGetLastError() != cudaSuccess) return EVO_ERR_CUDA;
+  EVO_CUDA(cudaGetLastError());
   if (h->cfg.debug_sync) return evo_get_status(h);
   return EVO_OK;
 }
@@ -910,6 +917,8 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
   h->prof_stop = reinterpret_cast<cudaEvent_t>(stop);
   return EVO_OK;
 }
+
+int32_t evo_last_cuda_error(void) { return g_last_cuda_error; }
 
 evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels) {
   if (!h) return EVO_ERR_ARG;

@@ -48,6 +48,7 @@
 #pragma once
 
 #include "evo_ptx.cuh"
+#include "evo_shapes.h"
 
 namespace evo {
 
@@ -84,7 +85,6 @@ struct Shape {
   __host__ __device__ static constexpr int pNs(int u, int q) {
     return pK(u, q) / 16 <= pK0(u, q) ? 1 : 1 + (pK(u, q) / 16 - pK0(u, q) + pKps(u, q) - 1) / pKps(u, q);
   }
-  static_assert((NSLOT & (NSLOT - 1)) == 0, "ring slots: a power of two");
   static_assert((Ec & (Ec - 1)) == 0 && (H & (H - 1)) == 0, "Ec and H: powers of two");
   static_assert(M * Ec <= 4 * NCT, "at most four residual columns per thread");
   // slab 0 of a piece holds its header and at least one k-tile
@@ -99,11 +99,21 @@ struct Loop {
   static constexpr int MEc = M * Ec;
   static constexpr int EPT = (MEc + NCT - 1) / NCT;          // residual elements per thread (1..4)
   static constexpr uint32_t XBYTES = (uint32_t)(M * E * 4);    // bytes one exchange delivers to a CTA
+  // bf16 attention on the tensor cores: q, k, v of each sample staged as bf16
+  // tiles (rows of LQ / LV elements) in the first GEMM's output region
+  static constexpr bool MMA_ATT = BF && H % 16 == 0 && dh % 32 == 0 && Ec % 16 == 0;
+  static constexpr int LQ = dh + 8, LV = Ec + 8;
+  template <int U>
+  __host__ __device__ static constexpr int att_keys() { return U == 0 ? H : 16; }
+  template <int U>
+  __host__ __device__ static constexpr int att_sample_elems() { return (H + att_keys<U>()) * LQ + att_keys<U>() * LV; }
+  static_assert(!MMA_ATT || S::G * att_sample_elems<0>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
+  static_assert(!MMA_ATT || S::G * att_sample_elems<1>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
 
   // ---------------------------------------------------------------- rings and barriers
   // wait for the oldest unreleased slab (cx.q)
   __device__ __forceinline__ static const uint8_t* ring_acquire(const JobParams& p, Ctx& cx) {
-    const uint32_t slot = cx.q & (S::NSLOT - 1);
+    const uint32_t slot = cx.q % S::NSLOT;
     const uint32_t ph = (cx.q / S::NSLOT) & 1u;
     wait_parity(smem_u32(&cx.full[slot]), ph, false, cx, p.status);
     return cx.smem + p.sm.ring + slot * S::SLOT;
@@ -111,7 +121,7 @@ struct Loop {
 
   __device__ __forceinline__ static void ring_release(Ctx& cx) {
     __syncwarp();
-    if (cx.lane == 0) mbar_arrive(&cx.empty[cx.q & (S::NSLOT - 1)]);
+    if (cx.lane == 0) mbar_arrive(&cx.empty[cx.q % S::NSLOT]);
     cx.q++;
   }
 
@@ -169,7 +179,7 @@ struct Loop {
               const int cnt = s == 0 ? k0 : min(kps, nkt - kt0);
               const uint32_t off = s == 0 ? 0u : (uint32_t)(hdr + kt0 * ktb);
               const uint32_t bytes = (uint32_t)((s == 0 ? hdr : 0) + cnt * ktb);
-              const uint32_t slot = q & (S::NSLOT - 1);
+              const uint32_t slot = q % S::NSLOT;
               const uint32_t ph = (q / S::NSLOT) & 1u;
               if (!mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
                 // the producer runs ahead of the compute warps: poll gently
@@ -193,7 +203,7 @@ struct Loop {
     // drain: every slab issued has landed before this CTA may exit (bounded waits)
     const uint32_t first = q > (uint32_t)S::NSLOT ? q - S::NSLOT : 0u;
     for (uint32_t k = first; k < q; ++k)
-      wait_parity(smem_u32(&cx.full[k & (S::NSLOT - 1)]), (k / S::NSLOT) & 1u, false, cx, p.status);
+      wait_parity(smem_u32(&cx.full[k % S::NSLOT]), (k / S::NSLOT) & 1u, false, cx, p.status);
   }
 
   // ---------------------------------------------------------------- GEMMs over streamed slabs
@@ -370,6 +380,15 @@ struct Loop {
                 if constexpr (U == 2) {
                   *reinterpret_cast<__nv_bfloat162*>(hid + m * S::ldh + n) =
                       __floats2bfloat162_rn(gelu_erf(v0), gelu_erf(v1));
+                } else if constexpr (MMA_ATT) {
+                  // q -> Q[i], k -> K[i], v -> V[i] of sample m / H
+                  __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) +
+                                      (m >> S::lH) * att_sample_elems<U>();
+                  const int i = m & (H - 1);
+                  __nv_bfloat16* dst = n < dh       ? st + i * LQ + n
+                                       : n < 2 * dh ? st + (H + i) * LQ + (n - dh)
+                                                    : st + (H + att_keys<U>()) * LQ + i * LV + (n - 2 * dh);
+                  *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(v0, v1);
                 } else {
                   *reinterpret_cast<float2*>(g1 + m * S::ldg1 + n) = make_float2(v0, v1);
                 }
@@ -454,8 +473,145 @@ struct Loop {
   // one output (row, dim of this CTA's slice) per thread.  SA: causal over the
   // H tokens of the same sample (q, k of the CTA's head and v of its slice are
   // rows of the first GEMM's output).  CA: the 1 + n_obs memory tokens in kvs.
+  // Tensor-core attention (bf16): warp s < G takes sample s.  S = Q K^T
+  // (mma.sync m16n8k16), causal (SA) or key-count (CA, memory tokens padded
+  // to 16) mask and softmax on the accumulators, O = P V with P taken from
+  // the score registers; O goes to the second GEMM's A operand.
+  template <int U>
+  __device__ __forceinline__ static void attention_mma(const JobParams& p, Ctx& cx, const float* kvs) {
+    constexpr int NK = att_keys<U>(), NKT = NK / 8, MTH = H / 16;
+    if (cx.warp >= S::G) return;
+    const int sm_ = cx.warp, lane = cx.lane;
+    __nv_bfloat16* Q = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) + sm_ * att_sample_elems<U>();
+    __nv_bfloat16* K = Q + H * LQ;
+    __nv_bfloat16* V = K + NK * LQ;
+    if constexpr (U == 1) {
+      // memory keys / values of this sample (fp32 in kvs) -> bf16 tiles, padded keys zero
+      const float* kv = kvs + sm_ * p.Cm * S::kvw;
+      for (int c = lane; c < NK * (dh / 2); c += 32) {
+        const int j = c / (dh / 2), d = 2 * (c % (dh / 2));
+        const float2 f = j < p.Cm ? *reinterpret_cast<const float2*>(kv + j * S::kvw + d) : make_float2(0.f, 0.f);
+        *reinterpret_cast<__nv_bfloat162*>(K + j * LQ + d) = __floats2bfloat162_rn(f.x, f.y);
+      }
+      for (int c = lane; c < NK * (Ec / 2); c += 32) {
+        const int j = c / (Ec / 2), d = 2 * (c % (Ec / 2));
+        const float2 f = j < p.Cm ? *reinterpret_cast<const float2*>(kv + j * S::kvw + dh + d) : make_float2(0.f, 0.f);
+        *reinterpret_cast<__nv_bfloat162*>(V + j * LV + d) = __floats2bfloat162_rn(f.x, f.y);
+      }
+      __syncwarp();
+    }
+    const int g = lane >> 2, tq = lane & 3;
+    float sc[MTH][NKT][4];
+#pragma unroll
+    for (int m = 0; m < MTH; ++m)
+#pragma unroll
+      for (int n = 0; n < NKT; ++n) sc[m][n][0] = sc[m][n][1] = sc[m][n][2] = sc[m][n][3] = 0.f;
+#pragma unroll
+    for (int k2 = 0; k2 < dh / 32; ++k2) {
+      uint32_t a0[MTH][4], a1[MTH][4];
+#pragma unroll
+      for (int m = 0; m < MTH; ++m) {
+        const __nv_bfloat16* qa = Q + (m * 16 + (lane & 15)) * LQ + k2 * 32 + (lane >> 4) * 8;
+        ldmatrix_x4(a0[m], qa);
+        ldmatrix_x4(a1[m], qa + 16);
+      }
+#pragma unroll
+      for (int n = 0; n < NKT; ++n) {
+        uint32_t b[4];
+        ldmatrix_x4(b, K + (n * 8 + (lane & 7)) * LQ + k2 * 32 + (lane >> 3) * 8);
+#pragma unroll
+        for (int m = 0; m < MTH; ++m) {
+          mma_bf16(sc[m][n], a0[m], make_uint2(b[0], b[1]));
+          mma_bf16(sc[m][n], a1[m], make_uint2(b[2], b[3]));
+        }
+      }
+    }
+    const float scale = rsqrtf((float)dh);
+    const int nkeys = U == 0 ? H : p.Cm;
+    float inv[MTH][2];
+#pragma unroll
+    for (int m = 0; m < MTH; ++m) {
+      float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+      for (int n = 0; n < NKT; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int row = m * 16 + g + (e >> 1) * 8, col = n * 8 + 2 * tq + (e & 1);
+          const bool keep = U == 0 ? col <= row : col < nkeys;
+          const float v = keep ? sc[m][n][e] * scale : -INFINITY;
+          sc[m][n][e] = v;
+          mx[e >> 1] = fmaxf(mx[e >> 1], v);
+        }
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        mx[hh] = fmaxf(mx[hh], __shfl_xor_sync(0xffffffffu, mx[hh], 1));
+        mx[hh] = fmaxf(mx[hh], __shfl_xor_sync(0xffffffffu, mx[hh], 2));
+      }
+      float sum[2] = {0.f, 0.f};
+#pragma unroll
+      for (int n = 0; n < NKT; ++n)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float v = sc[m][n][e] == -INFINITY ? 0.f : __expf(sc[m][n][e] - mx[e >> 1]);
+          sc[m][n][e] = v;
+          sum[e >> 1] += v;
+        }
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        sum[hh] += __shfl_xor_sync(0xffffffffu, sum[hh], 1);
+        sum[hh] += __shfl_xor_sync(0xffffffffu, sum[hh], 2);
+        inv[m][hh] = __frcp_rn(sum[hh]);
+      }
+    }
+    float o[MTH][Ec / 8][4];
+#pragma unroll
+    for (int m = 0; m < MTH; ++m)
+#pragma unroll
+      for (int n = 0; n < Ec / 8; ++n) o[m][n][0] = o[m][n][1] = o[m][n][2] = o[m][n][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < NK / 16; ++kk) {
+      uint32_t a[MTH][4];
+#pragma unroll
+      for (int m = 0; m < MTH; ++m) {
+        __nv_bfloat162 h0 = __floats2bfloat162_rn(sc[m][2 * kk][0], sc[m][2 * kk][1]);
+        __nv_bfloat162 h1 = __floats2bfloat162_rn(sc[m][2 * kk][2], sc[m][2 * kk][3]);
+        __nv_bfloat162 h2 = __floats2bfloat162_rn(sc[m][2 * kk + 1][0], sc[m][2 * kk + 1][1]);
+        __nv_bfloat162 h3 = __floats2bfloat162_rn(sc[m][2 * kk + 1][2], sc[m][2 * kk + 1][3]);
+        a[m][0] = *reinterpret_cast<uint32_t*>(&h0);
+        a[m][1] = *reinterpret_cast<uint32_t*>(&h1);
+        a[m][2] = *reinterpret_cast<uint32_t*>(&h2);
+        a[m][3] = *reinterpret_cast<uint32_t*>(&h3);
+      }
+#pragma unroll
+      for (int n2 = 0; n2 < Ec / 16; ++n2) {
+        uint32_t b[4];
+        ldmatrix_x4_trans(b, V + (kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * LV + n2 * 16 + (lane >> 4) * 8);
+#pragma unroll
+        for (int m = 0; m < MTH; ++m) {
+          mma_bf16(o[m][2 * n2], a[m], make_uint2(b[0], b[1]));
+          mma_bf16(o[m][2 * n2 + 1], a[m], make_uint2(b[2], b[3]));
+        }
+      }
+    }
+    T* oc = reinterpret_cast<T*>(cx.smem + p.sm.oc);
+#pragma unroll
+    for (int m = 0; m < MTH; ++m)
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        T* dst = oc + (sm_ * H + m * 16 + g + hh * 8) * S::ldo + 2 * tq;
+#pragma unroll
+        for (int n = 0; n < Ec / 8; ++n)
+          *reinterpret_cast<__nv_bfloat162*>(dst + n * 8) =
+              __floats2bfloat162_rn(o[m][n][2 * hh] * inv[m][hh], o[m][n][2 * hh + 1] * inv[m][hh]);
+      }
+  }
+
   template <int U>
   __device__ __forceinline__ static void attention(const JobParams& p, Ctx& cx, const float* kvs) {
+    if constexpr (MMA_ATT) {
+      attention_mma<U>(p, cx, kvs);
+      return;
+    }
     const float* g1 = reinterpret_cast<const float*>(cx.smem + p.sm.xln);
     float* pb = reinterpret_cast<float*>(cx.smem + p.sm.pb);
     T* oc = reinterpret_cast<T*>(cx.smem + p.sm.oc);
@@ -951,7 +1107,7 @@ cudaError_t shape_prepare(int smem_bytes, int* max_clusters) {
 
 template <typename T, class S>
 cudaError_t shape_launch(const JobParams& p, int n_clusters, cudaStream_t s) {
-  if (!shape_matches<T, S>(p)) return cudaErrorInvalidValue;
+  if (!shape_matches<T, S>(p)) return cudaErrorInvalidConfiguration;   // host plan and compiled shape disagree
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -966,5 +1122,9 @@ cudaError_t shape_launch(const JobParams& p, int n_clusters, cudaStream_t s) {
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, job_kernel<T, S>, p);
 }
+
+template <int ID>
+struct ShapeOf;
+EVO_SHAPES(EVO_SHAPE_SPEC)
 
 }  // namespace evo

@@ -5,8 +5,8 @@
 
 namespace evo {
 
-EVO_SHAPE_DEF(6, float, 64, 2, 8, 2, 1, 4, 32768, 4)
-EVO_SHAPE_DEF(7, float, 64, 2, 8, 4, 1, 4, 32768, 4)
-EVO_SHAPE_DEF(8, float, 64, 2, 8, 8, 1, 4, 32768, 4)
+EVO_SHAPE_DEF_ID(6)
+EVO_SHAPE_DEF_ID(7)
+EVO_SHAPE_DEF_ID(8)
 
 }  // namespace evo

@@ -5,7 +5,7 @@
 
 namespace evo {
 
-EVO_SHAPE_DEF(0, __nv_bfloat16, 256, 4, 16, 16, 1, 2, 32768, 4)
-EVO_SHAPE_DEF(1, __nv_bfloat16, 256, 4, 16, 16, 2, 2, 32768, 2)
+EVO_SHAPE_DEF_ID(0)
+EVO_SHAPE_DEF_ID(1)
 
 }  // namespace evo

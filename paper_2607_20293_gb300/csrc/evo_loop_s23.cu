@@ -5,7 +5,7 @@
 
 namespace evo {
 
-EVO_SHAPE_DEF(2, __nv_bfloat16, 256, 4, 16, 8, 1, 2, 32768, 4)
-EVO_SHAPE_DEF(3, __nv_bfloat16, 256, 4, 16, 4, 1, 2, 32768, 4)
+EVO_SHAPE_DEF_ID(2)
+EVO_SHAPE_DEF_ID(3)
 
 }  // namespace evo

@@ -5,7 +5,7 @@
 
 namespace evo {
 
-EVO_SHAPE_DEF(4, __nv_bfloat16, 512, 8, 32, 16, 1, 2, 16384, 2)
-EVO_SHAPE_DEF(5, __nv_bfloat16, 64, 2, 8, 4, 1, 2, 32768, 4)
+EVO_SHAPE_DEF_ID(4)
+EVO_SHAPE_DEF_ID(5)
 
 }  // namespace evo
