@@ -283,6 +283,7 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   if (p.Cm > 32 || p.M * p.Ec > 4 * NCT) return -1;
   if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
   if (es == 2 && p.Cm > 16) return -1;                      // tensor-core attention pads memory keys to 16
+  if (p.A > 16) return -1;                                  // action dimensions of the fused head
   if (es == 2) {
     if (p.Mp > 32) return -1;
   } else {
@@ -569,7 +570,8 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   std::memcpy(&vec[p.v_pos], W(W_POS), (size_t)H * E * 4);
   std::memcpy(&vec[p.v_lnfg], W(W_LNF_G), E * 4);
   std::memcpy(&vec[p.v_lnfb], W(W_LNF_B), E * 4);
-  std::memcpy(&vec[p.v_headw], W(W_HEAD_W), (size_t)E * A * 4);
+  for (int e = 0; e < E; ++e)   // W_head transposed: [A][E]
+    for (int a = 0; a < A; ++a) vec[p.v_headw + (size_t)a * E + e] = W(W_HEAD_W)[(size_t)e * A + a];
   std::memcpy(&vec[p.v_headb], W(W_HEAD_B), A * 4);
   if (cudaMalloc(&h->vec, vec.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMemcpy(h->vec, vec.data(), vec.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)

@@ -37,6 +37,7 @@ struct SmemLayout {
   int x;       // [M][A] f32: current sample x (replicated in every CTA of the cluster)
   int z;       // [M][A] f32: DDPM noise of the current step
   int sch;     // [T] u64: this job's lattice, bit b of word t = unit b refreshed at step t
+  int stb;     // [T][8] f32: sampler coefficients of every step
   int bars;    // mbarriers: full[nslot], empty[nslot], cluster, xg, xr, xh
   int total;
 };

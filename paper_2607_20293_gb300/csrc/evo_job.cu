@@ -193,6 +193,8 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   off += al(p.M * p.A * 4, 16);
   s.z = off;
   off += al(p.M * p.A * 4, 16);
+  s.stb = off;
+  off += al(p.T * 8 * 4, 16);
   s.sch = off;
   off += al(p.T * 8, 16);
   s.bars = off;

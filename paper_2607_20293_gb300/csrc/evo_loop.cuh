@@ -485,21 +485,6 @@ struct Loop {
     __nv_bfloat16* Q = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) + sm_ * att_sample_elems<U>();
     __nv_bfloat16* K = Q + H * LQ;
     __nv_bfloat16* V = K + NK * LQ;
-    if constexpr (U == 1) {
-      // memory keys / values of this sample (fp32 in kvs) -> bf16 tiles, padded keys zero
-      const float* kv = kvs + sm_ * p.Cm * S::kvw;
-      for (int c = lane; c < NK * (dh / 2); c += 32) {
-        const int j = c / (dh / 2), d = 2 * (c % (dh / 2));
-        const float2 f = j < p.Cm ? *reinterpret_cast<const float2*>(kv + j * S::kvw + d) : make_float2(0.f, 0.f);
-        *reinterpret_cast<__nv_bfloat162*>(K + j * LQ + d) = __floats2bfloat162_rn(f.x, f.y);
-      }
-      for (int c = lane; c < NK * (Ec / 2); c += 32) {
-        const int j = c / (Ec / 2), d = 2 * (c % (Ec / 2));
-        const float2 f = j < p.Cm ? *reinterpret_cast<const float2*>(kv + j * S::kvw + dh + d) : make_float2(0.f, 0.f);
-        *reinterpret_cast<__nv_bfloat162*>(V + j * LV + d) = __floats2bfloat162_rn(f.x, f.y);
-      }
-      __syncwarp();
-    }
     const int g = lane >> 2, tq = lane & 3;
     float sc[MTH][NKT][4];
 #pragma unroll
@@ -606,9 +591,31 @@ struct Loop {
       }
   }
 
+  // memory keys / values of every sample of the job (fp32 in kvs) -> the bf16
+  // K / V tiles of the cross-attention, padded keys zero; all compute threads
+  __device__ __forceinline__ static void stage_memory_kv(const JobParams& p, Ctx& cx, const float* kvs) {
+    constexpr int NK = att_keys<1>(), PK = NK * (dh / 2), PS = NK * ((dh + Ec) / 2);
+    for (int c = cx.tid; c < S::G * PS; c += NCT) {
+      const int s_ = c / PS, r = c - s_ * PS;
+      __nv_bfloat16* K = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) + s_ * att_sample_elems<1>() + H * LQ;
+      const float* kv = kvs + s_ * p.Cm * S::kvw;
+      const bool isk = r < PK;
+      const int j = isk ? r / (dh / 2) : (r - PK) / (Ec / 2);
+      const int d = isk ? 2 * (r % (dh / 2)) : 2 * ((r - PK) % (Ec / 2));
+      const float2 f =
+          j < p.Cm ? *reinterpret_cast<const float2*>(kv + j * S::kvw + (isk ? 0 : dh) + d) : make_float2(0.f, 0.f);
+      __nv_bfloat16* dst = isk ? K + j * LQ + d : K + NK * LQ + j * LV + d;
+      *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(f.x, f.y);
+    }
+  }
+
   template <int U>
   __device__ __forceinline__ static void attention(const JobParams& p, Ctx& cx, const float* kvs) {
     if constexpr (MMA_ATT) {
+      if constexpr (U == 1) {
+        stage_memory_kv(p, cx, kvs);
+        bar_compute();
+      }
       attention_mma<U>(p, cx, kvs);
       return;
     }
@@ -793,8 +800,7 @@ struct Loop {
   }
 
   // ---------------------------------------------------------------- output head + sampler step
-  __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t, const float4 tab0,
-                                                   const float4 tab1) {
+  __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t) {
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
     float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
     const float* z = reinterpret_cast<const float*>(cx.smem + p.sm.z);
@@ -827,6 +833,8 @@ struct Loop {
     }
     cp_async_wait_all();
     bar_compute();
+    const float4 tab0 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32);
+    const float4 tab1 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32 + 16);
     const float inv_sa = tab0.x, s1 = tab0.y, cx0 = tab0.z, cxt = tab0.w, sig = tab1.x;
     const float sab = tab1.y, sabp = tab1.z, s1p = tab1.w;
     constexpr int NV = E / 64;
@@ -855,21 +863,24 @@ struct Loop {
 #pragma unroll
         for (int j = 0; j < NV; ++j) {
           const int col = 4 * (hl + 16 * j);
-          v[j].x = (v[j].x - mean) * rstd * lnf_g[col] + lnf_b[col];
-          v[j].y = (v[j].y - mean) * rstd * lnf_g[col + 1] + lnf_b[col + 1];
-          v[j].z = (v[j].z - mean) * rstd * lnf_g[col + 2] + lnf_b[col + 2];
-          v[j].w = (v[j].w - mean) * rstd * lnf_g[col + 3] + lnf_b[col + 3];
+          const float4 g4 = *reinterpret_cast<const float4*>(lnf_g + col);
+          const float4 b4 = *reinterpret_cast<const float4*>(lnf_b + col);
+          v[j].x = (v[j].x - mean) * rstd * g4.x + b4.x;
+          v[j].y = (v[j].y - mean) * rstd * g4.y + b4.y;
+          v[j].z = (v[j].z - mean) * rstd * g4.z + b4.z;
+          v[j].w = (v[j].w - mean) * rstd * g4.w + b4.w;
         }
+        // one reduced dot per action dimension over rows of W_head^T (float4 loads)
         float eps = 0.f;
         for (int a = 0; a < p.A; ++a) {
           float part = 0.f;
 #pragma unroll
           for (int j = 0; j < NV; ++j) {
-            const float* w = hw + 4 * (hl + 16 * j) * p.A + a;
-            part = fmaf(v[j].x, w[0], part);
-            part = fmaf(v[j].y, w[p.A], part);
-            part = fmaf(v[j].z, w[2 * p.A], part);
-            part = fmaf(v[j].w, w[3 * p.A], part);
+            const float4 w = *reinterpret_cast<const float4*>(hw + a * E + 4 * (hl + 16 * j));
+            part = fmaf(v[j].x, w.x, part);
+            part = fmaf(v[j].y, w.y, part);
+            part = fmaf(v[j].z, w.z, part);
+            part = fmaf(v[j].w, w.w, part);
           }
           const float e = group_sum<16>(part);
           if (hl == a) eps = e + head_b[a];
@@ -927,8 +938,6 @@ struct Loop {
       for (int t = 0; t < p.T; ++t) {
         const uint64_t refresh = sch[t] | (p.force ? ~valid : 0ull);
         // sampler coefficients of this step (used at the head)
-        const float4 tab0 = *reinterpret_cast<const float4*>(p.stab + t * 8);
-        const float4 tab1 = *reinterpret_cast<const float4*>(p.stab + t * 8 + 4);
         // stage z_t (DDPM) and, when every layer has a slot, the memory keys/values
         // of this step's refreshed cross-attention units
         if (p.sampler == 0) {
@@ -970,7 +979,7 @@ struct Loop {
             b = b1;
           }
         }
-        head_step(p, cx, t, tab0, tab1);
+        head_step(p, cx, t);
       }
       // write the finished chunk
       if (cx.c == 0) {
@@ -1036,6 +1045,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   // zero the operand and exchange buffers once: padded rows and columns must read as 0
   for (int v = threadIdx.x; v < (p.sm.ac - p.sm.ablk) / 16; v += NTHREADS)
     reinterpret_cast<float4*>(smem + p.sm.ablk)[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+  // sampler coefficients of every step
+  for (int v = threadIdx.x; v < p.T * 8; v += NTHREADS) reinterpret_cast<float*>(smem + p.sm.stb)[v] = p.stab[v];
   // per-kernel constants: in_w[:, cols], in_b[cols], pos[:, cols], lnf_g, lnf_b, head_b, head_w
   {
     float* cst = reinterpret_cast<float*>(smem + p.sm.cst);
@@ -1056,7 +1067,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
     for (int v = threadIdx.x; v < p.A; v += NTHREADS) d[v] = p.vec[p.v_headb + v];
     d += (p.A + 3) & ~3;
     if (p.headw_smem)
-      for (int v = threadIdx.x; v < S::E * p.A; v += NTHREADS) d[v] = p.vec[p.v_headw + v];
+      for (int v = threadIdx.x; v < S::E * p.A; v += NTHREADS) d[v] = p.vec[p.v_headw + v];   // [A][E]
   }
   __syncthreads();
   hw_cluster_sync();
