@@ -368,3 +368,114 @@ def flops_closed_form(cfg: dict, S, policy: str = "zero") -> int:
             n += 1                           # first use computes the empty unit
         total += n * f[b % 3]
     return total
+
+
+# ---------------------------------------------------------------------------
+# Redundancy-aware initialisation (Sec. 3.3, Eq. 6 and Eq. 7)
+# ---------------------------------------------------------------------------
+#
+# Readings (the paper defines Eq. 6 with the cosine and names, without
+# defining them, MSE, L1 and Wasserstein-1 alternatives in its metric
+# ablation):
+# * a_{r,b,t} is the residual output of unit b at loop step t for sample r of
+#   the uncached (all-refresh) policy, flattened over its H x E entries.
+# * MSE / L1: the mean over the entries of (a - a')^2 / |a - a'|.
+# * Wasserstein-1: between the empirical distributions of the entries of a and
+#   a' (equal sample sizes), i.e. the mean of |sort(a) - sort(a')|.
+# * Cosine with a zero vector (undefined) counts as dissimilarity 1.
+# * "Normalising d into w" is w = d / max d.
+# * Eq. 7 draws K distinct positions.  For a result both implementations can
+#   reproduce exactly, the weights (eps + w)^gamma are taken in fixed point,
+#   q = floor((eps + w)^gamma * 2^40) with gamma a positive integer (repeated
+#   products in float64), and draw k picks, among the positions not yet drawn
+#   in index order, the first whose running sum of q exceeds rnd_k mod (sum of
+#   the remaining q): sequential sampling without replacement with
+#   probabilities proportional to q.
+
+METRICS = ("cosine", "mse", "l1", "w1")
+
+
+def pair_dissimilarity(x, y, metric: str) -> float:
+    """The term of Eq. 6 for two activations (cosine: 1 - cos; or a variant)."""
+    x = np.asarray(x, dtype=np.float64).ravel()
+    y = np.asarray(y, dtype=np.float64).ravel()
+    if metric == "cosine":
+        nx, ny = np.sqrt(np.dot(x, x)), np.sqrt(np.dot(y, y))
+        if nx == 0.0 or ny == 0.0:
+            return 1.0
+        return 1.0 - float(np.dot(x, y)) / (nx * ny)
+    if metric == "mse":
+        return float(np.mean((x - y) ** 2))
+    if metric == "l1":
+        return float(np.mean(np.abs(x - y)))
+    if metric == "w1":
+        return float(np.mean(np.abs(np.sort(x) - np.sort(y))))
+    raise ValueError(metric)
+
+
+def redundancy_map(acts, metric: str = "cosine"):
+    """Eq. 6: acts [R][B][T][...] (activations of R samples) -> d [B][T],
+    d_{b,t} = mean over r of 1/(T-1) sum_{t' != t} D(a_{r,b,t}, a_{r,b,t'})."""
+    acts = np.asarray(acts)
+    R, B, T = acts.shape[:3]
+    d = np.zeros((B, T))
+    for r in range(R):
+        for b in range(B):
+            for t in range(T):
+                s = 0.0
+                for t2 in range(T):
+                    if t2 != t:
+                        s += pair_dissimilarity(acts[r, b, t], acts[r, b, t2], metric)
+                d[b, t] += s / (T - 1)
+    return d / R
+
+
+def trace_activations(trace: dict, U: int, T: int):
+    """The denoise trace {(b, t): (refreshed, residual [N][H][E])} of an
+    all-refresh query -> activations [N][U][T][H][E]."""
+    first = trace[(0, 0)][1]
+    N = first.shape[0]
+    acts = np.zeros((N, U, T) + first.shape[1:])
+    for (b, t), (_, used) in trace.items():
+        acts[:, b, t] = used
+    return acts
+
+
+def guided_weights(d, eps: float, gamma: int):
+    """Eq. 7 numerators (eps + w)^gamma, w = d / max d, in fixed point (int64,
+    2^40 units); eps is taken at float32 precision (the API's argument type)."""
+    d = np.asarray(d, dtype=np.float64).ravel()
+    w = d / d.max()
+    e = np.float64(np.float32(eps))
+    q = np.empty(d.size, dtype=np.int64)
+    for i in range(d.size):
+        base = e + w[i]
+        v = base
+        for _ in range(gamma - 1):
+            v = v * base
+        q[i] = int(np.floor(v * 1099511627776.0))
+    return q
+
+
+def guided_sample(q, K: int, rnd):
+    """K distinct positions drawn sequentially without replacement with
+    probability proportional to q (Eq. 7); rnd [K] unsigned 64-bit integers.
+    Draw k: target = rnd_k mod (sum of q over positions not yet drawn); the
+    position drawn is the first, in index order, whose running sum of q over
+    the positions not yet drawn exceeds the target.  Returns the flat 0/1
+    lattice."""
+    q = np.asarray(q, dtype=np.int64)
+    out = np.zeros(q.size, dtype=np.uint8)
+    for k in range(K):
+        live = np.where(out == 0, q, 0)          # drawn positions add nothing to the running sum
+        run = np.cumsum(live)                     # exact: integers
+        target = int(rnd[k]) % int(run[-1])
+        out[int(np.searchsorted(run, target, side="right"))] = 1
+    return out
+
+
+def guided_schedules(d, K: int, eps: float, gamma: int, rnd):
+    """P lattices [P][B][T] by Eq. 7 from the map d [B][T]; rnd [P][K]."""
+    d = np.asarray(d)
+    q = guided_weights(d, eps, gamma)
+    return np.stack([guided_sample(q, K, rnd[p]).reshape(d.shape) for p in range(len(rnd))])

@@ -138,20 +138,13 @@ def dissimilarity_map(L: int, T: int, seed: int = 5) -> np.ndarray:
     return d
 
 
-def guided_population(d: np.ndarray, P: int, seed: int = 6, eps: float = 0.05, gamma: float = 2.0,
-                      rho: tuple[float, float] = (0.05, 0.60)) -> np.ndarray:
-    """P candidate lattices [P][L][T]: density ~ U[rho], cells drawn without
-    replacement with probability proportional to (eps + w)^gamma, w = d / max d
-    (guided sampling, Eq. 7)."""
+def guided_randoms(P: int, K: int, seed: int = 6) -> np.ndarray:
+    """Unsigned 64-bit random integers [P][K] for the draws of guided sampling."""
     rng = np.random.default_rng(seed)
-    L, T = d.shape
-    w = d / d.max()
-    p = (eps + w.ravel()) ** gamma
-    p = p / p.sum()
-    out = np.zeros((P, L, T), dtype=np.uint8)
-    for i in range(P):
-        k = max(1, int(round(rng.uniform(*rho) * L * T)))
-        idx = rng.choice(L * T, size=k, replace=False, p=p)
-        flat = out[i].reshape(-1)
-        flat[idx] = 1
-    return out
+    return rng.integers(0, np.iinfo(np.uint64).max, size=(P, K), dtype=np.uint64, endpoint=True)
+
+
+def population_budgets(P: int, cells: int, seed: int = 6, rho: tuple[float, float] = (0.05, 0.60)) -> np.ndarray:
+    """Refresh budgets K_p of P candidates: densities ~ U[rho] of the lattice's cells."""
+    rng = np.random.default_rng(seed)
+    return np.array([max(1, int(round(rng.uniform(*rho) * cells))) for _ in range(P)])

@@ -194,13 +194,23 @@ def test_scaleup(torch, B, n, frac):
     check(got[idx], oracle_subset(W, cfg, obs, noise, S, idx), TOL["bf16"], name)
 
 
+def population_lattices(P: int):
+    """P candidate lattices [P][8][100] drawn by Eq. 7 from the synthetic map
+    (the oracle's sampler), with budgets of 5-60 % of the cells."""
+    d = synth.dissimilarity_map(8, 100, 5)
+    Ks = synth.population_budgets(P, 800, 6)
+    rnd = synth.guided_randoms(P, int(Ks.max()), 7)
+    q = O.guided_weights(d, 0.05, 2)
+    return np.stack([O.guided_sample(q, int(Ks[p]), rnd[p]).reshape(8, 100) for p in range(P)])
+
+
 @pytest.mark.parametrize("path", ["wide", "cluster"])
 def test_population_64x16(torch, B, path):
     cfg = synth.config("population")
     W = synth.make_weights(cfg, 0)
     P, N = cfg["n_candidates"], cfg["batch"]
     obs, noise = synth.make_obs(cfg, N, 1), synth.make_noise(cfg, N, 2)
-    pop = synth.guided_population(synth.dissimilarity_map(8, 100, 5), P, 6)
+    pop = population_lattices(P)
     # the reference chunks below (N samples) must take the population's path
     ev = B.Evo(cfg, W, (P + 1) * N, wide_rows=N * cfg["horizon"] if path == "wide" else -1)
     x, dev = ev.population(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(), pop)
