@@ -40,7 +40,11 @@ WORKLOADS = {
     "manip": ("manip", [1.0, 0.5, 0.125], 0.125, "bernoulli"),
     "scale256": ("scale256", [1.0, 0.5, 0.25, 0.125], 0.125, "bernoulli"),
     "scale1024": ("scale1024", [1.0, 0.5, 0.25, 0.125], 0.125, "bernoulli"),
+    # redundancy-aware initialisation (Eq. 6 map + Eq. 7 sampling) on Push-T-shaped activations
+    "redundancy": ("pusht", [1.0], 1.0, "bernoulli"),
 }
+REDUNDANCY_SAMPLES = 16          # all-refresh queries whose activations build the map
+FP32_LANES_PER_SM = 128          # GB300 SM: 4 x 32 FP32 lanes, one FMA (2 FLOPs) per lane per clock
 L2_FLUSH_BYTES = 256 << 20
 
 
@@ -331,6 +335,68 @@ def run_ours(args, world, rank, local):
     return line, cfg
 
 
+def run_redundancy(args, rank):
+    """Dissimilarity maps (Eq. 6 and variants) from the all-refresh trace of
+    REDUNDANCY_SAMPLES Push-T-shaped queries, and 64 guided schedules (Eq. 7)."""
+    import torch
+    from paper_2607_20293_gb300 import binding, build
+    build.build()
+    binding.load()
+    cfg = synth.config("pusht")
+    N, U, T, H, E = REDUNDANCY_SAMPLES, 3 * cfg["n_layer"], cfg["n_steps"], cfg["horizon"], cfg["n_emb"]
+    W = synth.make_weights(cfg, 0)
+    ev = binding.Evo(cfg, W, N)
+    obs = torch.from_numpy(synth.make_obs(cfg, N, 1)).cuda()
+    noise = torch.from_numpy(synth.make_noise(cfg, N, 2)).cuda()
+    trace = torch.zeros((T, U, N, H, E), device="cuda")
+    ones = np.ones((U, T), np.uint8)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, device="cuda")
+
+    def timed(fn, reps):
+        out = []
+        for i in range(max(3, args.warmup) + reps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            if i >= max(3, args.warmup):
+                out.append(a.elapsed_time(b))
+        return statistics.median(out)
+
+    clocks = Clocks(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks.start()
+    trace_ms = timed(lambda: ev.denoise(obs, noise, ones, trace=trace), args.steps)
+    maps = {}
+    for m in binding.METRICS:
+        maps[m] = timed(lambda: binding.redundancy_map(trace, m), args.steps)
+    d = binding.redundancy_map(trace, "cosine")
+    P, K = 64, 240
+    rnd = torch.from_numpy(synth.guided_randoms(P, K, 7).view(np.int64)).cuda()
+    guided_ms = timed(lambda: binding.guided_schedules(d, K, rnd), args.steps)
+    clk = clocks.stop()
+    n = H * E
+    pair_flops = 2.0 * U * N * n * T * (T + 1) / 2          # cosine: one multiply-add per entry and pair
+    sm = torch.cuda.get_device_properties(0).multi_processor_count
+    mhz = (clk or {}).get("sm_max_mhz") or 2070.0
+    peak = sm * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
+    achieved = pair_flops / (maps["cosine"] * 1e-3) / 1e12
+    return {
+        "metric": "redundancy map latency (Eq. 6 cosine from 16 all-refresh Push-T queries) and guided schedules/s (Eq. 7)",
+        "value": maps["cosine"], "unit": "ms", "higher_is_better": False, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"redundancy map: {describe(cfg, N)}, U {U} x T {T} lattice, n {n} entries per activation",
+                   "l2": "flushed between timed calls (256 MiB write)"},
+        "map_ms": maps, "trace_collection_ms": trace_ms,
+        "guided": {"schedules": P, "K": K, "ms": guided_ms, "schedules_per_s": P / (guided_ms * 1e-3)},
+        "roofline": {"bound": "alu", "kernel": "pair_kernel (cosine)", "achieved": achieved, "peak": peak,
+                     "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                     "peak_source": f"{sm} SMs x {FP32_LANES_PER_SM} FP32 lanes x 2 FLOP x {mhz:.0f} MHz"},
+        "clocks": clk,
+    }
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -346,6 +412,10 @@ def main():
     name, fracs, head_frac, kind = WORKLOADS[args.workload]
     if args.fractions:
         head_frac = args.fractions[0]
+    if args.workload == "redundancy" and args.impl == "ours":
+        if rank == 0:
+            print(json.dumps(run_redundancy(args, rank)))
+        return
 
     if args.impl == "reference":
         if rank != 0:

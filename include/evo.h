@@ -193,6 +193,42 @@ evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* j
  * tensor-core GEMMs); kernels = kernel launches of that call. */
 evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels);
 
+/* Redundancy-aware initialisation (Sec. 3.3).
+ *
+ * Dissimilarity map of Eq. 6 and its variants from the residual activations of
+ * the uncached policy: trace = the device output of evo_denoise_trace with the
+ * all-refresh lattice, [T][U][N][n] fp32 (n = H*E entries per activation).
+ * For every unit b and step t, d[b][t] = mean over the N samples of
+ * 1/(T-1) sum_{t' != t} D(a_t, a_t'), with D by metric:
+ *   EVO_METRIC_COSINE  1 - cosine similarity (Eq. 6; a zero activation counts as 1)
+ *   EVO_METRIC_MSE     mean squared difference of the entries
+ *   EVO_METRIC_L1      mean absolute difference of the entries
+ *   EVO_METRIC_W1      Wasserstein-1 distance between the entries' empirical
+ *                      distributions (mean |sorted a_t - sorted a_t'|); n a power of two <= 16384
+ *   d       device [U][T] fp32 (output)
+ *   scratch device, evo_redundancy_scratch_bytes(...) bytes, caller-owned
+ * 2 <= T <= 128.  Asynchronous on the stream; deterministic. */
+enum { EVO_METRIC_COSINE = 0, EVO_METRIC_MSE = 1, EVO_METRIC_L1 = 2, EVO_METRIC_W1 = 3 };
+size_t evo_redundancy_scratch_bytes(int32_t T, int32_t U, int32_t N, int32_t n, int32_t metric);
+evo_status evo_redundancy_map(const float* trace, int32_t T, int32_t U, int32_t N, int32_t n, int32_t metric,
+                              float* d, void* scratch, void* stream);
+
+/* Guided sampling of P fixed-budget schedules (Eq. 7): K distinct lattice
+ * cells each, drawn without replacement with probability proportional to
+ * (eps + w)^gamma, w = d / max d (d > 0).  The weights are taken in fixed
+ * point, q = floor((eps + w)^gamma * 2^40) (double precision, gamma a positive
+ * integer <= 16), and draw k of schedule p takes, among the cells not yet
+ * drawn in index order (b * T + t), the first whose running sum of q exceeds
+ * rnd[p][k] mod (sum of the remaining q), or the first cell not yet drawn
+ * when only zero weights remain -- exact integer arithmetic, so the
+ * result is reproducible bit for bit.
+ *   d    device [U][T] fp32, U * T <= 4096
+ *   rnd  device [P][K] unsigned 64-bit random integers (caller-drawn)
+ *   S    device [P][U][T] uint8 (output, 0/1)
+ * Asynchronous on the stream. */
+evo_status evo_guided_schedules(const float* d, int32_t U, int32_t T, int32_t K, float eps, int32_t gamma,
+                                const uint64_t* rnd, int32_t P, uint8_t* S, void* stream);
+
 /* The cudaError_t of the most recent CUDA runtime failure behind an
  * EVO_ERR_CUDA on the calling thread (0 if none): the detail a caller needs to
  * tell, for instance, a launch-configuration error from a device fault. */

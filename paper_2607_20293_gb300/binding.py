@@ -66,6 +66,9 @@ def load() -> ctypes.CDLL:
                                       ctypes.POINTER(I32)]),
         "evo_get_last_call": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I64)]),
         "evo_last_cuda_error": (I32, []),
+        "evo_redundancy_scratch_bytes": (SZ, [I32, I32, I32, I32, I32]),
+        "evo_redundancy_map": (I32, [P, I32, I32, I32, I32, I32, P, P, P]),
+        "evo_guided_schedules": (I32, [P, I32, I32, I32, ctypes.c_float, I32, P, I32, P, P]),
         "evo_status_string": (ctypes.c_char_p, [I32]),
     }
     for name, (res, args) in sig.items():
@@ -242,3 +245,36 @@ class Evo:
 
     def status(self) -> int:
         return load().evo_get_status(self._h)
+
+
+METRICS = {"cosine": 0, "mse": 1, "l1": 2, "w1": 3}
+
+
+def redundancy_map(trace, metric: str = "cosine", stream=None):
+    """Eq. 6 map d [U][T] from a device trace [T][U][N][H][E] (evo_denoise_trace
+    with the all-refresh lattice)."""
+    import torch
+    T, U, N = trace.shape[:3]
+    n = int(np.prod(trace.shape[3:]))
+    m = METRICS[metric]
+    lib = load()
+    nb = lib.evo_redundancy_scratch_bytes(T, U, N, n, m)
+    if nb == 0:
+        raise EvoError(ERR_SHAPE, "evo_redundancy_scratch_bytes")
+    scratch = torch.empty(nb, dtype=torch.uint8, device=trace.device)
+    d = torch.empty((U, T), dtype=torch.float32, device=trace.device)
+    _check(lib.evo_redundancy_map(_ptr(trace), T, U, N, n, m, _ptr(d), _ptr(scratch), _stream(stream)),
+           "evo_redundancy_map")
+    return d
+
+
+def guided_schedules(d, K: int, rnd, eps: float = 0.05, gamma: int = 2, stream=None):
+    """P lattices [P][U][T] of K cells each by Eq. 7 from the device map d [U][T];
+    rnd: device uint64 tensor [P][K] (torch has no uint64: pass int64 with the same bits)."""
+    import torch
+    U, T = d.shape
+    P = rnd.shape[0]
+    S = torch.empty((P, U, T), dtype=torch.uint8, device=d.device)
+    _check(load().evo_guided_schedules(_ptr(d), U, T, K, float(eps), int(gamma), _ptr(rnd), P, _ptr(S),
+                                       _stream(stream)), "evo_guided_schedules")
+    return S

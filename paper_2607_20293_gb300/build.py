@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libevo.so")
 BUILD = os.path.join(ROOT, "_build")
-SOURCES = ["evo_api.cu", "evo_job.cu", "evo_loop_s01.cu", "evo_loop_s23.cu", "evo_loop_s45.cu", "evo_loop_f32.cu", "evo_wide.cu"]
+SOURCES = ["evo_api.cu", "evo_job.cu", "evo_loop_s01.cu", "evo_loop_s23.cu", "evo_loop_s45.cu", "evo_loop_f32.cu", "evo_wide.cu", "evo_redundancy.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "-I", os.path.join(ROOT, "include")]

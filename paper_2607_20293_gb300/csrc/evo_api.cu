@@ -922,6 +922,27 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
 
 int32_t evo_last_cuda_error(void) { return g_last_cuda_error; }
 
+size_t evo_redundancy_scratch_bytes(int32_t T, int32_t U, int32_t N, int32_t n, int32_t metric) {
+  if (!redundancy_shape_ok(T, U, N, n, metric)) return 0;
+  return redundancy_scratch_bytes(T, U, N, n, metric);
+}
+
+evo_status evo_redundancy_map(const float* trace, int32_t T, int32_t U, int32_t N, int32_t n, int32_t metric,
+                              float* d, void* scratch, void* stream) {
+  if (!trace || !d || !scratch) return EVO_ERR_ARG;
+  if (!redundancy_shape_ok(T, U, N, n, metric)) return EVO_ERR_SHAPE;
+  EVO_CUDA(launch_redundancy(trace, T, U, N, n, metric, d, scratch, reinterpret_cast<cudaStream_t>(stream)));
+  return EVO_OK;
+}
+
+evo_status evo_guided_schedules(const float* d, int32_t U, int32_t T, int32_t K, float eps, int32_t gamma,
+                                const uint64_t* rnd, int32_t P, uint8_t* S, void* stream) {
+  if (!d || !rnd || !S || !(eps >= 0.f)) return EVO_ERR_ARG;
+  if (!guided_shape_ok(U, T, K, gamma, P)) return EVO_ERR_SHAPE;
+  EVO_CUDA(launch_guided(d, U, T, K, eps, gamma, rnd, P, S, reinterpret_cast<cudaStream_t>(stream)));
+  return EVO_OK;
+}
+
 evo_status evo_get_last_call(const evo_handle* h, int32_t* path, int64_t* kernels) {
   if (!h) return EVO_ERR_ARG;
   if (path) *path = h->last_path;

@@ -127,6 +127,15 @@ long long wide_rows_capacity(const WideState* w);
 long long wide_last_launches(const WideState* w);
 cudaError_t wide_run(WideState* w, const WideCall& c);
 
+// redundancy map and guided sampling (evo_redundancy.cu)
+size_t redundancy_scratch_bytes(int T, int U, int N, int n, int metric);
+bool redundancy_shape_ok(int T, int U, int N, int n, int metric);
+cudaError_t launch_redundancy(const float* trace, int T, int U, int N, int n, int metric, float* d, void* scratch,
+                              cudaStream_t st);
+bool guided_shape_ok(int U, int T, int K, int gamma, int P);
+cudaError_t launch_guided(const float* d, int U, int T, int K, float eps, int gamma, const uint64_t* rnd, int P,
+                          uint8_t* S, cudaStream_t st);
+
 // offsets (in floats) of the named tensors inside the float32 weight blob
 enum WOff {
   W_OBS_W, W_OBS_B, W_COND_POS, W_CM_W1, W_CM_B1, W_CM_W2, W_CM_B2, W_IN_W, W_IN_B, W_POS,
