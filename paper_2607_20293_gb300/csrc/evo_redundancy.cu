@@ -13,9 +13,9 @@
 // and d_{r,b,t} = 1/(T-1) sum_{t' != t} of the term; d_{b,t} = mean over r.
 //
 // Pair kernel: one block per (b, r).  The T rows are streamed through shared
-// memory in chunks of 32 entries; every thread owns a fixed set of (t, t')
-// pairs (t <= t') and accumulates its dot products or differences over the
-// chunks.  Per-sample maps go to scratch and are averaged in a second pass in
+// memory in chunks of 32 entries; every thread owns register tiles of 4 x 4
+// (t, t') pairs and accumulates their dot products or differences over the
+// chunks (four FMA-class operations per shared-memory word loaded).  Per-sample maps go to scratch and are averaged in a second pass in
 // a fixed order (deterministic).
 //
 // Guided sampling: one warp per schedule.  The Eq. 7 weights are taken in
@@ -35,7 +35,7 @@ namespace evo {
 
 namespace {
 
-constexpr int RM_CH = 32;           // entries per chunk
+constexpr int RM_CH = 64;           // entries per chunk
 constexpr int RM_THREADS = 256;
 constexpr int RM_MAX_T = 128;
 
@@ -43,71 +43,126 @@ enum { M_COS = 0, M_MSE = 1, M_L1 = 2, M_W1 = 3 };
 
 __host__ __device__ inline int n_pairs(int T) { return T * (T + 1) / 2; }
 
-size_t pair_smem(int T) {
-  return (size_t)T * (RM_CH + 1) * sizeof(float) + (size_t)T * T * sizeof(float) +
-         (size_t)n_pairs(T) * 2 * sizeof(uint8_t);
+constexpr int RM_LD = RM_CH + 4;    // shared row stride (floats): 16-byte rows, interleaved tiles hit distinct banks
+
+size_t pair_smem(int T) { return 2 * (size_t)T * RM_LD * sizeof(float) + (size_t)T * T * sizeof(float); }
+
+__device__ __forceinline__ void cp16(float* dst, const float* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
 }
 
+template <int METRIC>
+__device__ __forceinline__ float pair_op(float x, float y, float acc) {
+  if constexpr (METRIC == M_COS) return fmaf(x, y, acc);
+  if constexpr (METRIC == M_MSE) {
+    const float e = x - y;
+    return fmaf(e, e, acc);
+  }
+  return acc + fabsf(x - y);
+}
+
+// One block per (b, r).  The T x T matrix of pair statistics is cut into
+// register tiles of 4 x 4 (t, t') pairs; tile (i, j) takes rows
+// t in {i, i + Tq, i + 2 Tq, i + 3 Tq} and t' likewise from j (Tq = ceil(T/4)),
+// so the float4 loads of neighbouring threads fall in different banks.
 // rows: row t of (b, r) starts at base + ((t * U + b) * N + r) * n
-__global__ void __launch_bounds__(RM_THREADS) pair_kernel(const float* rows, int T, int U, int N, int n, int metric,
+template <int METRIC>
+__global__ void __launch_bounds__(RM_THREADS, METRIC == M_COS ? 1 : 2) pair_kernel(const float* rows, int T, int U, int N, int n,
                                                           float* dr /* [U][N][T] */) {
   extern __shared__ __align__(16) float rm_smem[];
-  float* xs = rm_smem;                                  // [T][RM_CH + 1]
-  float* G = xs + T * (RM_CH + 1);                      // [T][T]
-  uint8_t* pt = reinterpret_cast<uint8_t*>(G + T * T);  // pair (t, t2) for pair index p
+  float* xb = rm_smem;                                  // 2 x [T][RM_LD]: chunk c in buffer c & 1
+  float* G = xb + 2 * T * RM_LD;                        // [T][T]
   const int b = blockIdx.x / N, r = blockIdx.x % N;
-  const int P = n_pairs(T);
-  for (int t = threadIdx.x; t < T; t += blockDim.x) {
-    const int base = t * T - t * (t - 1) / 2;           // pairs (t, t..T-1) start here
-    for (int t2 = t; t2 < T; ++t2) {
-      pt[2 * (base + t2 - t)] = (uint8_t)t;
-      pt[2 * (base + t2 - t) + 1] = (uint8_t)t2;
-    }
-  }
-  constexpr int PPT = (RM_MAX_T * (RM_MAX_T + 1) / 2 + RM_THREADS - 1) / RM_THREADS;   // pairs per thread (max)
-  float acc[PPT];
+  const int Tq = (T + 3) / 4, tiles = Tq * Tq;
+  constexpr int TPT = ((RM_MAX_T / 4) * (RM_MAX_T / 4) + RM_THREADS - 1) / RM_THREADS;   // tiles per thread (max)
+  float acc[TPT][4][4];
 #pragma unroll
-  for (int i = 0; i < PPT; ++i) acc[i] = 0.f;
-  __syncthreads();
-  for (int c0 = 0; c0 < n; c0 += RM_CH) {
-    const int w = min(RM_CH, n - c0);
-    for (int v = threadIdx.x; v < T * RM_CH; v += blockDim.x) {
-      const int t = v / RM_CH, k = v % RM_CH;
-      xs[t * (RM_CH + 1) + k] = k < w ? rows[((long long)(t * U + b) * N + r) * n + c0 + k] : 0.f;
-    }
-    __syncthreads();
+  for (int q = 0; q < TPT; ++q)
 #pragma unroll
-    for (int i = 0; i < PPT; ++i) {
-      const int p = threadIdx.x + i * RM_THREADS;
-      if (p < P) {
-        const float* x = xs + pt[2 * p] * (RM_CH + 1);
-        const float* y = xs + pt[2 * p + 1] * (RM_CH + 1);
-        float s = 0.f;
-        if (metric == M_COS) {
-#pragma unroll 8
-          for (int k = 0; k < RM_CH; ++k) s = fmaf(x[k], y[k], s);
-        } else if (metric == M_MSE) {
-#pragma unroll 8
-          for (int k = 0; k < RM_CH; ++k) {
-            const float e = x[k] - y[k];
-            s = fmaf(e, e, s);
-          }
-        } else {
-#pragma unroll 8
-          for (int k = 0; k < RM_CH; ++k) s += fabsf(x[k] - y[k]);
-        }
-        acc[i] += s;
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[q][a][c] = 0.f;
+  // chunk c of every row -> buffer c & 1: 16-byte asynchronous copies when the
+  // rows are a multiple of 4 entries, plain loads otherwise (zero-padded tail)
+  const int nch = (n + RM_CH - 1) / RM_CH;
+  auto load_chunk = [&](int c) {
+    float* xs = xb + (c & 1) * T * RM_LD;
+    const int c0 = c * RM_CH, w = min(RM_CH, n - c0);
+    for (int v = threadIdx.x; v < T * (RM_CH / 4); v += blockDim.x) {
+      const int t = v / (RM_CH / 4), k = 4 * (v % (RM_CH / 4));
+      const float* src = rows + ((long long)(t * U + b) * N + r) * n + c0 + k;
+      float* dst = xs + t * RM_LD + k;
+      if (k + 3 < w && (n & 3) == 0) {
+        cp16(dst, src);
+      } else {
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (k < w) f.x = src[0];
+        if (k + 1 < w) f.y = src[1];
+        if (k + 2 < w) f.z = src[2];
+        if (k + 3 < w) f.w = src[3];
+        *reinterpret_cast<float4*>(dst) = f;
       }
     }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  load_chunk(0);
+  for (int c = 0; c < nch; ++c) {
+    if (c + 1 < nch) {
+      load_chunk(c + 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
     __syncthreads();
+    const float* xs = xb + (c & 1) * T * RM_LD;
+#pragma unroll
+    for (int q = 0; q < TPT; ++q) {
+      const int tile = threadIdx.x + q * RM_THREADS;
+      if (tile < tiles) {
+        const int i = tile / Tq, j = tile % Tq;
+        int ra[4], rc[4];
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+          ra[a] = min(i + a * Tq, T - 1);   // rows beyond T repeat the last row; their results are dropped
+          rc[a] = min(j + a * Tq, T - 1);
+        }
+#pragma unroll 2
+        for (int k = 0; k < RM_CH; k += 4) {
+          float4 x[4], y[4];
+#pragma unroll
+          for (int a = 0; a < 4; ++a) {
+            x[a] = *reinterpret_cast<const float4*>(xs + ra[a] * RM_LD + k);
+            y[a] = *reinterpret_cast<const float4*>(xs + rc[a] * RM_LD + k);
+          }
+#pragma unroll
+          for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+              float v = acc[q][a][c];
+              v = pair_op<METRIC>(x[a].x, y[c].x, v);
+              v = pair_op<METRIC>(x[a].y, y[c].y, v);
+              v = pair_op<METRIC>(x[a].z, y[c].z, v);
+              v = pair_op<METRIC>(x[a].w, y[c].w, v);
+              acc[q][a][c] = v;
+            }
+        }
+      }
+    }
+    __syncthreads();   // buffer c & 1 is refilled with chunk c + 2 next
   }
 #pragma unroll
-  for (int i = 0; i < PPT; ++i) {
-    const int p = threadIdx.x + i * RM_THREADS;
-    if (p < P) {
-      const int t = pt[2 * p], t2 = pt[2 * p + 1];
-      G[t * T + t2] = acc[i];
-      G[t2 * T + t] = acc[i];
+  for (int q = 0; q < TPT; ++q) {
+    const int tile = threadIdx.x + q * RM_THREADS;
+    if (tile < tiles) {
+      const int i = tile / Tq, j = tile % Tq;
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int t = i + a * Tq, t2 = j + c * Tq;
+          if (t < T && t2 < T) G[t * T + t2] = acc[q][a][c];
+        }
     }
   }
   __syncthreads();
@@ -116,7 +171,7 @@ __global__ void __launch_bounds__(RM_THREADS) pair_kernel(const float* rows, int
     for (int t2 = 0; t2 < T; ++t2) {
       if (t2 == t) continue;
       float term;
-      if (metric == M_COS) {
+      if (METRIC == M_COS) {
         const float nn = sqrtf(G[t * T + t]) * sqrtf(G[t2 * T + t2]);
         term = nn == 0.f ? 1.f : 1.f - G[t * T + t2] / nn;
       } else {
@@ -258,9 +313,22 @@ cudaError_t launch_redundancy(const float* trace, int T, int U, int N, int n, in
     rows = sorted;
   }
   const int sm = (int)pair_smem(T);
-  cudaError_t e = cudaFuncSetAttribute(pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+  cudaError_t e = cudaSuccess;
+  switch (metric) {
+    case M_COS:
+      e = cudaFuncSetAttribute(pair_kernel<M_COS>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+      if (e == cudaSuccess) pair_kernel<M_COS><<<U * N, RM_THREADS, sm, st>>>(rows, T, U, N, n, dr);
+      break;
+    case M_MSE:
+      e = cudaFuncSetAttribute(pair_kernel<M_MSE>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+      if (e == cudaSuccess) pair_kernel<M_MSE><<<U * N, RM_THREADS, sm, st>>>(rows, T, U, N, n, dr);
+      break;
+    default:
+      e = cudaFuncSetAttribute(pair_kernel<M_L1>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+      if (e == cudaSuccess) pair_kernel<M_L1><<<U * N, RM_THREADS, sm, st>>>(rows, T, U, N, n, dr);
+      break;
+  }
   if (e != cudaSuccess) return e;
-  pair_kernel<<<U * N, RM_THREADS, sm, st>>>(rows, T, U, N, n, metric, dr);
   mean_kernel<<<(U * T + 255) / 256, 256, 0, st>>>(dr, T, U, N, d);
   return cudaGetLastError();
 }

@@ -78,6 +78,16 @@ def test_map_push_t_sized_rows(torch, B, metric):
     _close(got, O.redundancy_map(trace.transpose(2, 1, 0, 3).astype(np.float64), metric))
 
 
+@pytest.mark.parametrize("metric", ["mse", "l1"])
+def test_map_ragged_rows(torch, B, metric):
+    # n = 77 entries: a partial chunk and rows that are not 16-byte multiples
+    rng = np.random.default_rng(22)
+    T, U, N, n = 7, 3, 2, 77
+    trace = rng.standard_normal((T, U, N, n)).astype(np.float32)
+    got = B.redundancy_map(torch.from_numpy(trace).cuda(), metric).cpu().numpy()
+    _close(got, O.redundancy_map(trace.transpose(2, 1, 0, 3).astype(np.float64), metric))
+
+
 def test_map_rejects_bad_shapes(torch, B):
     assert B.load().evo_redundancy_scratch_bytes(1, 4, 2, 64, 0) == 0          # T < 2
     assert B.load().evo_redundancy_scratch_bytes(10, 4, 2, 100, 3) == 0        # w1 needs a power of two
