@@ -42,6 +42,8 @@ WORKLOADS = {
     "scale1024": ("scale1024", [1.0, 0.5, 0.25, 0.125], 0.125, "bernoulli"),
     # redundancy-aware initialisation (Eq. 6 map + Eq. 7 sampling) on Push-T-shaped activations
     "redundancy": ("pusht", [1.0], 1.0, "bernoulli"),
+    # published and baseline schedules on the Push-T-shaped policy, batch 1
+    "schedules": ("pusht", [1.0], 1.0, "bernoulli"),
 }
 REDUNDANCY_SAMPLES = 16          # all-refresh queries whose activations build the map
 FP32_LANES_PER_SM = 128          # GB300 SM: 4 x 32 FP32 lanes, one FMA (2 FLOPs) per lane per clock
@@ -397,6 +399,72 @@ def run_redundancy(args, rank):
     }
 
 
+def published_lattices(task: str):
+    """BAC and EVO lattices [24][100] of the paper's appendix tables (tests/golden)."""
+    bac = np.zeros((24, 100), np.uint8)
+    evo = np.zeros((24, 100), np.uint8)
+    b = 0
+    with open(os.path.join(ROOT, "tests", "golden", f"schedules_{task}.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            _, bl, el = [p.strip() for p in line.split(";")]
+            bac[b, [int(v) for v in bl.split()]] = 1
+            evo[b, [int(v) for v in el.split()]] = 1
+            b += 1
+    return bac, evo
+
+
+def run_schedules(args):
+    """Push-T batch 1: chunks/s of the full lattice, EfficientVLA's fixed interval
+    (M = 8, 10), the paper's BAC and EVO Push-T lattices and Bernoulli(0.125)."""
+    import torch
+    from paper_2607_20293_gb300 import binding, build
+    build.build()
+    binding.load()
+    cfg = synth.config("pusht")
+    W = synth.make_weights(cfg, 0)
+    ev = binding.Evo(cfg, W, 1)
+    obs = torch.from_numpy(synth.make_obs(cfg, 1, 1)).cuda()
+    noise = torch.from_numpy(synth.make_noise(cfg, 1, 2)).cuda()
+    out = torch.empty((1, cfg["horizon"], cfg["action_dim"]), device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, device="cuda")
+    bac, evo = published_lattices("pusht")
+    lattices = {"full": np.ones((24, 100), np.uint8),
+                "EfficientVLA M=8": binding.schedule_fixed_interval(24, 100, 8),
+                "EfficientVLA M=10": binding.schedule_fixed_interval(24, 100, 10),
+                "BAC (paper, Push-T)": bac, "EVO (paper, Push-T, K=240)": evo,
+                "Bernoulli 0.125": schedule(cfg, 0.125, "bernoulli")}
+    clocks = Clocks(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks.start()
+    rows = {}
+    for name, S in lattices.items():
+        ts = []
+        for i in range(max(3, args.warmup) + args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            ev.denoise(obs, noise, S, out=out)
+            b.record()
+            b.synchronize()
+            if i >= max(3, args.warmup):
+                ts.append(a.elapsed_time(b))
+        rows[name] = {"cells": int(S.sum()), "gflop_per_chunk": ev.flops(S) / 1e9, "p50_ms": statistics.median(ts),
+                      "chunks_per_s": 1000.0 / statistics.mean(ts)}
+    clk = clocks.stop()
+    full = rows["full"]
+    for r in rows.values():
+        r["flop_ratio_vs_full"] = full["gflop_per_chunk"] / r["gflop_per_chunk"]
+        r["speedup_vs_full"] = r["chunks_per_s"] / full["chunks_per_s"]
+    best = rows["EVO (paper, Push-T, K=240)"]
+    return {"metric": "action chunks/s per schedule (Push-T-shaped, batch 1)", "value": best["chunks_per_s"],
+            "unit": "chunks/s", "higher_is_better": True, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "dtype": cfg["dtype"], "data": "synthetic",
+            "config": {"workload": f"published / baseline schedules: {describe(cfg, 1)}; value = the paper's EVO lattice",
+                       "l2": "flushed between timed steps (256 MiB write)"},
+            "schedules": rows, "clocks": clk}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -415,6 +483,10 @@ def main():
     if args.workload == "redundancy" and args.impl == "ours":
         if rank == 0:
             print(json.dumps(run_redundancy(args, rank)))
+        return
+    if args.workload == "schedules" and args.impl == "ours":
+        if rank == 0:
+            print(json.dumps(run_schedules(args)))
         return
 
     if args.impl == "reference":

@@ -138,6 +138,8 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
  * FLOPs of that unit.  Under EVO_EMPTY_FORCE a row whose first entry is 0 adds
  * one refresh. */
 evo_status evo_flops(const evo_handle* h, const uint8_t* S, int32_t S_rows, int64_t* flops_per_sample);
+/* The same count for a configuration without a handle; only the shape fields
+ * (and empty_cache) matter, and any positive model is accepted. */
 evo_status evo_flops_cfg(const evo_config* cfg, const uint8_t* S, int32_t S_rows, int64_t* flops_per_sample);
 
 /* Individual encoding of Eq. 3 -> lattice.  bt: K pairs (b, t) in host memory;
@@ -145,6 +147,12 @@ evo_status evo_flops_cfg(const evo_config* cfg, const uint8_t* S, int32_t S_rows
  * duplicates (EVO_ERR_SCHEDULE); S_out is written only on success. */
 evo_status evo_schedule_from_positions(const int16_t* bt, int32_t K, int32_t n_units, int32_t T,
                                        uint8_t* S_out);
+
+/* Fixed-interval baseline schedule (EfficientVLA, as the paper describes it:
+ * every unit refreshed synchronously at a fixed temporal interval, M refreshes
+ * per unit): S_out[n_units][T] (host) has ones at t_i = floor(i * T / M),
+ * i = 0..M-1, in every row.  1 <= M <= T. */
+evo_status evo_schedule_fixed_interval(int32_t n_units, int32_t T, int32_t M, uint8_t* S_out);
 
 /* Debug variant of evo_denoise that also records the residual added at every
  * lattice cell: trace device [T][3L][N][H][E] float32 (refreshed cells: r_{b,t};

@@ -462,13 +462,16 @@ def guided_sample(q, K: int, rnd):
     probability proportional to q (Eq. 7); rnd [K] unsigned 64-bit integers.
     Draw k: target = rnd_k mod (sum of q over positions not yet drawn); the
     position drawn is the first, in index order, whose running sum of q over
-    the positions not yet drawn exceeds the target.  Returns the flat 0/1
-    lattice."""
+    the positions not yet drawn exceeds the target (when only zero weights
+    remain, the first position not yet drawn).  Returns the flat 0/1 lattice."""
     q = np.asarray(q, dtype=np.int64)
     out = np.zeros(q.size, dtype=np.uint8)
     for k in range(K):
         live = np.where(out == 0, q, 0)          # drawn positions add nothing to the running sum
         run = np.cumsum(live)                     # exact: integers
+        if run[-1] == 0:                          # only zero weights left: the first position not yet drawn
+            out[int(np.flatnonzero(out == 0)[0])] = 1
+            continue
         target = int(rnd[k]) % int(run[-1])
         out[int(np.searchsorted(run, target, side="right"))] = 1
     return out
@@ -479,3 +482,18 @@ def guided_schedules(d, K: int, eps: float, gamma: int, rnd):
     d = np.asarray(d)
     q = guided_weights(d, eps, gamma)
     return np.stack([guided_sample(q, K, rnd[p]).reshape(d.shape) for p in range(len(rnd))])
+
+
+# ---------------------------------------------------------------------------
+# Baseline schedules (Sec. 1, Sec. 4.1 baselines) and the FLOP table (Table 1)
+# ---------------------------------------------------------------------------
+
+def fixed_interval_schedule(B: int, T: int, M: int):
+    """EfficientVLA as the paper describes it: every unit refreshed
+    synchronously at a fixed temporal interval, M refreshes per unit.  Reading:
+    the refresh steps are t_i = floor(i * T / M), i = 0..M-1 (t = 0 included,
+    so no unit starts from an empty cache)."""
+    S = np.zeros((B, T), dtype=np.uint8)
+    for i in range(M):
+        S[:, (i * T) // M] = 1
+    return S

@@ -60,6 +60,7 @@ def load() -> ctypes.CDLL:
         "evo_flops": (I32, [P, P, I32, ctypes.POINTER(I64)]),
         "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
         "evo_schedule_from_positions": (I32, [P, I32, I32, I32, P]),
+        "evo_schedule_fixed_interval": (I32, [I32, I32, I32, P]),
         "evo_get_status": (I32, [P]),
         "evo_set_profile_events": (I32, [P, P, P]),
         "evo_get_launch_info": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I32), ctypes.POINTER(I32),
@@ -150,6 +151,13 @@ def schedule_from_positions(positions, n_units: int, T: int) -> np.ndarray:
     out = np.zeros((n_units, T), dtype=np.uint8)
     _check(load().evo_schedule_from_positions(bt.ctypes.data if bt.size else None, bt.shape[0], n_units, T,
                                               out.ctypes.data), "evo_schedule_from_positions")
+    return out
+
+
+def schedule_fixed_interval(n_units: int, T: int, M: int) -> np.ndarray:
+    """Fixed-interval baseline lattice [n_units][T]: every unit at t = floor(i T / M), i < M."""
+    out = np.zeros((n_units, T), dtype=np.uint8)
+    _check(load().evo_schedule_fixed_interval(n_units, T, M, out.ctypes.data), "evo_schedule_fixed_interval")
     return out
 
 

@@ -97,6 +97,14 @@ bool config_ok(const evo_config* c) {
   return true;
 }
 
+// The FLOP accountant is arithmetic on the shapes only: any positive model
+// (the kernels' limits above do not apply)
+bool flops_config_ok(const evo_config* c) {
+  return c && c->n_layer > 0 && c->n_layer <= 21 && c->n_emb > 0 && c->n_head > 0 && c->n_emb % c->n_head == 0 &&
+         c->horizon > 0 && c->action_dim > 0 && c->n_obs >= 0 && c->obs_dim > 0 && c->n_steps > 0 &&
+         (c->empty_cache == EVO_EMPTY_ZERO || c->empty_cache == EVO_EMPTY_FORCE);
+}
+
 void weight_offsets(const evo_config* c, int* wo) {
   const int E = c->n_emb, A = c->action_dim, D = c->obs_dim, H = c->horizon, Cm = 1 + c->n_obs;
   int o = 0;
@@ -337,7 +345,7 @@ size_t evo_weight_count(const evo_config* cfg) {
 }
 
 evo_status evo_flops_cfg(const evo_config* cfg, const uint8_t* S, int32_t S_rows, int64_t* out) {
-  if (!config_ok(cfg) || !S || !out) return EVO_ERR_ARG;
+  if (!flops_config_ok(cfg) || !S || !out) return EVO_ERR_ARG;
   const int U = 3 * cfg->n_layer;
   if (S_rows != U && S_rows != cfg->n_layer) return EVO_ERR_SCHEDULE;
   if (!lattice_ok(S, (size_t)S_rows * cfg->n_steps)) return EVO_ERR_SCHEDULE;
@@ -361,6 +369,14 @@ evo_status evo_schedule_from_positions(const int16_t* bt, int32_t K, int32_t n_u
     cell = 1;
   }
   std::memcpy(S_out, s.data(), s.size());
+  return EVO_OK;
+}
+
+evo_status evo_schedule_fixed_interval(int32_t n_units, int32_t T, int32_t M, uint8_t* S_out) {
+  if (!S_out || n_units <= 0 || T <= 0 || M < 1 || M > T) return EVO_ERR_ARG;
+  std::memset(S_out, 0, (size_t)n_units * T);
+  for (int b = 0; b < n_units; ++b)
+    for (int i = 0; i < M; ++i) S_out[(size_t)b * T + (long long)i * T / M] = 1;
   return EVO_OK;
 }
 

@@ -325,3 +325,14 @@ def test_published_evo_schedules_have_budget_240(task):
     assert O.budget(S) == 240
     bac = O.schedule_from_positions([(b, t) for b, (_, bl, _) in enumerate(rows) for t in bl], 24, 100)
     assert np.all(bac[:, 0] == 1)          # every BAC row refreshes at the first step
+
+
+@pytest.mark.parametrize("T,M", [(100, 8), (100, 10), (100, 100), (10, 3), (7, 1)])
+def test_fixed_interval_schedule_properties(T, M):
+    S = O.fixed_interval_schedule(5, T, M)
+    assert np.all(S.sum(1) == M)                       # M refreshes per unit
+    assert np.all(S == S[0])                           # all units synchronous
+    assert S[0, 0] == 1                                # the first step refreshes
+    steps = np.flatnonzero(S[0])
+    gaps = np.diff(np.append(steps, T))                # fixed interval: gaps differ by at most one
+    assert gaps.max() - gaps.min() <= 1 and gaps.sum() == T
