@@ -237,6 +237,48 @@ evo_status evo_redundancy_map(const float* trace, int32_t T, int32_t U, int32_t 
 evo_status evo_guided_schedules(const float* d, int32_t U, int32_t T, int32_t K, float eps, int32_t gamma,
                                 const uint64_t* rnd, int32_t P, uint8_t* S, void* stream);
 
+/* Schedule search (Sec. 3.2 genetic algorithm, Sec. 3.3 redundancy-guided
+ * initialisation and target-conditioned early stopping, Eq. 8 and 9).  Host
+ * code; fitness comes from the caller:
+ *   evo_fitness_fn(user, S [P][n_units][T] uint8 host, P, n_units, T, fitness[P])
+ * returns 0 on success (e.g. -dev_l2 of evo_denoise_population; higher is better).
+ * The search keeps every individual at exactly `budget` unique positions
+ * (block_wise: `budget` steps in every unit row, the ablation's Block-wise GA),
+ * evaluates each distinct schedule once (signature memo), carries `elites`
+ * over, breeds the rest by tournament selection, set-level crossover (common
+ * positions kept, each other one with probability 1/2), mutation (each
+ * position resampled with probability mutation_rate) and repair; `guided` of
+ * the initial individuals follow Eq. 7 (d_map host [n_units][T], as from
+ * evo_redundancy_map), the others are uniform.  With early_stop, candidates
+ * whose quick fitness reaches q_base are evaluated by `formal`; the first (in
+ * fitness order) whose formal fitness is at least q_base - delta_acc is
+ * returned and the search stops.  Every random choice draws from one
+ * SplitMix64 stream seeded by `seed`: the search is reproducible.
+ * best_S: host [n_units][T] uint8 (the accepted schedule, else the best seen). */
+typedef int32_t (*evo_fitness_fn)(void* user, const uint8_t* S, int32_t P, int32_t n_units, int32_t T,
+                                  double* fitness);
+typedef struct evo_search_config {
+  int32_t n_units, n_steps;
+  int32_t budget;            /* K (block_wise = 0) or refresh steps per unit (block_wise = 1) */
+  int32_t block_wise;
+  int32_t population, elites, generations, tournament;
+  int32_t guided;            /* initial individuals drawn by Eq. 7 (needs d_map) */
+  int32_t gamma;             /* Eq. 7 exponent (positive integer) */
+  float eps;                 /* Eq. 7 offset */
+  float pad_;
+  double crossover_rate, mutation_rate;
+  int32_t early_stop;
+  int32_t pad2_;
+  double q_base, delta_acc;  /* Eq. 8 / Eq. 9 */
+  uint64_t seed;
+} evo_search_config;
+typedef struct evo_search_result {
+  double best_fitness;
+  int32_t generations, evaluations, formal_evaluations, memo_hits, stopped_early, pad_;
+} evo_search_result;
+evo_status evo_search(const evo_search_config* cfg, const float* d_map, evo_fitness_fn quick, evo_fitness_fn formal,
+                      void* user, uint8_t* best_S, evo_search_result* result);
+
 /* The cudaError_t of the most recent CUDA runtime failure behind an
  * EVO_ERR_CUDA on the calling thread (0 if none): the detail a caller needs to
  * tell, for instance, a launch-configuration error from a device fault. */

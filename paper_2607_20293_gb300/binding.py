@@ -28,6 +28,26 @@ class EvoConfig(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int32) for f in _FIELDS]
 
 
+class SearchConfig(ctypes.Structure):
+    _fields_ = [("n_units", ctypes.c_int32), ("n_steps", ctypes.c_int32), ("budget", ctypes.c_int32),
+                ("block_wise", ctypes.c_int32), ("population", ctypes.c_int32), ("elites", ctypes.c_int32),
+                ("generations", ctypes.c_int32), ("tournament", ctypes.c_int32), ("guided", ctypes.c_int32),
+                ("gamma", ctypes.c_int32), ("eps", ctypes.c_float), ("pad_", ctypes.c_float),
+                ("crossover_rate", ctypes.c_double), ("mutation_rate", ctypes.c_double),
+                ("early_stop", ctypes.c_int32), ("pad2_", ctypes.c_int32), ("q_base", ctypes.c_double),
+                ("delta_acc", ctypes.c_double), ("seed", ctypes.c_uint64)]
+
+
+class SearchResult(ctypes.Structure):
+    _fields_ = [("best_fitness", ctypes.c_double), ("generations", ctypes.c_int32), ("evaluations", ctypes.c_int32),
+                ("formal_evaluations", ctypes.c_int32), ("memo_hits", ctypes.c_int32),
+                ("stopped_early", ctypes.c_int32), ("pad_", ctypes.c_int32)]
+
+
+FITNESS_FN = ctypes.CFUNCTYPE(ctypes.c_int32, ctypes.c_void_p, ctypes.POINTER(ctypes.c_uint8), ctypes.c_int32,
+                              ctypes.c_int32, ctypes.c_int32, ctypes.POINTER(ctypes.c_double))
+
+
 class EvoError(RuntimeError):
     def __init__(self, code: int, what: str):
         self.code = code
@@ -67,6 +87,7 @@ def load() -> ctypes.CDLL:
                                       ctypes.POINTER(I32)]),
         "evo_get_last_call": (I32, [P, ctypes.POINTER(I32), ctypes.POINTER(I64)]),
         "evo_last_cuda_error": (I32, []),
+        "evo_search": (I32, [ctypes.POINTER(SearchConfig), P, FITNESS_FN, FITNESS_FN, P, P, ctypes.POINTER(SearchResult)]),
         "evo_redundancy_scratch_bytes": (SZ, [I32, I32, I32, I32, I32]),
         "evo_redundancy_map": (I32, [P, I32, I32, I32, I32, I32, P, P, P]),
         "evo_guided_schedules": (I32, [P, I32, I32, I32, ctypes.c_float, I32, P, I32, P, P]),
@@ -286,3 +307,45 @@ def guided_schedules(d, K: int, rnd, eps: float = 0.05, gamma: int = 2, stream=N
     _check(load().evo_guided_schedules(_ptr(d), U, T, K, float(eps), int(gamma), _ptr(rnd), P, _ptr(S),
                                        _stream(stream)), "evo_guided_schedules")
     return S
+
+
+def search(n_units: int, n_steps: int, budget: int, quick, formal=None, d_map=None, block_wise: bool = False,
+           population: int = 30, elites: int = 10, generations: int = 30, tournament: int = 3, guided: int = 0,
+           crossover_rate: float = 0.9, mutation_rate: float = 0.02, eps: float = 0.05, gamma: int = 2,
+           early_stop: bool = False, q_base: float = 0.0, delta_acc: float = 0.0, seed: int = 0):
+    """evo_search with Python fitness callables: f(S [P][n_units][T] uint8) -> [P] floats.
+    Returns (best lattice, best fitness, stats dict)."""
+    cfg = SearchConfig(n_units, n_steps, budget, int(block_wise), population, elites, generations, tournament,
+                       guided, gamma, eps, 0.0, crossover_rate, mutation_rate, int(early_stop), 0, q_base,
+                       delta_acc, seed & ((1 << 64) - 1))
+    errors = []
+
+    def wrap(f):
+        if f is None:
+            return ctypes.cast(None, FITNESS_FN)
+
+        def cb(user, S, P, U, T, out):
+            try:
+                arr = np.ctypeslib.as_array(S, shape=(P, U, T)).copy()
+                vals = f(arr)
+                for i in range(P):
+                    out[i] = float(vals[i])
+                return 0
+            except Exception as e:          # reported after the call returns
+                errors.append(e)
+                return 1
+        return FITNESS_FN(cb)
+
+    qf, ff = wrap(quick), wrap(formal)
+    dm = None if d_map is None else np.ascontiguousarray(d_map, dtype=np.float32)
+    best = np.zeros((n_units, n_steps), dtype=np.uint8)
+    res = SearchResult()
+    rc = load().evo_search(ctypes.byref(cfg), None if dm is None else dm.ctypes.data, qf, ff, None,
+                           best.ctypes.data, ctypes.byref(res))
+    if errors:
+        raise errors[0]
+    _check(rc, "evo_search")
+    stats = dict(generations=res.generations, evaluations=res.evaluations,
+                 formal_evaluations=res.formal_evaluations, memo_hits=res.memo_hits,
+                 stopped_early=res.stopped_early)
+    return best, res.best_fitness, stats

@@ -16,9 +16,9 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libevo.so")
 BUILD = os.path.join(ROOT, "_build")
-SOURCES = ["evo_api.cu", "evo_job.cu", "evo_loop_s01.cu", "evo_loop_s23.cu", "evo_loop_s45.cu", "evo_loop_f32.cu", "evo_wide.cu", "evo_redundancy.cu"]
+SOURCES = ["evo_api.cu", "evo_job.cu", "evo_loop_s01.cu", "evo_loop_s23.cu", "evo_loop_s45.cu", "evo_loop_f32.cu", "evo_wide.cu", "evo_redundancy.cu", "evo_search.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
+FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2", "-Xcompiler", "-ffp-contract=off",
          "-I", os.path.join(ROOT, "include")]
 
 
@@ -45,7 +45,7 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
         objs.append(o)
         if _stale(o, [s] + headers):
             jobs.append([nvcc, *ARCH, *FLAGS, *(extra or []), "-c", s, "-o", o])
