@@ -292,6 +292,9 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
   if (es == 2 && p.Cm > 16) return -1;                      // tensor-core attention pads memory keys to 16
   if (p.A > 16) return -1;                                  // action dimensions of the fused head
+  // head partials per row segment of min(Ec, 32) columns: sum, sum of squares, A dots
+  p.npr = rup((2 + p.A) * (p.Ec > 32 ? p.Ec / 32 : 1), 4);
+  if (p.C * (p.Ec > 32 ? p.Ec / 32 : 1) > 16) return -1;   // partials a head row sums
   if (es == 2) {
     if (p.Mp > 32) return -1;
   } else {
@@ -308,14 +311,13 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   // head exchange, head weights on chip
   for (int cache_smem = 1; cache_smem >= 0; --cache_smem)
     for (int kvall = 1; kvall >= 0; --kvall)
-      for (int head_sep = 1; head_sep >= 0; --head_sep)
-        for (int headw = 1; headw >= 0; --headw) {
-          p.kv_slots = kvall ? p.L : 1;
-          p.head_sep = head_sep;
-          p.headw_smem = headw;
-          const int total = smem_layout(p, es, cache_smem);
-          if (total <= smem_limit) return total;
-        }
+      for (int head_sep = 1; head_sep >= 0; --head_sep) {
+        if (!head_sep && p.M * p.npr > p.blk) continue;     // one head landing block per ablk block
+        p.kv_slots = kvall ? p.L : 1;
+        p.head_sep = head_sep;
+        const int total = smem_layout(p, es, cache_smem);
+        if (total <= smem_limit) return total;
+      }
   return -1;
 }
 
@@ -581,6 +583,8 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   vtake(p.v_lnfb, E);
   vtake(p.v_headw, (size_t)E * A);
   vtake(p.v_headb, A);
+  vtake(p.v_headG, A);
+  vtake(p.v_headB, A);
   std::memcpy(&vec[p.v_inw], W(W_IN_W), (size_t)A * E * 4);
   std::memcpy(&vec[p.v_inb], W(W_IN_B), E * 4);
   std::memcpy(&vec[p.v_pos], W(W_POS), (size_t)H * E * 4);
@@ -589,6 +593,16 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   for (int e = 0; e < E; ++e)   // W_head transposed: [A][E]
     for (int a = 0; a < A; ++a) vec[p.v_headw + (size_t)a * E + e] = W(W_HEAD_W)[(size_t)e * A + a];
   std::memcpy(&vec[p.v_headb], W(W_HEAD_B), A * 4);
+  // LN_f folded into the head: (LN(a) . W)_a = rstd (sum_e a_e g_e W_ea - mean G_a) + B_a
+  for (int a = 0; a < A; ++a) {
+    double G = 0.0, B = 0.0;
+    for (int e = 0; e < E; ++e) {
+      G += (double)W(W_LNF_G)[e] * (double)W(W_HEAD_W)[(size_t)e * A + a];
+      B += (double)W(W_LNF_B)[e] * (double)W(W_HEAD_W)[(size_t)e * A + a];
+    }
+    vec[p.v_headG + a] = (float)G;
+    vec[p.v_headB + a] = (float)B;
+  }
   if (cudaMalloc(&h->vec, vec.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMemcpy(h->vec, vec.data(), vec.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
     return fail(EVO_ERR_CUDA);

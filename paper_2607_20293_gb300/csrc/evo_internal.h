@@ -26,18 +26,19 @@ struct SmemLayout {
   int ablk;    // [C][blk] f32: gathered residual columns, block c from CTA c; also the staging of outgoing partial sums
   int rs;      // [C][blk] f32: incoming partial sums of the second GEMM, block c from CTA c
   int xln;     // [Mp][lda] T: normalised rows, the first GEMM's A operand; aliased by the first GEMM's output
-  int hblk;    // 2 x [C][blk] f32: gathered columns for the output head, by step parity (or -1: the head uses ablk)
-  int hsrc;    // 2 x [M*Ec] f32: the head's outgoing copy of this CTA's columns, by step parity
+  int hblk;    // 2 x [C][M][npr] f32: the output head's gathered row partials by step parity (head_sep), else = ablk
+  int hsrc;    // (2 or 1) x [M][npr] f32: this CTA's row partials for the head
   int pb;      // [M][PLD] f32: attention probabilities
   int oc;      // [Mp][ldo] T: attention output slice, A operand of the second GEMM
   int ac;      // [M][Ec] f32: this CTA's columns of the residual stream
   int cs;      // [3L][M][Ec] T: this CTA's columns of every unit's cache (or -1: caches in global memory)
   int kvs;     // [kv_slots][g][1+n_obs][kvw] f32: memory keys/values for cross-attention
-  int cst;     // f32 constants: in_w[:, cols], in_b[cols], pos[:, cols], lnf_g, lnf_b, head_b, (head_w)
+  int cst;     // f32 constants: in_w[:, cols], in_b[cols], pos[:, cols], head_b, G, B (4-padded), gw[A][cols]
   int x;       // [M][A] f32: current sample x (replicated in every CTA of the cluster)
   int z;       // [M][A] f32: DDPM noise of the current step
   int sch;     // [T] u64: this job's lattice, bit b of word t = unit b refreshed at step t
   int stb;     // [T][8] f32: sampler coefficients of every step
+  int psch;    // [T] u64: the producer warp's own copy of the job's refresh masks
   int bars;    // mbarriers: full[nslot], empty[nslot], cluster, xg, xr, xh
   int total;
 };
@@ -58,7 +59,8 @@ struct JobParams {
   int n_jobs;
   int sampler, force;
   int nslot, slot_bytes;
-  int head_sep, headw_smem;
+  int head_sep;                   // 1: head partials double-buffered by step parity; 0: one buffer + cluster barrier
+  int npr;                        // floats per row of a head partial block: (2 + A) per row segment, 4-padded
   // samples
   int samples;                    // real samples in this launch
   int per_sched;                  // samples that share one schedule
@@ -82,6 +84,7 @@ struct JobParams {
   // float32 vectors
   const float* vec;
   long long v_inw, v_inb, v_pos, v_lnfg, v_lnfb, v_headw, v_headb;
+  long long v_headG, v_headB;     // [A]: sum_e lnf_g[e] W_head[e][a], sum_e lnf_b[e] W_head[e][a]
   // caches [n_jobs][U][C][M][Ec] (dtype T), used when sm.cs < 0
   void* cache;
   float* trace;                   // [T][U][samples][H][E] or null

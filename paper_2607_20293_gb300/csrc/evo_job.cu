@@ -165,14 +165,16 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   const int g1b = p.M * p.ldg1 * 4 > p.Mp * p.ldh * es ? p.M * p.ldg1 * 4 : p.Mp * p.ldh * es;
   s.xln = off;
   off += al(xb > g1b ? xb : g1b, 128);
+  // head partials: double-buffered landing blocks of M*npr floats, or one set
+  // landing in ablk (block c at c*blk, where a unit's exchanges put c's data)
   if (p.head_sep) {
     s.hblk = off;
-    off += al(2 * p.C * p.blk * 4, 128);
-    s.hsrc = off;
-    off += al(2 * p.M * p.Ec * 4, 128);
+    off += al(2 * p.C * p.M * p.npr * 4, 128);
   } else {
-    s.hblk = s.hsrc = -1;
+    s.hblk = s.ablk;
   }
+  s.hsrc = off;
+  off += al((p.head_sep ? 2 : 1) * p.M * p.npr * 4, 128);
   s.pb = off;
   off += al(p.M * PLD * 4, 128);
   s.oc = off;
@@ -188,7 +190,7 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   s.kvs = off;
   off += al(p.kv_slots * p.g * p.Cm * p.kvw * 4, 128);
   s.cst = off;
-  off += al((p.A * p.Ec + p.Ec + p.H * p.Ec + 2 * p.E + ((p.A + 3) & ~3) + (p.headw_smem ? p.E * p.A : 0)) * 4, 128);
+  off += al((p.A * p.Ec + p.Ec + p.H * p.Ec + 3 * ((p.A + 3) & ~3) + p.A * p.Ec) * 4, 128);
   s.x = off;
   off += al(p.M * p.A * 4, 16);
   s.z = off;
@@ -196,6 +198,8 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   s.stb = off;
   off += al(p.T * 8 * 4, 16);
   s.sch = off;
+  off += al(p.T * 8, 16);
+  s.psch = off;
   off += al(p.T * 8, 16);
   s.bars = off;
   off += (2 * p.nslot + 5) * 8;

@@ -156,18 +156,33 @@ struct Loop {
   }
 
   // ---------------------------------------------------------------- producer warp
+  // The whole warp turns the job's lattice into one refresh mask per step (its
+  // own copy, psch); lane 0 then walks the refreshed units in order and streams
+  // their weight slabs through the ring.
   __device__ __forceinline__ static void producer(const JobParams& p, Ctx& cx, uint32_t cid, uint32_t ncl) {
+    uint64_t* psch = reinterpret_cast<uint64_t*>(cx.smem + p.sm.psch);
+    const uint64_t units = p.U >= 64 ? ~0ull : (1ull << p.U) - 1ull;
     uint32_t q = 0;
     for (int job = cid; job < p.n_jobs; job += ncl) {
       const int s0 = min(job * S::G, p.samples - 1);
       const uint8_t* Sl = p.S + (long long)(s0 / p.per_sched) * p.S_stride;
-      uint64_t valid = 0;
-      for (int t = 0; t < p.T; ++t) {
+      for (int t = cx.lane; t < p.T; t += 32) {
+        uint64_t mask = 0;
+#pragma unroll 8
         for (int b = 0; b < p.U; ++b) {
           const int row = (p.S_rows == p.U) ? b : b / 3;
-          const bool vb = (valid >> b) & 1ull;
-          if (!(Sl[row * p.T + t] != 0 || (p.force && !vb))) continue;   // same rule as the compute warps
-          valid |= 1ull << b;
+          if (Sl[row * p.T + t] != 0) mask |= 1ull << b;
+        }
+        psch[t] = mask;
+      }
+      __syncwarp();
+      uint64_t valid = 0;
+      for (int t = 0; t < p.T && cx.lane == 0; ++t) {
+        uint64_t refresh = (psch[t] | (p.force ? ~valid : 0ull)) & units;   // same rule as the compute warps
+        valid |= refresh;
+        while (refresh) {
+          const int b = __ffsll((long long)refresh) - 1;
+          refresh &= refresh - 1ull;
           const int l = b / 3, u = b % 3;
           for (int piece = 0; piece < 2; ++piece) {
             const uint8_t* src =
@@ -199,7 +214,9 @@ struct Loop {
           }
         }
       }
+      __syncwarp();
     }
+    if (cx.lane != 0) return;
     // drain: every slab issued has landed before this CTA may exit (bounded waits)
     const uint32_t first = q > (uint32_t)S::NSLOT ? q - S::NSLOT : 0u;
     for (uint32_t k = first; k < q; ++k)
@@ -800,106 +817,116 @@ struct Loop {
   }
 
   // ---------------------------------------------------------------- output head + sampler step
+  // eps = LN_f(a) W_head + b_head (Eq. 1's denoiser output) from per-row partial
+  // sums: with mean, rstd of the full row, (LN_f(a) W)_a = rstd (sum_e a_e g_e W_ea
+  // - mean G_a) + B_a, G_a = sum_e g_e W_ea, B_a = sum_e b_e W_ea.  Each CTA
+  // reduces its own columns to 2 + A numbers per row (sum, sum of squares, the
+  // A dots with gw = g W) and all-gathers them; every CTA then adds the C
+  // partials of each row in the same order, so all CTAs hold the same x.
+  // Without head_sep the blocks land in ablk at c*blk: block c of CTA r last
+  // held r's second-GEMM partials for this CTA, which this CTA has received.
   __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t) {
-    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
+    constexpr int L = Ec < 32 ? Ec : 32;             // lanes holding one row segment of this CTA's columns
+    constexpr int SEG = Ec / L;                      // segments per row
+    static_assert(C * SEG <= 16, "head: at most 16 partials per row");
+    const float* ac = reinterpret_cast<const float*>(cx.smem + p.sm.ac);
     float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
     const float* z = reinterpret_cast<const float*>(cx.smem + p.sm.z);
     const float* cst = reinterpret_cast<const float*>(cx.smem + p.sm.cst);
-    const float* lnf_g = cst + p.A * Ec + Ec + H * Ec;
-    const float* lnf_b = lnf_g + E;
-    const float* head_b = lnf_b + E;
-    const float* hw = p.headw_smem ? head_b + ((p.A + 3) & ~3) : p.vec + p.v_headw;
-    const float* hb;
-    if (p.head_sep) {
-      // double-buffered by step parity: source, landing blocks and barrier
-      const int par = t & 1;
-      float* src = reinterpret_cast<float*>(cx.smem + p.sm.hsrc) + par * MEc;
+    const int A4 = (p.A + 3) & ~3, NP = 2 + p.A, npr = p.npr;
+    const float* head_b = cst + p.A * Ec + Ec + H * Ec;
+    const float* Gs = head_b + A4;
+    const float* Bs = head_b + 2 * A4;
+    const float* gw = head_b + 3 * A4;
+    const int par = p.head_sep ? (t & 1) : 0;
+    float* ps = reinterpret_cast<float*>(cx.smem + p.sm.hsrc) + par * M * npr;
+    const int hstr = p.head_sep ? M * npr : S::blk;   // landing stride between the C blocks
+    const float* hb = reinterpret_cast<const float*>(cx.smem + p.sm.hblk) + par * C * M * npr;
+    // 1. this CTA's partials (MEc is a multiple of 64: the guard is warp-uniform)
 #pragma unroll
-      for (int k = 0; k < EPT; ++k) {
-        const int e = cx.tid + k * NCT;
-        if (MEc % NCT == 0 || e < MEc) src[e] = ac[e];
+    for (int k = 0; k < EPT; ++k) {
+      const int e = cx.tid + k * NCT;
+      if (MEc % NCT == 0 || e < MEc) {
+        const int m = e >> S::lEc, j = e & (Ec - 1);
+        const bool lead = (j & (L - 1)) == 0;
+        float* dst = ps + m * npr + (j / L) * NP;
+        const float v = ac[e];
+        float s0 = v, s1 = v * v;
+#pragma unroll
+        for (int o = L / 2; o > 0; o >>= 1) {
+          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+        }
+        if (lead) {
+          dst[0] = s0;
+          dst[1] = s1;
+        }
+        for (int a = 0; a < p.A; ++a) {
+          float d = v * gw[a * Ec + j];
+#pragma unroll
+          for (int o = L / 2; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+          if (lead) dst[2 + a] = d;
+        }
       }
-      hb = reinterpret_cast<const float*>(cx.smem + p.sm.hblk) + par * C * S::blk;
-      fence_proxy_async();
-      bar_compute();
-      send_blocks(cx, src, 0, hb, cx.xh + par);
-      exchange_wait(p, cx, cx.xh + par, par ? cx.ph1 : cx.ph0);
-    } else {
-      hb = reinterpret_cast<const float*>(cx.smem + p.sm.ablk);
-      fence_proxy_async();
-      bar_compute();
-      send_blocks(cx, ac, 0, hb, cx.xg);
-      exchange_wait(p, cx, cx.xg, cx.pg);
+    }
+    fence_proxy_async();
+    bar_compute();
+    // 2. all-gather: the block of M*npr floats to every CTA, issue spread over the warps
+    {
+      constexpr int PER = (C + NCW - 1) / NCW;
+      const int r = cx.warp + NCW * cx.lane;
+      if (cx.lane < PER && r < C)
+        bulk_s2c(mapa(smem_u32(hb + cx.c * hstr), (uint32_t)r), ps, (uint32_t)(M * npr * 4),
+                 mapa(smem_u32(cx.xh + par), (uint32_t)r));
+      if (cx.tid == 0) mbar_arrive_expect_tx(cx.xh + par, (uint32_t)(C * M * npr * 4));
+      wait_parity(smem_u32(cx.xh + par), par ? cx.ph1 : cx.ph0, true, cx, p.status);
+      if (par) cx.ph1 ^= 1u; else cx.ph0 ^= 1u;
     }
     cp_async_wait_all();
     bar_compute();
+    // 3. rows: half a warp per row; lane hl adds quantity hl (and hl + 16) over the partials
     const float4 tab0 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32);
     const float4 tab1 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32 + 16);
-    const float inv_sa = tab0.x, s1 = tab0.y, cx0 = tab0.z, cxt = tab0.w, sig = tab1.x;
+    const float inv_sa = tab0.x, s1c = tab0.y, cx0 = tab0.z, cxt = tab0.w, sig = tab1.x;
     const float sab = tab1.y, sabp = tab1.z, s1p = tab1.w;
-    constexpr int NV = E / 64;
     const int half = cx.lane >> 4, hl = cx.lane & 15;
 #pragma unroll
     for (int m0 = 0; m0 < M; m0 += 2 * NCW) {
       if (M % (2 * NCW) == 0 || m0 + cx.warp * 2 < M) {
         const int m = m0 + cx.warp * 2 + half;
-        float4 v[NV];
-        float s = 0.f, s2 = 0.f;
+        float t0 = 0.f, t1 = 0.f;
 #pragma unroll
-        for (int j = 0; j < NV; ++j) {
-          const int col = 4 * (hl + 16 * j);
-          v[j] = *reinterpret_cast<const float4*>(hb + (col >> S::lEc) * S::blk + (m << S::lEc) + (col & (Ec - 1)));
-          s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
-          s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
-        }
+        for (int r = 0; r < C; ++r)
 #pragma unroll
-        for (int o = 8; o > 0; o >>= 1) {
-          s += __shfl_xor_sync(0xffffffffu, s, o);
-          s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-        }
-        const float mean = s * S::invE;
-        const float rstd = rsqrtf(fmaxf(s2 * S::invE - mean * mean, 0.f) + 1e-5f);
-        // normalised values of this lane's columns, then one reduced dot per action dim
-#pragma unroll
-        for (int j = 0; j < NV; ++j) {
-          const int col = 4 * (hl + 16 * j);
-          const float4 g4 = *reinterpret_cast<const float4*>(lnf_g + col);
-          const float4 b4 = *reinterpret_cast<const float4*>(lnf_b + col);
-          v[j].x = (v[j].x - mean) * rstd * g4.x + b4.x;
-          v[j].y = (v[j].y - mean) * rstd * g4.y + b4.y;
-          v[j].z = (v[j].z - mean) * rstd * g4.z + b4.z;
-          v[j].w = (v[j].w - mean) * rstd * g4.w + b4.w;
-        }
-        // one reduced dot per action dimension over rows of W_head^T (float4 loads)
-        float eps = 0.f;
-        for (int a = 0; a < p.A; ++a) {
-          float part = 0.f;
-#pragma unroll
-          for (int j = 0; j < NV; ++j) {
-            const float4 w = *reinterpret_cast<const float4*>(hw + a * E + 4 * (hl + 16 * j));
-            part = fmaf(v[j].x, w.x, part);
-            part = fmaf(v[j].y, w.y, part);
-            part = fmaf(v[j].z, w.z, part);
-            part = fmaf(v[j].w, w.w, part);
+          for (int sg = 0; sg < SEG; ++sg) {
+            const float* src = hb + r * hstr + m * npr + sg * NP;
+            if (hl < NP) t0 += src[hl];
+            if (hl + 16 < NP) t1 += src[hl + 16];
           }
-          const float e = group_sum<16>(part);
-          if (hl == a) eps = e + head_b[a];
-        }
+        const float S0 = __shfl_sync(0xffffffffu, t0, 0, 16);
+        const float S1 = __shfl_sync(0xffffffffu, t0, 1, 16);
+        const int qd = 2 + hl;
+        const float d0 = __shfl_sync(0xffffffffu, t0, qd & 15, 16);
+        const float d1 = __shfl_sync(0xffffffffu, t1, qd & 15, 16);
         if (hl < p.A) {
+          const float D = qd < 16 ? d0 : d1;
+          const float mean = S0 * S::invE;
+          const float rstd = rsqrtf(fmaxf(S1 * S::invE - mean * mean, 0.f) + 1e-5f);
+          const float eps = rstd * (D - mean * Gs[hl]) + Bs[hl] + head_b[hl];
           const float xv = x[m * p.A + hl];
-          float x0 = (xv - s1 * eps) * inv_sa;
+          float x0 = (xv - s1c * eps) * inv_sa;
           x0 = fminf(1.0f, fmaxf(-1.0f, x0));
           float xn;
           if (p.sampler == 0) {
             xn = cx0 * x0 + cxt * xv + sig * z[m * p.A + hl];
           } else {
-            xn = sabp * x0 + s1p * ((xv - sab * x0) / s1);
+            xn = sabp * x0 + s1p * ((xv - sab * x0) / s1c);
           }
           x[m * p.A + hl] = xn;
         }
       }
     }
-    if (!p.head_sep) csync(p, cx);                    // ablk is the next gather's landing zone
+    if (!p.head_sep) csync(p, cx);                    // one landing buffer: every CTA has read it
     bar_compute();
   }
 
@@ -933,25 +960,33 @@ struct Loop {
         x[v] = p.noise[((long long)(s % p.obs_mod) * H + (m & (H - 1))) * p.A + (v % p.A)];
       }
       stage_kv_job(p, cx, sample0);
+      // DDPM noise: thread v < G*H*A/4 copies 16 bytes of z_t per step (one chunk per thread)
+      const float* zsrc = nullptr;
+      int zdst = 0;
+      if (p.sampler == 0) {
+        const int per = H * p.A / 4;
+        if (cx.tid < S::G * per) {
+          const int i = cx.tid / per, w = cx.tid - i * per;
+          const int s = min(sample0 + i, p.samples - 1);
+          zsrc = p.noise + ((long long)p.obs_mod + (s % p.obs_mod)) * H * p.A + 4 * w;   // slot 1 + t at t = 0
+          zdst = i * H * p.A + 4 * w;
+        }
+      }
+      const long long zstep = (long long)p.obs_mod * H * p.A;
+      const uint64_t units = p.U >= 64 ? ~0ull : (1ull << p.U) - 1ull;
+      constexpr uint64_t CA_UNITS = 0x2492492492492492ull;     // bits 3l + 1: cross-attention units
       bar_compute();
       uint64_t valid = 0;
       for (int t = 0; t < p.T; ++t) {
-        const uint64_t refresh = sch[t] | (p.force ? ~valid : 0ull);
-        // sampler coefficients of this step (used at the head)
+        const uint64_t refresh = (sch[t] | (p.force ? ~valid : 0ull)) & units;
         // stage z_t (DDPM) and, when every layer has a slot, the memory keys/values
         // of this step's refreshed cross-attention units
-        if (p.sampler == 0) {
-          const int per = H * p.A / 4;
-          for (int v = cx.tid; v < S::G * per; v += NCT) {
-            const int i = v / per, w = v - i * per;
-            const int s = min(sample0 + i, p.samples - 1);
-            cp_async16(z + i * H * p.A + 4 * w,
-                       p.noise + ((long long)(1 + t) * p.obs_mod + (s % p.obs_mod)) * H * p.A + 4 * w);
-          }
-        }
+        if (zsrc) cp_async16(z + zdst, zsrc + t * zstep);
         if (p.kv_slots > 1)
-          for (int l = 0; l < p.L; ++l)
-            if ((refresh >> (3 * l + 1)) & 1ull) stage_kv(p, cx, l, t, kvs + l * S::G * p.Cm * S::kvw);
+          for (uint64_t ca = refresh & CA_UNITS; ca; ca &= ca - 1ull) {
+            const int l = (__ffsll((long long)ca) - 1) / 3;
+            stage_kv(p, cx, l, t, kvs + l * S::G * p.Cm * S::kvw);
+          }
         // input embedding into this CTA's columns
 #pragma unroll
         for (int k = 0; k < EPT; ++k) {
@@ -963,9 +998,11 @@ struct Loop {
             ac[e] = acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j];
           }
         }
+        // units in order: a refreshed unit, or a run of up to 8 skipped ones
         int b = 0;
         while (b < p.U) {
-          if ((refresh >> b) & 1ull) {
+          const uint64_t rest = refresh >> b;
+          if (rest & 1ull) {
             valid |= 1ull << b;
             const int u = b % 3;
             if (u == 0) unit<0>(p, cx, job, b, t, sample0);
@@ -973,8 +1010,8 @@ struct Loop {
             else unit<2>(p, cx, job, b, t, sample0);
             ++b;
           } else {
-            int b1 = b + 1;
-            while (b1 < p.U && b1 - b < 8 && !((refresh >> b1) & 1ull)) ++b1;
+            const int gap = rest ? __ffsll((long long)rest) - 1 : 64;
+            const int b1 = min(min(b + gap, p.U), b + 8);
             skip_run(p, cx, job, b, b1, t, sample0, valid);
             b = b1;
           }
@@ -1059,22 +1096,24 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
     for (int v = threadIdx.x; v < S::H * S::Ec; v += NTHREADS)
       d[v] = p.vec[p.v_pos + (v / S::Ec) * S::E + c0 + (v % S::Ec)];
     d += S::H * S::Ec;
-    for (int v = threadIdx.x; v < S::E; v += NTHREADS) {
-      d[v] = p.vec[p.v_lnfg + v];
-      d[S::E + v] = p.vec[p.v_lnfb + v];
+    const int A4 = (p.A + 3) & ~3;
+    for (int v = threadIdx.x; v < p.A; v += NTHREADS) {
+      d[v] = p.vec[p.v_headb + v];
+      d[A4 + v] = p.vec[p.v_headG + v];
+      d[2 * A4 + v] = p.vec[p.v_headB + v];
     }
-    d += 2 * S::E;
-    for (int v = threadIdx.x; v < p.A; v += NTHREADS) d[v] = p.vec[p.v_headb + v];
-    d += (p.A + 3) & ~3;
-    if (p.headw_smem)
-      for (int v = threadIdx.x; v < S::E * p.A; v += NTHREADS) d[v] = p.vec[p.v_headw + v];   // [A][E]
+    d += 3 * A4;
+    for (int v = threadIdx.x; v < p.A * S::Ec; v += NTHREADS) {   // gw[a][j] = lnf_g[col] * W_head[col][a]
+      const int a = v / S::Ec, col = c0 + v % S::Ec;
+      d[v] = p.vec[p.v_lnfg + col] * p.vec[p.v_headw + (long long)a * S::E + col];
+    }
   }
   __syncthreads();
   hw_cluster_sync();
   const bool bad = p.sched_err != nullptr && *p.sched_err != 0;
   if (!bad) {
     if (cx.warp == NCW) {
-      if (cx.lane == 0) Loop<T, S>::producer(p, cx, cid, ncl);
+      Loop<T, S>::producer(p, cx, cid, ncl);
       __syncwarp();
     } else {
       Loop<T, S>::compute(p, cx, cid, ncl);
@@ -1096,7 +1135,15 @@ bool shape_matches(const JobParams& p) {
 
 template <typename T, class S>
 cudaError_t shape_prepare(int smem_bytes, int* max_clusters) {
-  cudaError_t e = cudaFuncSetAttribute(job_kernel<T, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  // The limit is a process-wide attribute of the kernel: allow the device
+  // maximum, so that handles with different plans of this shape coexist (each
+  // launch passes its own size).
+  int dev = 0, optin = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(job_kernel<T, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           optin > smem_bytes ? optin : smem_bytes);
   if (e != cudaSuccess) return e;
   if (S::C > 8) {
     e = cudaFuncSetAttribute(job_kernel<T, S>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);

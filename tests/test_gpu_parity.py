@@ -170,6 +170,24 @@ def test_odd_batch_with_two_samples_per_job(torch, B):
     check(ev.denoise(d_obs, d_noise, S).cpu().numpy(), O.denoise(W, cfg, obs, noise, S), TOL["bf16"])
 
 
+def test_handles_with_different_plans_coexist(torch, B):
+    # one compiled shape, two shared-memory plans (100 and 10 loop steps): the
+    # smaller handle, created second, must not shrink the larger one's launch limit
+    big = setup("pusht", 1, torch, B)
+    cfg_s = synth.config("pusht", n_steps=10)
+    W_s = synth.make_weights(cfg_s, 0)
+    obs_s, noise_s = synth.make_obs(cfg_s, 1, 1), synth.make_noise(cfg_s, 1, 2)
+    ev_s = B.Evo(cfg_s, W_s, 1)
+    cfg, W, obs, noise, ev, d_obs, d_noise = big
+    S = synth.bernoulli_schedule(24, 100, 0.2, 8)
+    S_s = synth.bernoulli_schedule(24, 10, 0.5, 9)
+    for _ in range(2):
+        got_s = ev_s.denoise(torch.from_numpy(obs_s).cuda(), torch.from_numpy(noise_s).cuda(), S_s).cpu().numpy()
+        got = ev.denoise(d_obs, d_noise, S).cpu().numpy()
+        check(got_s, O.denoise(W_s, cfg_s, obs_s, noise_s, S_s), TOL["bf16"], "10 steps")
+        check(got, O.denoise(W, cfg, obs, noise, S), TOL["bf16"], "100 steps")
+
+
 # ------------------------------------------------------------------ batched configs at full size
 
 @pytest.mark.parametrize("path", ["wide", "cluster"])
