@@ -111,10 +111,12 @@ struct Loop {
   static_assert(!MMA_ATT || S::G * att_sample_elems<1>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
 
   // ---------------------------------------------------------------- rings and barriers
-  // wait for the oldest unreleased slab (cx.q)
+  // wait for the next slab not yet acquired (cx.qa); slabs are released in
+  // the same order (cx.q), a warp holds at most two at a time
   __device__ __forceinline__ static const uint8_t* ring_acquire(const JobParams& p, Ctx& cx) {
-    const uint32_t slot = cx.q % S::NSLOT;
-    const uint32_t ph = (cx.q / S::NSLOT) & 1u;
+    const uint32_t slot = cx.qa % S::NSLOT;
+    const uint32_t ph = (cx.qa / S::NSLOT) & 1u;
+    cx.qa++;
     wait_parity(smem_u32(&cx.full[slot]), ph, false, cx, p.status);
     return cx.smem + p.sm.ring + slot * S::SLOT;
   }
@@ -239,7 +241,12 @@ struct Loop {
     return kt == S::pK(U, Q) / 16 - 1 || slab_first<U, Q>(kt + 1);
   }
 
-  // bf16: warp w owns n-tiles w, w+8, ... (NTW of them)
+  // bf16: warp w owns n-tiles w, w+8, ... (NTW of them).  The A and B
+  // fragments of k-tile kt + PD are loaded before the MMAs of k-tile kt, so
+  // shared-memory latency overlaps the MMA chain; a slab is acquired when its
+  // first k-tile is loaded and released after its last k-tile's MMAs.  With
+  // PD = 2 a load window spans at most two slabs unless a middle slab holds a
+  // single k-tile (then PD = 1).
   template <int U, int Q>
   __device__ __forceinline__ static void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda,
                                                    const uint8_t* slab0,
@@ -247,6 +254,8 @@ struct Loop {
     constexpr int NT = S::pN(U, Q) / 8, NTW = (NT + NCW - 1) / NCW;
     constexpr int NKT = S::pK(U, Q) / 16, K0 = S::pK0(U, Q), KPS = S::pKps(U, Q);
     constexpr int HDR = S::pHdr(U, Q);
+    constexpr int PD = (KPS >= 2 || NKT <= K0 + 1) ? 2 : 1, NB = PD + 1;
+    static_assert(S::NSLOT >= 2, "prefetch holds two slabs");
     const uint8_t* sl = slab0 + HDR + cx.lane * 8;
 #pragma unroll
     for (int m = 0; m < MT; ++m)
@@ -255,20 +264,31 @@ struct Loop {
 #pragma unroll
         for (int r = 0; r < 4; ++r) acc[m][i][r] = 0.f;
     const __nv_bfloat16* arow = A + (cx.lane & 15) * lda + (cx.lane >> 4) * 8;
-#pragma unroll
-    for (int kt = 0; kt < NKT; ++kt) {
+    uint32_t af[NB][MT][4];
+    uint2 bf[NB][NTW];
+    auto load = [&](const int kt) {
       if (slab_first<U, Q>(kt)) sl = ring_acquire(p, cx) + cx.lane * 8;
       const int kk = kt < K0 ? kt : (kt - K0) % KPS;
-      uint32_t a[MT][4];
 #pragma unroll
-      for (int m = 0; m < MT; ++m) ldmatrix_x4(a[m], arow + m * 16 * lda + kt * 16);
+      for (int m = 0; m < MT; ++m) ldmatrix_x4(af[kt % NB][m], arow + m * 16 * lda + kt * 16);
+#pragma unroll
+      for (int i = 0; i < NTW; ++i) {
+        const int nt = cx.warp + i * NCW;
+        if (NT % NCW == 0 || nt < NT) bf[kt % NB][i] = *reinterpret_cast<const uint2*>(sl + (kk * NT + nt) * 256);
+      }
+    };
+#pragma unroll
+    for (int kt = 0; kt < PD; ++kt)
+      if (kt < NKT) load(kt);
+#pragma unroll
+    for (int kt = 0; kt < NKT; ++kt) {
+      if (kt + PD < NKT) load(kt + PD);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
         const int nt = cx.warp + i * NCW;
         if (NT % NCW == 0 || nt < NT) {
-          const uint2 bf = *reinterpret_cast<const uint2*>(sl + (kk * NT + nt) * 256);
 #pragma unroll
-          for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], a[m], bf);
+          for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], af[kt % NB][m], bf[kt % NB][i]);
         }
       }
       if (slab_last<U, Q>(kt)) ring_release(cx);
@@ -1045,7 +1065,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   cx.xg = cx.cbar + 1;
   cx.xr = cx.cbar + 2;
   cx.xh = cx.cbar + 3;
-  cx.q = 0;
+  cx.q = cx.qa = 0;
   cx.cph = cx.pg = cx.pr = cx.ph0 = cx.ph1 = 0;
   cx.dead = 0;
   {

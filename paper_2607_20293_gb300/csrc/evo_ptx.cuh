@@ -211,7 +211,8 @@ struct Ctx {
   uint64_t* xg;    // receives the all-gather of a for a unit (and the head when it uses ablk)
   uint64_t* xr;    // receives the reduce-scatter partial sums
   uint64_t* xh;    // receives the head's all-gather, two barriers by step parity
-  uint32_t q;      // slab counter (same sequence as the producer)
+  uint32_t q;      // next slab to release (same sequence as the producer)
+  uint32_t qa;     // next slab to acquire (qa - q slabs are held)
   uint32_t cph, pg, pr, ph0, ph1;   // phase parities
   int dead;
   int c, tid, warp, lane;

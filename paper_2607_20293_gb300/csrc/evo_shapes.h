@@ -5,7 +5,7 @@
 #pragma once
 
 #define EVO_SHAPES(X)                                           \
-  X(0, __nv_bfloat16, 256, 4, 16, 16, 1, 2, 32768, 3)          \
+  X(0, __nv_bfloat16, 256, 4, 16, 16, 1, 2, 32768, 4)          \
   X(1, __nv_bfloat16, 256, 4, 16, 16, 2, 2, 32768, 2)          \
   X(2, __nv_bfloat16, 256, 4, 16, 8, 1, 2, 32768, 4)           \
   X(3, __nv_bfloat16, 256, 4, 16, 4, 1, 2, 32768, 4)           \
