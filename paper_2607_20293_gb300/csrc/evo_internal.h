@@ -31,6 +31,7 @@ struct SmemLayout {
   int pb;      // [M][PLD] f32: attention probabilities
   int oc;      // [Mp][ldo] T: attention output slice, A operand of the second GEMM
   int ac;      // [M][Ec] f32: this CTA's columns of the residual stream
+  int acb;     // [M][Ec] bf16: copy of ac sent by the bf16 gather (operand type bf16)
   int cs;      // [3L][M][Ec] T: this CTA's columns of every unit's cache (or -1: caches in global memory)
   int kvs;     // [kv_slots][g][1+n_obs][kvw] f32: memory keys/values for cross-attention
   int cst;     // f32 constants: in_w[:, cols], in_b[cols], pos[:, cols], head_b, G, B (4-padded), gw[A][cols]

@@ -181,6 +181,8 @@ int smem_layout(JobParams& p, int es, int cache_smem) {
   off += al(p.Mp * p.ldo * es, 128);
   s.ac = off;                                   // end of the zero-initialised block
   off += al(p.M * p.Ec * 4, 128);
+  s.acb = off;
+  off += al(p.M * p.Ec * 2, 128);
   if (cache_smem) {
     s.cs = off;
     off += al(p.U * p.M * p.Ec * es, 128);

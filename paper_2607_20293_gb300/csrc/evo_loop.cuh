@@ -137,9 +137,10 @@ struct Loop {
     cx.cph ^= 1u;
   }
 
-  // receive one exchange phase (XBYTES) on barrier `bar`
-  __device__ __forceinline__ static void exchange_wait(const JobParams& p, Ctx& cx, uint64_t* bar, uint32_t& parity) {
-    if (cx.tid == 0) mbar_arrive_expect_tx(bar, XBYTES);
+  // receive one exchange phase (`bytes` in total, XBYTES by default) on barrier `bar`
+  __device__ __forceinline__ static void exchange_wait(const JobParams& p, Ctx& cx, uint64_t* bar, uint32_t& parity,
+                                                       uint32_t bytes = XBYTES) {
+    if (cx.tid == 0) mbar_arrive_expect_tx(bar, bytes);
     wait_parity(smem_u32(bar), parity, true, cx, p.status);
     parity ^= 1u;
   }
@@ -155,6 +156,18 @@ struct Loop {
       bulk_s2c(mapa(smem_u32(dst + cx.c * S::blk), r), src + r * src_stride, (uint32_t)(MEc * 4),
                mapa(smem_u32(rbar), r));
     }
+  }
+
+  // Send `bytes` from src to every CTA r of the cluster, landing at dst (this
+  // CTA's slot in r's buffer, same offset in every CTA), counted on r's
+  // barrier `rbar`; the C copies are issued by lanes of different warps.  The
+  // writers of src have executed fence_proxy_async() and a bar_compute().
+  __device__ __forceinline__ static void send_spread(Ctx& cx, const void* src, uint32_t bytes, const void* dst,
+                                                     uint64_t* rbar) {
+    constexpr int PER = (C + NCW - 1) / NCW;
+    const int r = cx.warp + NCW * cx.lane;
+    if (cx.lane < PER && r < C)
+      bulk_s2c(mapa(smem_u32(dst), (uint32_t)r), src, bytes, mapa(smem_u32(rbar), (uint32_t)r));
   }
 
   // ---------------------------------------------------------------- producer warp
@@ -329,6 +342,7 @@ struct Loop {
   // Rows m < M, half a warp per row, one pass for the mean and the second
   // moment.  Row m is read from the gathered blocks (column col is in block
   // col/Ec) and written to the A operand xln in type T.
+  // In bf16 mode the gathered blocks hold bf16 (block c at c * 2blk elements).
   __device__ __forceinline__ static void layernorm_rows(Ctx& cx, const float* blk, T* xln, const float* gam,
                                                         const float* bet) {
     constexpr int NV = E / 64;
@@ -342,7 +356,16 @@ struct Loop {
 #pragma unroll
         for (int j = 0; j < NV; ++j) {
           const int col = 4 * (hl + 16 * j);
-          v[j] = *reinterpret_cast<const float4*>(blk + (col >> S::lEc) * S::blk + (m << S::lEc) + (col & (Ec - 1)));
+          if constexpr (BF) {
+            const uint2 raw = *reinterpret_cast<const uint2*>(reinterpret_cast<const __nv_bfloat16*>(blk) +
+                                                              (col >> S::lEc) * (2 * S::blk) + (m << S::lEc) +
+                                                              (col & (Ec - 1)));
+            const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
+            const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
+            v[j] = make_float4(lo.x, lo.y, hi.x, hi.y);
+          } else {
+            v[j] = *reinterpret_cast<const float4*>(blk + (col >> S::lEc) * S::blk + (m << S::lEc) + (col & (Ec - 1)));
+          }
           s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
           s2 += (v[j].x * v[j].x + v[j].y * v[j].y) + (v[j].z * v[j].z + v[j].w * v[j].w);
         }
@@ -745,13 +768,27 @@ struct Loop {
       if (p.kv_slots == 1) stage_kv(p, cx, l, t, kvs);
       else kvs += l * S::G * p.Cm * S::kvw;
     }
-    // exchange 1: every CTA receives every CTA's columns of a.  ablk is read by
-    // LayerNorm below; CTA r sends into it again only after this CTA's partial
-    // sums (sent after the first GEMM) reached r.
-    fence_proxy_async();
-    bar_compute();                     // ac final for this unit
-    send_blocks(cx, ac, 0, ablk, cx.xg);
-    exchange_wait(p, cx, cx.xg, cx.pg);
+    // exchange 1: every CTA receives every CTA's columns of a (rounded to bf16
+    // in bf16 mode: they are only LayerNorm's input, whose output is bf16).
+    // ablk is read by LayerNorm below; CTA r sends into it again only after
+    // this CTA's partial sums (sent after the first GEMM) reached r.
+    if constexpr (BF) {
+      __nv_bfloat16* acb = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb);
+#pragma unroll
+      for (int k = 0; k < EPT; ++k) {
+        const int e = cx.tid + k * NCT;
+        if (MEc % NCT == 0 || e < MEc) acb[e] = __float2bfloat16_rn(ac[e]);
+      }
+      fence_proxy_async();
+      bar_compute();                   // ac final for this unit
+      send_spread(cx, acb, (uint32_t)(MEc * 2), ablk + cx.c * S::blk, cx.xg);
+      exchange_wait(p, cx, cx.xg, cx.pg, XBYTES / 2);
+    } else {
+      fence_proxy_async();
+      bar_compute();                   // ac final for this unit
+      send_blocks(cx, ac, 0, ablk, cx.xg);
+      exchange_wait(p, cx, cx.xg, cx.pg);
+    }
     // slab 0 of piece 1: [gamma | beta | first bias | second-GEMM bias slice | k-tiles]
     const uint8_t* s1 = ring_acquire(p, cx);
     const float* hdr = reinterpret_cast<const float*>(s1);
@@ -892,16 +929,8 @@ struct Loop {
     fence_proxy_async();
     bar_compute();
     // 2. all-gather: the block of M*npr floats to every CTA, issue spread over the warps
-    {
-      constexpr int PER = (C + NCW - 1) / NCW;
-      const int r = cx.warp + NCW * cx.lane;
-      if (cx.lane < PER && r < C)
-        bulk_s2c(mapa(smem_u32(hb + cx.c * hstr), (uint32_t)r), ps, (uint32_t)(M * npr * 4),
-                 mapa(smem_u32(cx.xh + par), (uint32_t)r));
-      if (cx.tid == 0) mbar_arrive_expect_tx(cx.xh + par, (uint32_t)(C * M * npr * 4));
-      wait_parity(smem_u32(cx.xh + par), par ? cx.ph1 : cx.ph0, true, cx, p.status);
-      if (par) cx.ph1 ^= 1u; else cx.ph0 ^= 1u;
-    }
+    send_spread(cx, ps, (uint32_t)(M * npr * 4), hb + cx.c * hstr, cx.xh + par);
+    exchange_wait(p, cx, cx.xh + par, par ? cx.ph1 : cx.ph0, (uint32_t)(C * M * npr * 4));
     cp_async_wait_all();
     bar_compute();
     // 3. rows: half a warp per row; lane hl adds quantity hl (and hl + 16) over the partials
