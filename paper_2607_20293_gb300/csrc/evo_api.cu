@@ -284,7 +284,7 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   p.kp_h = rup(p.hid, 16);
   p.ldh = es == 2 ? p.kp_h + 8 : p.kp_h;
   p.ldo = es == 2 ? p.kp_o + 8 : p.kp_o;
-  for (int u = 0; u < 3; ++u) p.hdr1[u] = rup(2 * E + p.n1[u] + p.Ec, 4) * 4;
+  for (int u = 0; u < 3; ++u) p.hdr1[u] = rup(p.n1[u] + p.Ec, 4) * 4;
   p.sampler = c->sampler;
   p.force = c->empty_cache == EVO_EMPTY_FORCE;
   p.invE = 1.0f / (float)E;
@@ -527,16 +527,20 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
         for (int n = 0; n < N; ++n) d[(size_t)k * N + n] = get(k, n);
     }
   };
-  // piece 1 = [float32 header][k-tiles], header = LayerNorm gain, shift, the
-  // first GEMM's bias columns and this CTA's columns of the second GEMM's bias;
-  // piece 2 = [k-tiles]
-  auto header = [&](uint8_t* dst, const float* g, const float* b, const float* bias, int nbias, auto colmap,
+  // piece 1 = [float32 header][k-tiles], header = the first GEMM's bias
+  // columns and this CTA's columns of the second GEMM's bias; piece 2 =
+  // [k-tiles].  The unit's LayerNorm affine is folded into the first GEMM:
+  // LN(a) W + b = xhat (g o W) + (beta W + b), xhat = (a - mean) * rstd, so the
+  // k-tiles hold g_k W[k][n] and the bias beta W + b (summed in double).
+  auto header = [&](uint8_t* dst, const float* beta, const float* bias, int nbias, auto colmap, auto wcol,
                     const float* bias2) {
     float* d = reinterpret_cast<float*>(dst);
-    for (int i = 0; i < E; ++i) d[i] = g[i];
-    for (int i = 0; i < E; ++i) d[E + i] = b[i];
-    for (int i = 0; i < nbias; ++i) d[2 * E + i] = bias[colmap(i)];
-    for (int i = 0; i < Ec; ++i) d[2 * E + nbias + i] = bias2[i];
+    for (int i = 0; i < nbias; ++i) {
+      double v = (double)bias[colmap(i)];
+      for (int k = 0; k < E; ++k) v += (double)beta[k] * (double)wcol(k, i);
+      d[i] = (float)v;
+    }
+    for (int i = 0; i < Ec; ++i) d[nbias + i] = bias2[i];
   };
   for (int c = 0; c < C; ++c) {
     const int h0 = (c * Ec) / dh;
@@ -549,20 +553,25 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
       const float* wo2 = WL(l, WL_CA_WO);
       const float* w1 = WL(l, WL_FF_W1);
       const float* w2 = WL(l, WL_FF_W2);
+      const float* g1 = WL(l, WL_LN1G);
+      const float* g2 = WL(l, WL_LN2G);
+      const float* g3 = WL(l, WL_LN3G);
+      auto sa_w = [&](int k, int n) { return wqkv[(size_t)k * 3 * E + qkv_col(n)]; };
+      auto ca_w = [&](int k, int n) { return wq[(size_t)k * E + h0 * dh + n]; };
+      auto ff_w = [&](int k, int n) { return w1[(size_t)k * 4 * E + c * hid + n]; };
       // SA
-      header(base + p.poff[0][0], WL(l, WL_LN1G), WL(l, WL_LN1B), WL(l, WL_SA_BQKV), p.n1[0], qkv_col,
-             WL(l, WL_SA_BO) + c * Ec);
-      put(base + p.poff[0][0] + p.hdr1[0], E, p.n1[0], [&](int k, int n) { return wqkv[(size_t)k * 3 * E + qkv_col(n)]; });
+      header(base + p.poff[0][0], WL(l, WL_LN1B), WL(l, WL_SA_BQKV), p.n1[0], qkv_col, sa_w, WL(l, WL_SA_BO) + c * Ec);
+      put(base + p.poff[0][0] + p.hdr1[0], E, p.n1[0], [&](int k, int n) { return g1[k] * sa_w(k, n); });
       put(base + p.poff[0][1], p.kp_o, E, [&](int k, int n) { return k < Ec ? wo1[(size_t)(c * Ec + k) * E + n] : 0.f; });
       // CA
-      header(base + p.poff[1][0], WL(l, WL_LN2G), WL(l, WL_LN2B), WL(l, WL_CA_BQ), p.n1[1],
-             [&](int n) { return h0 * dh + n; }, WL(l, WL_CA_BO) + c * Ec);
-      put(base + p.poff[1][0] + p.hdr1[1], E, p.n1[1], [&](int k, int n) { return wq[(size_t)k * E + h0 * dh + n]; });
+      header(base + p.poff[1][0], WL(l, WL_LN2B), WL(l, WL_CA_BQ), p.n1[1], [&](int n) { return h0 * dh + n; }, ca_w,
+             WL(l, WL_CA_BO) + c * Ec);
+      put(base + p.poff[1][0] + p.hdr1[1], E, p.n1[1], [&](int k, int n) { return g2[k] * ca_w(k, n); });
       put(base + p.poff[1][1], p.kp_o, E, [&](int k, int n) { return k < Ec ? wo2[(size_t)(c * Ec + k) * E + n] : 0.f; });
       // FFN
-      header(base + p.poff[2][0], WL(l, WL_LN3G), WL(l, WL_LN3B), WL(l, WL_FF_B1), p.n1[2],
-             [&](int n) { return c * hid + n; }, WL(l, WL_FF_B2) + c * Ec);
-      put(base + p.poff[2][0] + p.hdr1[2], E, p.n1[2], [&](int k, int n) { return w1[(size_t)k * 4 * E + c * hid + n]; });
+      header(base + p.poff[2][0], WL(l, WL_LN3B), WL(l, WL_FF_B1), p.n1[2], [&](int n) { return c * hid + n; }, ff_w,
+             WL(l, WL_FF_B2) + c * Ec);
+      put(base + p.poff[2][0] + p.hdr1[2], E, p.n1[2], [&](int k, int n) { return g3[k] * ff_w(k, n); });
       put(base + p.poff[2][1], p.kp_h, E, [&](int k, int n) { return k < hid ? w2[(size_t)(c * hid + k) * E + n] : 0.f; });
     }
   }

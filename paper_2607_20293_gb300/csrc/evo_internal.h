@@ -53,7 +53,7 @@ struct JobParams {
   int lda, ldg1, ldh, ldo, kvw;   // row strides (elements) of xln, q|k|v, hidden, attention output, memory k|v
   int lEc, lH;                    // log2 of Ec and H
   int n1[3];                      // first-GEMM width per unit kind (SA, CA, FFN)
-  int hdr1[3];                    // header bytes of piece 1: gamma, beta, first bias, second-GEMM bias slice
+  int hdr1[3];                    // header bytes of piece 1: first bias (LayerNorm shift folded in), second-GEMM bias slice
   int kv_slots;                   // L: memory keys/values of every layer prefetched per step; 1: per unit
   float invE;                     // 1 / E
   int kp_o, kp_h;                 // K of the second GEMMs (attention: Ec, FFN: hid), multiples of 16

@@ -74,7 +74,7 @@ struct Shape {
   static constexpr int ldh = ES == 2 ? kp_h + 8 : kp_h, ldo = ES == 2 ? kp_o + 8 : kp_o;
   static constexpr float invE = 1.0f / E;
   __host__ __device__ static constexpr int n1(int u) { return u == 0 ? n1_sa : (u == 1 ? n1_ca : n1_ff); }
-  __host__ __device__ static constexpr int hdr1(int u) { return ct_rup(2 * E + n1(u) + Ec, 4) * 4; }
+  __host__ __device__ static constexpr int hdr1(int u) { return ct_rup(n1(u) + Ec, 4) * 4; }
   // piece q of unit kind u: K x N slice behind a header, cut into ring slabs
   __host__ __device__ static constexpr int pK(int u, int q) { return q == 0 ? E : (u == 2 ? kp_h : kp_o); }
   __host__ __device__ static constexpr int pN(int u, int q) { return q == 0 ? n1(u) : E; }
@@ -343,8 +343,8 @@ struct Loop {
   // moment.  Row m is read from the gathered blocks (column col is in block
   // col/Ec) and written to the A operand xln in type T.
   // In bf16 mode the gathered blocks hold bf16 (block c at c * 2blk elements).
-  __device__ __forceinline__ static void layernorm_rows(Ctx& cx, const float* blk, T* xln, const float* gam,
-                                                        const float* bet) {
+  // The affine (gain, shift) is folded into the first GEMM's weights and bias.
+  __device__ __forceinline__ static void layernorm_rows(Ctx& cx, const float* blk, T* xln) {
     constexpr int NV = E / 64;
     const int half = cx.lane >> 4, hl = cx.lane & 15;
 #pragma unroll
@@ -379,10 +379,8 @@ struct Loop {
 #pragma unroll
         for (int j = 0; j < NV; ++j) {
           const int col = 4 * (hl + 16 * j);
-          const float4 g = *reinterpret_cast<const float4*>(gam + col);
-          const float4 bb = *reinterpret_cast<const float4*>(bet + col);
-          const float y0 = (v[j].x - mean) * rstd * g.x + bb.x, y1 = (v[j].y - mean) * rstd * g.y + bb.y;
-          const float y2 = (v[j].z - mean) * rstd * g.z + bb.z, y3 = (v[j].w - mean) * rstd * g.w + bb.w;
+          const float y0 = (v[j].x - mean) * rstd, y1 = (v[j].y - mean) * rstd;
+          const float y2 = (v[j].z - mean) * rstd, y3 = (v[j].w - mean) * rstd;
           T* dst = xln + m * S::lda + col;
           if constexpr (BF) {
             __nv_bfloat162 lo = __floats2bfloat162_rn(y0, y1), hi = __floats2bfloat162_rn(y2, y3);
@@ -410,7 +408,7 @@ struct Loop {
   template <int U>
   __device__ __forceinline__ static void gemm1(const JobParams& p, Ctx& cx, const uint8_t* slab0) {
     constexpr int N = S::n1(U);
-    const float* bias = reinterpret_cast<const float*>(slab0) + 2 * E;
+    const float* bias = reinterpret_cast<const float*>(slab0);
     float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.xln);
     T* hid = reinterpret_cast<T*>(cx.smem + p.sm.xln);
     if constexpr (BF) {
@@ -789,13 +787,13 @@ struct Loop {
       send_blocks(cx, ac, 0, ablk, cx.xg);
       exchange_wait(p, cx, cx.xg, cx.pg);
     }
-    // slab 0 of piece 1: [gamma | beta | first bias | second-GEMM bias slice | k-tiles]
+    // slab 0 of piece 1: [first bias | second-GEMM bias slice | k-tiles]
     const uint8_t* s1 = ring_acquire(p, cx);
     const float* hdr = reinterpret_cast<const float*>(s1);
     float b2[EPT];
 #pragma unroll
-    for (int k = 0; k < EPT; ++k) b2[k] = hdr[2 * E + S::n1(U) + ((cx.tid + k * NCT) & (Ec - 1))];
-    layernorm_rows(cx, ablk, reinterpret_cast<T*>(cx.smem + p.sm.xln), hdr, hdr + E);
+    for (int k = 0; k < EPT; ++k) b2[k] = hdr[S::n1(U) + ((cx.tid + k * NCT) & (Ec - 1))];
+    layernorm_rows(cx, ablk, reinterpret_cast<T*>(cx.smem + p.sm.xln));
     bar_compute();
     gemm1<U>(p, cx, s1);
     if constexpr (U == 1) cp_async_wait_all();
