@@ -107,6 +107,37 @@ struct Loop {
   __host__ __device__ static constexpr int att_keys() { return U == 0 ? H : 16; }
   template <int U>
   __host__ __device__ static constexpr int att_sample_elems() { return (H + att_keys<U>()) * LQ + att_keys<U>() * LV; }
+  // bf16 GEMMs: warps 0..NWG-1 take the n-tiles (warp w: tiles w, w + NWG, ...).
+  // Every warp loads the same A fragment, so NWG trades shared-memory traffic
+  // per k-tile (NWG x 512 B of A + NT x 256 B of B at 128 B/cycle) against the
+  // MMAs per SM sub-partition (warp w runs on w % 4, ~8 cycles per MMA).
+  __host__ __device__ static constexpr int gemm_cost(int NT, int nwg) {
+    const int smem = (nwg * 512 * MT + NT * 256) / 128;
+    int worst = 21;                                          // one dependent MMA
+    for (int s = 0; s < 4; ++s) {
+      int mm = 0;
+      for (int w = s; w < nwg; w += 4) mm += (NT > w ? (NT - w + nwg - 1) / nwg : 0) * MT;
+      worst = worst > 8 * mm ? worst : 8 * mm;
+    }
+    return smem > worst ? smem : worst;
+  }
+  // n-tiles per warp at most max(2, those of all NCW warps): accumulators and
+  // prefetched fragments fit the register file (9 warps per CTA, three share
+  // one sub-partition: at most 168 registers per thread)
+  __host__ __device__ static constexpr int gemm_warps_for(int NT) {
+    const int cap = (NT + NCW - 1) / NCW > 2 ? (NT + NCW - 1) / NCW : 2;
+    int best = NCW;
+    for (int w = NCW - 1; w >= 1; --w)
+      if ((NT + w - 1) / w <= cap && gemm_cost(NT, w) < gemm_cost(NT, best)) best = w;
+    return best;
+  }
+  // (the FFN's first GEMM keeps all warps: its GELU epilogue is per tile)
+  template <int U, int Q>
+  __host__ __device__ static constexpr int gemm_warps() {
+    return U == 2 && Q == 0 ? NCW : gemm_warps_for(S::pN(U, Q) / 8);
+  }
+  template <int U, int Q>
+  __host__ __device__ static constexpr int gemm_ntw() { return (S::pN(U, Q) / 8 + gemm_warps<U, Q>() - 1) / gemm_warps<U, Q>(); }
   static_assert(!MMA_ATT || S::G * att_sample_elems<0>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
   static_assert(!MMA_ATT || S::G * att_sample_elems<1>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
 
@@ -162,12 +193,14 @@ struct Loop {
   // CTA's slot in r's buffer, same offset in every CTA), counted on r's
   // barrier `rbar`; the C copies are issued by lanes of different warps.  The
   // writers of src have executed fence_proxy_async() and a bar_compute().
+  // (with src_stride > 0, CTA r gets src + r * src_stride bytes instead)
   __device__ __forceinline__ static void send_spread(Ctx& cx, const void* src, uint32_t bytes, const void* dst,
-                                                     uint64_t* rbar) {
+                                                     uint64_t* rbar, uint32_t src_stride = 0) {
     constexpr int PER = (C + NCW - 1) / NCW;
     const int r = cx.warp + NCW * cx.lane;
     if (cx.lane < PER && r < C)
-      bulk_s2c(mapa(smem_u32(dst), (uint32_t)r), src, bytes, mapa(smem_u32(rbar), (uint32_t)r));
+      bulk_s2c(mapa(smem_u32(dst), (uint32_t)r), reinterpret_cast<const uint8_t*>(src) + r * src_stride, bytes,
+               mapa(smem_u32(rbar), (uint32_t)r));
   }
 
   // ---------------------------------------------------------------- producer warp
@@ -254,7 +287,7 @@ struct Loop {
     return kt == S::pK(U, Q) / 16 - 1 || slab_first<U, Q>(kt + 1);
   }
 
-  // bf16: warp w owns n-tiles w, w+8, ... (NTW of them).  The A and B
+  // bf16: warp w < NWG owns n-tiles w, w + NWG, ... (NTW of them).  The A and B
   // fragments of k-tile kt + PD are loaded before the MMAs of k-tile kt, so
   // shared-memory latency overlaps the MMA chain; a slab is acquired when its
   // first k-tile is loaded and released after its last k-tile's MMAs.  With
@@ -262,13 +295,20 @@ struct Loop {
   // single k-tile (then PD = 1).
   template <int U, int Q>
   __device__ __forceinline__ static void gemm_bf16(const JobParams& p, Ctx& cx, const __nv_bfloat16* A, int lda,
-                                                   const uint8_t* slab0,
-                                                   float (&acc)[MT][(S::pN(U, Q) / 8 + NCW - 1) / NCW][4]) {
-    constexpr int NT = S::pN(U, Q) / 8, NTW = (NT + NCW - 1) / NCW;
+                                                   const uint8_t* slab0, float (&acc)[MT][gemm_ntw<U, Q>()][4]) {
+    constexpr int NT = S::pN(U, Q) / 8, NWG = gemm_warps<U, Q>(), NTW = gemm_ntw<U, Q>();
     constexpr int NKT = S::pK(U, Q) / 16, K0 = S::pK0(U, Q), KPS = S::pKps(U, Q);
     constexpr int HDR = S::pHdr(U, Q);
     constexpr int PD = (KPS >= 2 || NKT <= K0 + 1) ? 2 : 1, NB = PD + 1;
     static_assert(S::NSLOT >= 2, "prefetch holds two slabs");
+    if (NWG < NCW && cx.warp >= NWG) {                  // warps without tiles only pass the slabs on
+#pragma unroll
+      for (int kt = 0; kt < NKT; ++kt) {
+        if (slab_first<U, Q>(kt)) ring_acquire(p, cx);
+        if (slab_last<U, Q>(kt)) ring_release(cx);
+      }
+      return;
+    }
     const uint8_t* sl = slab0 + HDR + cx.lane * 8;
 #pragma unroll
     for (int m = 0; m < MT; ++m)
@@ -286,8 +326,8 @@ struct Loop {
       for (int m = 0; m < MT; ++m) ldmatrix_x4(af[kt % NB][m], arow + m * 16 * lda + kt * 16);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (NT % NCW == 0 || nt < NT) bf[kt % NB][i] = *reinterpret_cast<const uint2*>(sl + (kk * NT + nt) * 256);
+        const int nt = cx.warp + i * NWG;
+        if (NT % NWG == 0 || nt < NT) bf[kt % NB][i] = *reinterpret_cast<const uint2*>(sl + (kk * NT + nt) * 256);
       }
     };
 #pragma unroll
@@ -298,8 +338,8 @@ struct Loop {
       if (kt + PD < NKT) load(kt + PD);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (NT % NCW == 0 || nt < NT) {
+        const int nt = cx.warp + i * NWG;
+        if (NT % NWG == 0 || nt < NT) {
 #pragma unroll
           for (int m = 0; m < MT; ++m) mma_bf16(acc[m][i], af[kt % NB][m], bf[kt % NB][i]);
         }
@@ -412,21 +452,22 @@ struct Loop {
     float* g1 = reinterpret_cast<float*>(cx.smem + p.sm.xln);
     T* hid = reinterpret_cast<T*>(cx.smem + p.sm.xln);
     if constexpr (BF) {
-      constexpr int NT = N / 8, NTW = (NT + NCW - 1) / NCW;
+      constexpr int NT = N / 8, NWG = gemm_warps<U, 0>(), NTW = gemm_ntw<U, 0>();
       float2 bv[NTW];
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
-        const int nt = cx.warp + i * NCW;
-        bv[i] = (NT % NCW == 0 || nt < NT) ? *reinterpret_cast<const float2*>(bias + nt * 8 + 2 * (cx.lane & 3))
-                                            : make_float2(0.f, 0.f);
+        const int nt = cx.warp + i * NWG;
+        bv[i] = (cx.warp < NWG && (NT % NWG == 0 || nt < NT))
+                    ? *reinterpret_cast<const float2*>(bias + nt * 8 + 2 * (cx.lane & 3))
+                    : make_float2(0.f, 0.f);
       }
       float acc[MT][NTW][4];
       gemm_bf16<U, 0>(p, cx, reinterpret_cast<const __nv_bfloat16*>(cx.smem + p.sm.xln), S::lda, slab0, acc);
       bar_compute();
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (NT % NCW == 0 || nt < NT) {
+        const int nt = cx.warp + i * NWG;
+        if (cx.warp < NWG && (NT % NWG == 0 || nt < NT)) {
           const int n = nt * 8 + 2 * (cx.lane & 3);
 #pragma unroll
           for (int mt = 0; mt < MT; ++mt)
@@ -482,7 +523,8 @@ struct Loop {
 
   // ---------------------------------------------------------------- second GEMM
   // Partial sums over this CTA's K slice, staged in ablk in block layout
-  // (block r = columns r*Ec.. destined for CTA r).  Staging into ablk is safe
+  // (block r = columns r*Ec.. destined for CTA r; in bf16 mode as bf16 in the
+  // first half of the block).  Staging into ablk is safe
   // block by block: CTA r's next gather writes only block r of ablk, and r can
   // only send it after it has received this CTA's partial block r.
   template <int U>
@@ -491,22 +533,23 @@ struct Loop {
     constexpr int lda = U == 2 ? S::ldh : S::ldo;
     float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
     if constexpr (BF) {
-      constexpr int NT = E / 8, NTW = (NT + NCW - 1) / NCW;
+      constexpr int NT = E / 8, NWG = gemm_warps<U, 1>(), NTW = gemm_ntw<U, 1>();
       float acc[MT][NTW][4];
       gemm_bf16<U, 1>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, ring_acquire(p, cx), acc);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
-        const int nt = cx.warp + i * NCW;
-        if (NT % NCW == 0 || nt < NT) {
+        const int nt = cx.warp + i * NWG;
+        if (cx.warp < NWG && (NT % NWG == 0 || nt < NT)) {
           const int n = nt * 8 + 2 * (cx.lane & 3);
-          float* dst = stage + (n >> S::lEc) * S::blk + (n & (Ec - 1));
+          __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(stage + (n >> S::lEc) * S::blk) + (n & (Ec - 1));
 #pragma unroll
           for (int mt = 0; mt < MT; ++mt)
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
               const int m = mt * 16 + (cx.lane >> 2) + 8 * h;
               if (M % 16 == 0 || m < M)
-                *reinterpret_cast<float2*>(dst + (m << S::lEc)) = make_float2(acc[mt][i][2 * h], acc[mt][i][2 * h + 1]);
+                *reinterpret_cast<__nv_bfloat162*>(dst + (m << S::lEc)) =
+                    __floats2bfloat162_rn(acc[mt][i][2 * h], acc[mt][i][2 * h + 1]);
             }
         }
       }
@@ -803,14 +846,20 @@ struct Loop {
       bar_compute();
     }
     gemm2<U>(p, cx);
-    // exchange 2: block r of the staged partial sums goes to CTA r.  rs is read
-    // below; CTA r sends into it again only after this CTA's next gather.
+    // exchange 2: block r of the staged partial sums goes to CTA r (bf16 in
+    // bf16 mode).  rs is read below; CTA r sends into it again only after this
+    // CTA's next gather.
     fence_proxy_async();
     bar_compute();
-    send_blocks(cx, ablk, S::blk, reinterpret_cast<const float*>(cx.smem + p.sm.rs), cx.xr);
-    exchange_wait(p, cx, cx.xr, cx.pr);
-    // finish this CTA's columns: r = sum of partials + bias; c_b <- r; a += r
     const float* rs = reinterpret_cast<const float*>(cx.smem + p.sm.rs);
+    if constexpr (BF) {
+      send_spread(cx, ablk, (uint32_t)(MEc * 2), rs + cx.c * S::blk, cx.xr, (uint32_t)(S::blk * 4));
+      exchange_wait(p, cx, cx.xr, cx.pr, XBYTES / 2);
+    } else {
+      send_blocks(cx, ablk, S::blk, rs, cx.xr);
+      exchange_wait(p, cx, cx.xr, cx.pr);
+    }
+    // finish this CTA's columns: r = sum of partials + bias; c_b <- r; a += r
     T* cache = cache_ptr(p, cx, job, b);
 #pragma unroll
     for (int k = 0; k < EPT; ++k) {
@@ -818,7 +867,9 @@ struct Loop {
       if (MEc % NCT == 0 || e < MEc) {
         float part[C];
 #pragma unroll
-        for (int cc = 0; cc < C; ++cc) part[cc] = rs[cc * S::blk + e];
+        for (int cc = 0; cc < C; ++cc)
+          part[cc] = BF ? to_f<__nv_bfloat16>(reinterpret_cast<const __nv_bfloat16*>(rs + cc * S::blk)[e])
+                        : rs[cc * S::blk + e];
 #pragma unroll
         for (int w = C / 2; w > 0; w >>= 1)
 #pragma unroll
