@@ -799,8 +799,11 @@ struct Loop {
   }
 
   // ---------------------------------------------------------------- one refreshed unit (Eq. 1, (b,t) in S)
+  // bnext: the next refreshed unit of this step (U if none); the finish adds
+  // the cached outputs of b+1..bnext-1 and, when bnext < U, prepares its gather.
   template <int U>
-  __device__ __forceinline__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0) {
+  __device__ __forceinline__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0,
+                                              int bnext, uint64_t valid) {
     const int l = b / 3;
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
     float* ablk = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
@@ -814,12 +817,7 @@ struct Loop {
     // ablk is read by LayerNorm below; CTA r sends into it again only after
     // this CTA's partial sums (sent after the first GEMM) reached r.
     if constexpr (BF) {
-      __nv_bfloat16* acb = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb);
-#pragma unroll
-      for (int k = 0; k < EPT; ++k) {
-        const int e = cx.tid + k * NCT;
-        if (MEc % NCT == 0 || e < MEc) acb[e] = __float2bfloat16_rn(ac[e]);
-      }
+      __nv_bfloat16* acb = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb);   // written by the preceding pass
       fence_proxy_async();
       bar_compute();                   // ac final for this unit
       send_spread(cx, acb, (uint32_t)(MEc * 2), ablk + cx.c * S::blk, cx.xg);
@@ -876,50 +874,48 @@ struct Loop {
           for (int cc = 0; cc < w; ++cc) part[cc] += part[cc + w];
         const float r = part[0] + b2[k];
         cache[e] = from_f<T>(r);
-        ac[e] += r;
         if (p.trace) {
           const int m = e >> S::lEc, j = e & (Ec - 1);
           const int s = sample0 + (m >> S::lH);
           if (s < p.samples)
             p.trace[(((long long)t * p.U + b) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] = r;
         }
+        const float a = add_cached(p, cx, job, b + 1, bnext, t, sample0, valid, e, ac[e] + r);
+        ac[e] = a;
+        if (BF && bnext < p.U) reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb)[e] = __float2bfloat16_rn(a);
       }
     }
   }
 
-  // ---------------------------------------------------------------- skipped units b0..b1-1: a += c_b (in unit order)
-  __device__ __forceinline__ static void skip_run(const JobParams& p, Ctx& cx, int job, int b0, int b1, int t,
-                                                  int sample0, uint64_t valid) {
-    float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
-    // units of the run whose cache holds a value (bit k = unit b0 + k)
-    const uint32_t live = (uint32_t)((valid >> b0) & ((1ull << (b1 - b0)) - 1ull));
-    const T* cb = cache_ptr(p, cx, job, b0);
+  // ---------------------------------------------------------------- skipped units b0..b1-1 (Eq. 1: a += c_b)
+  // Element e of this CTA's columns: a + the cached outputs of the skipped
+  // units b0..b1-1 whose caches hold a value (valid), loaded eight at a time and
+  // summed pairwise before the add.  Runs inside the per-element pass that
+  // precedes them (the embedding or a refreshed unit's finish).
+  __device__ __forceinline__ static float add_cached(const JobParams& p, Ctx& cx, int job, int b0, int b1, int t,
+                                                     int sample0, uint64_t valid, int e, float a) {
+    if (b0 >= b1) return a;
+    const T* cb = cache_ptr(p, cx, job, 0);
     const int cstride = p.sm.cs >= 0 ? MEc : C * MEc;
+    for (int b = b0; b < b1; b += 8) {
+      const uint32_t live = (uint32_t)(valid >> b) & (b1 - b >= 8 ? 0xffu : (1u << (b1 - b)) - 1u);
+      float cv[8];
 #pragma unroll
-    for (int k = 0; k < EPT; ++k) {
-      const int e = cx.tid + k * NCT;
-      if (MEc % NCT == 0 || e < MEc) {
-        float cv[8];
+      for (int q = 0; q < 8; ++q) cv[q] = ((live >> q) & 1u) ? to_f<T>(cb[(b + q) * cstride + e]) : 0.f;
+      a += ((cv[0] + cv[1]) + (cv[2] + cv[3])) + ((cv[4] + cv[5]) + (cv[6] + cv[7]));
+      if (p.trace) {
+        const int m = e >> S::lEc, j = e & (Ec - 1);
+        const int s = sample0 + (m >> S::lH);
+        if (s < p.samples) {
 #pragma unroll
-        for (int q = 0; q < 8; ++q) cv[q] = ((live >> q) & 1u) ? to_f<T>(cb[q * cstride + e]) : 0.f;
-        float a = ac[e];
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          if ((live >> q) & 1u) a += cv[q];
-        ac[e] = a;
-        if (p.trace) {
-          const int m = e >> S::lEc, j = e & (Ec - 1);
-          const int s = sample0 + (m >> S::lH);
-          if (s < p.samples) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              if (b0 + q < b1)
-                p.trace[(((long long)t * p.U + b0 + q) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] =
-                    cv[q];
-          }
+          for (int q = 0; q < 8; ++q)
+            if (b + q < b1)
+              p.trace[(((long long)t * p.U + b + q) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] =
+                  cv[q];
         }
       }
     }
+    return a;
   }
 
   // ---------------------------------------------------------------- output head + sampler step
@@ -1085,7 +1081,9 @@ struct Loop {
             const int l = (__ffsll((long long)ca) - 1) / 3;
             stage_kv(p, cx, l, t, kvs + l * S::G * p.Cm * S::kvw);
           }
-        // input embedding into this CTA's columns
+        // input embedding into this CTA's columns, plus the cached outputs of the
+        // skipped units before the first refreshed one
+        int b = refresh ? __ffsll((long long)refresh) - 1 : p.U;
 #pragma unroll
         for (int k = 0; k < EPT; ++k) {
           const int e = cx.tid + k * NCT;
@@ -1093,26 +1091,21 @@ struct Loop {
             const int m = e >> S::lEc, j = e & (Ec - 1);
             float acc = 0.f;
             for (int a = 0; a < p.A; ++a) acc = fmaf(x[m * p.A + a], c_inw[a * Ec + j], acc);
-            ac[e] = acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j];
+            const float a = add_cached(p, cx, job, 0, b, t, sample0, valid, e, acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j]);
+            ac[e] = a;
+            if (BF && b < p.U) reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb)[e] = __float2bfloat16_rn(a);
           }
         }
-        // units in order: a refreshed unit, or a run of up to 8 skipped ones
-        int b = 0;
+        // refreshed units in order; each finish adds the skipped units up to the next one
         while (b < p.U) {
-          const uint64_t rest = refresh >> b;
-          if (rest & 1ull) {
-            valid |= 1ull << b;
-            const int u = b % 3;
-            if (u == 0) unit<0>(p, cx, job, b, t, sample0);
-            else if (u == 1) unit<1>(p, cx, job, b, t, sample0);
-            else unit<2>(p, cx, job, b, t, sample0);
-            ++b;
-          } else {
-            const int gap = rest ? __ffsll((long long)rest) - 1 : 64;
-            const int b1 = min(min(b + gap, p.U), b + 8);
-            skip_run(p, cx, job, b, b1, t, sample0, valid);
-            b = b1;
-          }
+          valid |= 1ull << b;
+          const uint64_t later = b + 1 < 64 ? refresh >> (b + 1) : 0ull;
+          const int bnext = later ? b + __ffsll((long long)later) : p.U;
+          const int u = b % 3;
+          if (u == 0) unit<0>(p, cx, job, b, t, sample0, bnext, valid);
+          else if (u == 1) unit<1>(p, cx, job, b, t, sample0, bnext, valid);
+          else unit<2>(p, cx, job, b, t, sample0, bnext, valid);
+          b = bnext;
         }
         head_step(p, cx, t);
       }
