@@ -288,9 +288,10 @@ struct Loop {
   }
 
   // bf16: warp w < NWG owns n-tiles w, w + NWG, ... (NTW of them).  The A and B
-  // fragments of k-tile kt + PD are loaded before the MMAs of k-tile kt, so
-  // shared-memory latency overlaps the MMA chain; a slab is acquired when its
-  // first k-tile is loaded and released after its last k-tile's MMAs.  With
+  // fragments of k-tile kt + PD are loaded right after the MMAs of k-tile kt,
+  // PD k-tiles ahead of their use, so shared-memory latency and slab waits
+  // overlap the MMA chain; a slab is acquired when its first k-tile is loaded
+  // and released after its last k-tile's MMAs.  With
   // PD = 2 a load window spans at most two slabs unless a middle slab holds a
   // single k-tile (then PD = 1).
   template <int U, int Q>
@@ -335,7 +336,6 @@ struct Loop {
       if (kt < NKT) load(kt);
 #pragma unroll
     for (int kt = 0; kt < NKT; ++kt) {
-      if (kt + PD < NKT) load(kt + PD);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
         const int nt = cx.warp + i * NWG;
@@ -345,6 +345,7 @@ struct Loop {
         }
       }
       if (slab_last<U, Q>(kt)) ring_release(cx);
+      if (kt + PD < NKT) load(kt + PD);          // after the MMAs: a slab wait overlaps them
     }
   }
 
@@ -528,14 +529,14 @@ struct Loop {
   // block by block: CTA r's next gather writes only block r of ablk, and r can
   // only send it after it has received this CTA's partial block r.
   template <int U>
-  __device__ __forceinline__ static void gemm2(const JobParams& p, Ctx& cx) {
+  __device__ __forceinline__ static void gemm2(const JobParams& p, Ctx& cx, const uint8_t* slab0) {
     const T* A = reinterpret_cast<const T*>(cx.smem + (U == 2 ? p.sm.xln : p.sm.oc));
     constexpr int lda = U == 2 ? S::ldh : S::ldo;
     float* stage = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
     if constexpr (BF) {
       constexpr int NT = E / 8, NWG = gemm_warps<U, 1>(), NTW = gemm_ntw<U, 1>();
       float acc[MT][NTW][4];
-      gemm_bf16<U, 1>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, ring_acquire(p, cx), acc);
+      gemm_bf16<U, 1>(p, cx, reinterpret_cast<const __nv_bfloat16*>(A), lda, slab0, acc);
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
         const int nt = cx.warp + i * NWG;
@@ -556,7 +557,7 @@ struct Loop {
     } else {
       constexpr int NOUT = M * E, NO = (NOUT + NCT - 1) / NCT;
       float acc[F32_MAXO];
-      gemm_f32<U, 1>(p, cx, reinterpret_cast<const float*>(A), lda, ring_acquire(p, cx), acc);
+      gemm_f32<U, 1>(p, cx, reinterpret_cast<const float*>(A), lda, slab0, acc);
 #pragma unroll
       for (int i = 0; i < NO; ++i) {
         const int o = cx.tid + i * NCT;
@@ -816,20 +817,23 @@ struct Loop {
     // in bf16 mode: they are only LayerNorm's input, whose output is bf16).
     // ablk is read by LayerNorm below; CTA r sends into it again only after
     // this CTA's partial sums (sent after the first GEMM) reached r.
+    // slab 0 of piece 1 ([first bias | second-GEMM bias slice | k-tiles]) is
+    // acquired while the exchange is in flight
+    const uint8_t* s1;
     if constexpr (BF) {
       __nv_bfloat16* acb = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb);   // written by the preceding pass
       fence_proxy_async();
       bar_compute();                   // ac final for this unit
       send_spread(cx, acb, (uint32_t)(MEc * 2), ablk + cx.c * S::blk, cx.xg);
+      s1 = ring_acquire(p, cx);
       exchange_wait(p, cx, cx.xg, cx.pg, XBYTES / 2);
     } else {
       fence_proxy_async();
       bar_compute();                   // ac final for this unit
       send_blocks(cx, ac, 0, ablk, cx.xg);
+      s1 = ring_acquire(p, cx);
       exchange_wait(p, cx, cx.xg, cx.pg);
     }
-    // slab 0 of piece 1: [first bias | second-GEMM bias slice | k-tiles]
-    const uint8_t* s1 = ring_acquire(p, cx);
     const float* hdr = reinterpret_cast<const float*>(s1);
     float b2[EPT];
 #pragma unroll
@@ -837,13 +841,14 @@ struct Loop {
     layernorm_rows(cx, ablk, reinterpret_cast<T*>(cx.smem + p.sm.xln));
     bar_compute();
     gemm1<U>(p, cx, s1);
+    const uint8_t* s2 = ring_acquire(p, cx);      // slab 0 of piece 2, held through the attention
     if constexpr (U == 1) cp_async_wait_all();
     bar_compute();
     if constexpr (U != 2) {
       attention<U>(p, cx, kvs);
       bar_compute();
     }
-    gemm2<U>(p, cx);
+    gemm2<U>(p, cx, s2);
     // exchange 2: block r of the staged partial sums goes to CTA r (bf16 in
     // bf16 mode).  rs is read below; CTA r sends into it again only after this
     // CTA's next gather.
@@ -971,13 +976,12 @@ struct Loop {
         }
       }
     }
+    cp_async_wait_all();                 // z_t (issued after the previous step's head)
     fence_proxy_async();
     bar_compute();
     // 2. all-gather: the block of M*npr floats to every CTA, issue spread over the warps
     send_spread(cx, ps, (uint32_t)(M * npr * 4), hb + cx.c * hstr, cx.xh + par);
     exchange_wait(p, cx, cx.xh + par, par ? cx.ph1 : cx.ph0, (uint32_t)(C * M * npr * 4));
-    cp_async_wait_all();
-    bar_compute();
     // 3. rows: half a warp per row; lane hl adds quantity hl (and hl + 16) over the partials
     const float4 tab0 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32);
     const float4 tab1 = *reinterpret_cast<const float4*>(cx.smem + p.sm.stb + t * 32 + 16);
@@ -1067,15 +1071,15 @@ struct Loop {
         }
       }
       const long long zstep = (long long)p.obs_mod * H * p.A;
+      if (zsrc) cp_async16(z + zdst, zsrc);                      // z_0
       const uint64_t units = p.U >= 64 ? ~0ull : (1ull << p.U) - 1ull;
       constexpr uint64_t CA_UNITS = 0x2492492492492492ull;     // bits 3l + 1: cross-attention units
       bar_compute();
       uint64_t valid = 0;
       for (int t = 0; t < p.T; ++t) {
         const uint64_t refresh = (sch[t] | (p.force ? ~valid : 0ull)) & units;
-        // stage z_t (DDPM) and, when every layer has a slot, the memory keys/values
-        // of this step's refreshed cross-attention units
-        if (zsrc) cp_async16(z + zdst, zsrc + t * zstep);
+        // when every layer has a slot, stage the memory keys/values of this
+        // step's refreshed cross-attention units
         if (p.kv_slots > 1)
           for (uint64_t ca = refresh & CA_UNITS; ca; ca &= ca - 1ull) {
             const int l = (__ffsll((long long)ca) - 1) / 3;
@@ -1108,6 +1112,8 @@ struct Loop {
           b = bnext;
         }
         head_step(p, cx, t);
+        // DDPM noise of the next step (every thread has read z_t: head_step ends with a barrier)
+        if (zsrc && t + 1 < p.T) cp_async16(z + zdst, zsrc + (t + 1) * zstep);
       }
       // write the finished chunk
       if (cx.c == 0) {
