@@ -140,7 +140,7 @@ def measured_peaks() -> dict:
 
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
-    for f in ("evo_loop.cuh", "evo_ptx.cuh", "evo_shapes.h", "evo_internal.h"):
+    for f in ("evo_loop.cuh", "evo_ptx.cuh", "evo_shapes.h", "evo_internal.h", "evo_job.cu", "evo_api.cu"):
         h.update(open(os.path.join(ROOT, "paper_2607_20293_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
