@@ -46,6 +46,8 @@ WORKLOADS = {
     "schedules": ("pusht", [1.0], 1.0, "bernoulli"),
     # schedule search with GPU population fitness (the paper's GA configuration)
     "search": ("pusht", [1.0], 1.0, "bernoulli"),
+    # 64 candidate lattices (Eq. 7 from a synthetic map, density 5-60 %) x 16 observations, one call
+    "population": ("population", [1.0], 1.0, "guided"),
 }
 REDUNDANCY_SAMPLES = 16          # all-refresh queries whose activations build the map
 FP32_LANES_PER_SM = 128          # GB300 SM: 4 x 32 FP32 lanes, one FMA (2 FLOPs) per lane per clock
@@ -417,6 +419,122 @@ def published_lattices(task: str):
     return bac, evo
 
 
+POP_MAP_SEED, POP_BUDGET_SEED, POP_RANDOM_SEED = 5, 6, 7
+POP_METRIC = "candidate action chunks/s (P x N per evo_denoise_population call, p50 call latency alongside)"
+
+
+def _oracle_pop_chunk(args):
+    """One (candidate, observation) chunk of the population workload on the oracle;
+    the candidate lattice is drawn with the oracle's own Eq. 7 sampler."""
+    p, seed = args
+    from oracle import evo_oracle as O
+    cfg = synth.config("population")
+    W = synth.make_weights(cfg, 0)
+    P, L, T = cfg["n_candidates"], cfg["n_layer"], cfg["n_steps"]
+    d = synth.dissimilarity_map(L, T, POP_MAP_SEED)
+    Ks = synth.population_budgets(P, L * T, POP_BUDGET_SEED)
+    rnd = synth.guided_randoms(P, int(Ks.max()), POP_RANDOM_SEED)
+    S = O.guided_sample(O.guided_weights(d, 0.05, 2), int(Ks[p % P]), rnd[p % P]).reshape(L, T)
+    O.denoise(W, cfg, synth.make_obs(cfg, 1, 1000 + seed), synth.make_noise(cfg, 1, 2000 + seed), S)
+    return 1
+
+
+def run_population(args, pool, workers):
+    """Population evaluation: P candidate lattices [P][L][T] drawn by the library's
+    Eq. 7 sampler from a synthetic dissimilarity map (densities 5-60 %), each on
+    N observations, plus the all-refresh reference, in one evo_denoise_population
+    call; dev_l2 per candidate.  value = candidate chunks (P x N) per second."""
+    import torch
+    from paper_2607_20293_gb300 import binding, build
+    build.build()
+    binding.load()
+    cfg = synth.config("population")
+    W = synth.make_weights(cfg, 0)
+    P, N, L, T = cfg["n_candidates"], cfg["batch"], cfg["n_layer"], cfg["n_steps"]
+    obs, noise = synth.make_obs(cfg, N, 1), synth.make_noise(cfg, N, 2)
+    d = torch.from_numpy(synth.dissimilarity_map(L, T, POP_MAP_SEED).astype(np.float32)).cuda()
+    Ks = synth.population_budgets(P, L * T, POP_BUDGET_SEED)
+    rnd = torch.from_numpy(synth.guided_randoms(P, int(Ks.max()), POP_RANDOM_SEED).view(np.int64)).cuda()
+    pop = torch.cat([binding.guided_schedules(d, int(Ks[p]), rnd[p:p + 1, :int(Ks[p])]) for p in range(P)])
+    ev = binding.Evo(cfg, W, (P + 1) * N)
+    d_obs, d_noise = torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda()
+    h_obs, h_noise = torch.from_numpy(obs).pin_memory(), torch.from_numpy(noise).pin_memory()
+    out = torch.empty((P, N, cfg["horizon"], cfg["action_dim"]), device="cuda")
+    dev = torch.empty((P,), device="cuda")
+    h_dev = torch.empty((P,)).pin_memory()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, device="cuda")
+    k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    k0.record()
+    k1.record()
+    ev.set_profile_events(k0, k1)
+
+    def one(e2e=False):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        if e2e:
+            d_obs.copy_(h_obs, non_blocking=True)
+            d_noise.copy_(h_noise, non_blocking=True)
+        ev.population(d_obs, d_noise, pop, out=out, dev=dev)
+        if e2e:
+            h_dev.copy_(dev, non_blocking=True)
+        b.record()
+        b.synchronize()
+        return a.elapsed_time(b), k0.elapsed_time(k1)
+
+    for _ in range(max(3, args.warmup)):
+        one()
+    clocks = Clocks(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks.start()
+    steps, kern, launches = [], [], 0
+    for _ in range(args.steps):
+        ms, kms = one()
+        steps.append(ms)
+        kern.append(kms)
+        launches += ev.last_call()["kernels"]
+    clk = clocks.stop()
+    e2e = [one(e2e=True)[0] for _ in range(args.steps)]
+    if ev.status() != binding.OK:
+        raise RuntimeError("device status reported an error")
+    S_host = pop.cpu().numpy()
+    flops = N * (sum(ev.flops(S_host[p]) for p in range(P)) + ev.flops(np.ones((L, T), np.uint8)))
+    full = N * (P + 1) * ev.flops(np.ones((L, T), np.uint8))
+    kern_ms = statistics.mean(kern)
+    peaks = measured_peaks()
+    peak = peaks.get("bf16_tflops", 1900.0)
+    achieved = flops / (kern_ms / 1000.0) / 1e12
+    line = {
+        "metric": POP_METRIC,
+        "value": P * N * 1000.0 / statistics.mean(steps), "unit": "chunks/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": statistics.mean(steps), "p50_ms": statistics.median(steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": cfg["dtype"],
+        "data": "synthetic (seeded weights, observations, noise; candidates by Eq. 7 from a synthetic map)",
+        "config": {"workload": f"population evaluation: {P} candidates x {N} observations + the all-refresh "
+                               f"reference, lattice {L} x {T}; {describe(cfg, N)}",
+                   "candidates": P, "observations": N, "density": [float(Ks.min()) / (L * T), float(Ks.max()) / (L * T)],
+                   "l2": "flushed between timed steps (256 MiB write)", "parallelism": "replicas x1"},
+        "flop_ratio_vs_all_full": full / flops,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                     "traffic": None, "peak_source": "measured bf16 burst" if "bf16_tflops" in peaks else "fallback",
+                     "kernel": ("batch-wide sequence (tcgen05 GEMMs + row/attention kernels)"
+                                if ev.last_call()["path"] == "wide" else "evo::job_kernel"),
+                     "algorithmic_per_launch": flops, "kernel_ms": kern_ms},
+        "e2e": {"value": P * N * 1000.0 / statistics.mean(e2e), "unit": "chunks/s",
+                "h2d_bytes_per_step": int(obs.nbytes + noise.nbytes), "d2h_bytes_per_step": int(h_dev.numel() * 4)},
+        "gpu_launches": launches, "clocks": clk, "launch": dict(ev.launch_info(), path=ev.last_call()["path"]),
+    }
+    if pool is not None:
+        pool.map(_oracle_pop_chunk, [(p, p) for p in range(workers)])          # warm the workers
+        n = workers * 2
+        t0 = time.perf_counter()
+        pool.map(_oracle_pop_chunk, [(3 * i, 100 + i) for i in range(n)])
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": n / dt, "unit": "chunks/s", "cores": workers, "kind": "oracle",
+                                "sample": f"{n} single (candidate, observation) chunks of the same population "
+                                          f"(candidates 0, 3, 6, ...), one float64 numpy oracle process per core"}
+    return line
+
+
 def run_schedules(args):
     """Push-T batch 1: chunks/s of the full lattice, EfficientVLA's fixed interval
     (M = 8, 10), the paper's BAC and EVO Push-T lattices and Bernoulli(0.125)."""
@@ -548,22 +666,43 @@ def main():
         if rank == 0:
             print(json.dumps(run_schedules(args)))
         return
+    if args.workload == "population" and args.impl == "ours":
+        if rank == 0:
+            pool = workers = None
+            if world == 1 and not args.no_cpu_baseline:
+                pool, workers = make_pool()          # spawned before the first GPU call
+            try:
+                print(json.dumps(run_population(args, pool, workers)))
+            finally:
+                if pool is not None:
+                    pool.close()
+        return
 
     if args.impl == "reference":
         if rank != 0:
             return
         pool, workers = make_pool()
+
+        def rnd(base):
+            if args.workload != "population":
+                return oracle_round(pool, name, head_frac, kind, workers, base_seed=base)
+            t0 = time.perf_counter()
+            pool.map(_oracle_pop_chunk, [(3 * (base + i), base + i) for i in range(workers)])
+            return time.perf_counter() - t0
+
         try:
             for _ in range(max(1, min(args.warmup, 3))):
-                oracle_round(pool, name, head_frac, kind, workers)
-            times = [oracle_round(pool, name, head_frac, kind, workers, base_seed=10 * i) for i in range(args.steps)]
+                rnd(0)
+            times = [rnd(10 * i) for i in range(args.steps)]
         finally:
             pool.close()
         total = sum(times)
         v = workers * args.steps / total
         cfg = synth.config(name)
         print(json.dumps({
-            "impl": "reference", "metric": "action chunks/s (p50 chunk latency and refresh-fraction sweep alongside)",
+            "impl": "reference",
+            "metric": POP_METRIC if args.workload == "population"
+            else "action chunks/s (p50 chunk latency and refresh-fraction sweep alongside)",
             "value": v, "unit": "chunks/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * total / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
