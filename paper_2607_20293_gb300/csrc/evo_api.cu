@@ -63,6 +63,18 @@ struct evo_handle {
   long long wide_rows = 1024;
   int last_path = 0;
   long long last_kernels = 0;
+  // Further cluster decompositions of the same model (automatic cluster size
+  // only): a smaller cluster is slower per job but more clusters run at once,
+  // so a call takes the decomposition with the fewest estimated job rounds.
+  struct Alt {
+    JobParams base{};
+    int shape = -1, max_clusters = 0;
+    uint8_t* wpack = nullptr;
+  };
+  Alt alt[2];
+  int n_alt = 0;
+  const JobParams* last_base = nullptr;   // decomposition of the last cluster launch
+  int last_mc = 0;
 };
 
 namespace {
@@ -385,10 +397,11 @@ evo_status evo_schedule_fixed_interval(int32_t n_units, int32_t T, int32_t M, ui
 evo_status evo_get_launch_info(const evo_handle* h, int32_t* cluster, int32_t* job_samples, int32_t* max_clusters,
                                int32_t* smem_bytes) {
   if (!h) return EVO_ERR_ARG;
-  if (cluster) *cluster = h->base.C;
-  if (job_samples) *job_samples = h->base.g;
-  if (max_clusters) *max_clusters = h->max_clusters;
-  if (smem_bytes) *smem_bytes = h->base.sm.total;
+  const JobParams& b = h->last_base ? *h->last_base : h->base;
+  if (cluster) *cluster = b.C;
+  if (job_samples) *job_samples = b.g;
+  if (max_clusters) *max_clusters = h->last_base ? h->last_mc : h->max_clusters;
+  if (smem_bytes) *smem_bytes = b.sm.total;
   return EVO_OK;
 }
 
@@ -398,6 +411,7 @@ evo_status evo_destroy(evo_handle* h) {
   cudaFree(h->wf32);
   cudaFree(h->woff_d);
   cudaFree(h->wpack);
+  for (int i = 0; i < h->n_alt; ++i) cudaFree(h->alt[i].wpack);
   cudaFree(h->vec);
   cudaFree(h->stab);
   cudaFree(h->kstep);
@@ -495,6 +509,9 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   auto W = [&](int id) { return weights + wo[id]; };
   auto WL = [&](int l, int id) { return weights + wo[W_LAYER0] + (size_t)l * wo[W_LAYER_STRIDE] + wo[id]; };
   const int es = h->es;
+  // packed weights of one decomposition (fills p.poff, p.layer_stride, p.cta_stride)
+  auto pack_for = [&](JobParams& p, uint8_t** dst) -> evo_status {
+  const int C = p.C;
   const int Ec = p.Ec, hid = p.hid;
   // piece sizes (bytes) and offsets within one layer block
   const long long sz[3][2] = {{p.hdr1[0] + (long long)E * p.n1[0] * es, (long long)p.kp_o * E * es},
@@ -575,9 +592,36 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
       put(base + p.poff[2][1], p.kp_h, E, [&](int k, int n) { return k < hid ? w2[(size_t)(c * hid + k) * E + n] : 0.f; });
     }
   }
-  if (cudaMalloc(&h->wpack, pack.size()) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMemcpy(h->wpack, pack.data(), pack.size(), cudaMemcpyHostToDevice) != cudaSuccess)
-    return fail(EVO_ERR_CUDA);
+  if (cudaMalloc(dst, pack.size()) != cudaSuccess) return EVO_ERR_OOM;
+  if (cudaMemcpy(*dst, pack.data(), pack.size(), cudaMemcpyHostToDevice) != cudaSuccess) return EVO_ERR_CUDA;
+  return EVO_OK;
+  };
+  {
+    const evo_status ps = pack_for(p, &h->wpack);
+    if (ps != EVO_OK) return fail(ps);
+  }
+  // smaller-cluster decompositions (automatic cluster size, one sample per job)
+  if (cfg->cluster == 0 && g == 1) {
+    for (int C2 = C / 2; C2 >= 4 && h->n_alt < 2; C2 /= 2) {
+      int slot2 = 0, nslot2 = 0;
+      if (!cluster_ok(cfg, C2)) continue;
+      const int sh = shape_find(cfg->dtype, E, cfg->n_head, H, C2, 1, &slot2, &nslot2);
+      if (sh < 0) continue;
+      evo_handle::Alt& a = h->alt[h->n_alt];
+      const int sm2 = plan(cfg, C2, 1, slot2, nslot2, smem_optin, a.base);
+      if (sm2 < 0) continue;
+      int mc = 0;
+      if (job_kernel_prepare(sh, sm2, &mc) != cudaSuccess || mc <= 0) {
+        cudaGetLastError();
+        continue;
+      }
+      a.shape = sh;
+      a.max_clusters = mc;
+      const evo_status ps = pack_for(a.base, &a.wpack);
+      ++h->n_alt;                                     // evo_destroy frees its weights
+      if (ps != EVO_OK) return fail(ps);
+    }
+  }
 
   // float32 vectors
   std::vector<float> vec;
@@ -655,6 +699,28 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
   p.vec = h->vec;
   p.cache = h->cache;
   p.status = h->status;
+  for (int i = 0; i < h->n_alt; ++i) {
+    JobParams& q = h->alt[i].base;
+    q.v_inw = p.v_inw;
+    q.v_inb = p.v_inb;
+    q.v_pos = p.v_pos;
+    q.v_lnfg = p.v_lnfg;
+    q.v_lnfb = p.v_lnfb;
+    q.v_headw = p.v_headw;
+    q.v_headb = p.v_headb;
+    q.v_headG = p.v_headG;
+    q.v_headB = p.v_headB;
+    q.stab = p.stab;
+    q.kv_time = p.kv_time;
+    q.kv_obs = p.kv_obs;
+    q.wpack = h->alt[i].wpack;
+    q.vec = p.vec;
+    q.cache = p.cache;
+    q.status = p.status;
+  }
+  // with a cluster of 4 at hand the cluster path stays ahead of the batch-wide
+  // one up to about 2048 action-token rows
+  if (cfg->wide_rows == 0 && h->n_alt > 0 && h->alt[h->n_alt - 1].base.C <= 4) h->wide_rows = 2048;
   *out = h;
   return EVO_OK;
 }
@@ -700,13 +766,42 @@ evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int row
 // kernels of the observation-condition path per call (embedding + three GEMVs)
 constexpr int COND_KERNELS = 4;
 
-cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, int shape = -1) {
+// The decomposition a cluster-path call of `samples` samples takes: the fewest
+// estimated job rounds, weighting a round of a smaller cluster by (C_max/C)^0.4
+// (per-job time measured at n_emb 256: 1.0 / 1.23 / 2.0 for C = 16 / 8 / 4 at
+// refresh fraction 0.125, 1.0 / 1.15 / 1.41 at 1.0).
+struct Pick {
+  const JobParams* base;
+  int shape, max_clusters;
+};
+
+Pick pick_decomposition(const evo_handle* h, long long samples) {
+  Pick best{&h->base, h->shape, h->max_clusters};
+  auto cost = [&](const JobParams& b, int mc) {
+    const long long jobs = (samples + b.g - 1) / b.g;
+    const long long rounds = (jobs + mc - 1) / mc;
+    return (double)rounds * std::pow((double)h->base.C / (double)b.C, 0.4);
+  };
+  double bc = cost(h->base, h->max_clusters);
+  for (int i = 0; i < h->n_alt; ++i) {
+    const double c = cost(h->alt[i].base, h->alt[i].max_clusters);
+    if (c < bc) {
+      bc = c;
+      best = {&h->alt[i].base, h->alt[i].shape, h->alt[i].max_clusters};
+    }
+  }
+  return best;
+}
+
+cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, const Pick& pk) {
   if (h->prof_start && h->prof_stop) {
     cudaError_t e = cudaEventRecord(h->prof_start, st);
     if (e != cudaSuccess) return e;
   }
-  cudaError_t e = launch_job(shape >= 0 ? shape : h->shape, p, std::min(p.n_jobs, h->max_clusters), st);
+  cudaError_t e = launch_job(pk.shape, p, std::min(p.n_jobs, pk.max_clusters), st);
   if (e != cudaSuccess) return e;
+  h->last_base = pk.base;
+  h->last_mc = pk.max_clusters;
   h->last_path = 0;
   h->last_kernels = COND_KERNELS + 1 + (p.sched_err ? 1 : 0);
   if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
@@ -787,7 +882,8 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   if (s != EVO_OK) return s;
   EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
                            h->cond_scratch, h->kv_obs, st));
-  JobParams p = h->base;
+  const Pick pk = pick_decomposition(h, N);
+  JobParams p = *pk.base;
   p.samples = N;
   p.per_sched = N;
   p.obs_mod = N;
@@ -799,7 +895,7 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   p.noise = noise;
   p.out = out;
   p.trace = trace;
-  EVO_CUDA(launch_loop(h, p, st));
+  EVO_CUDA(launch_loop(h, p, st, pk));
   return finish(h, st);
 }
 
@@ -868,7 +964,8 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
   if (s != EVO_OK) return s;
   EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
                            kv + kv_floats, kv, st));
-  JobParams p = h->base;
+  const Pick pk = pick_decomposition(h, N);
+  JobParams p = *pk.base;
   p.kv_obs = kv;
   p.samples = N;
   p.per_sched = N;
@@ -881,7 +978,7 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
   p.noise = noise;
   p.out = out_actions;
   p.trace = nullptr;
-  EVO_CUDA(launch_loop(h, p, st));
+  EVO_CUDA(launch_loop(h, p, st, pk));
   return finish(h, st);
 }
 
@@ -912,19 +1009,19 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   if (s != EVO_OK) return s;
   EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
                            h->cond_scratch, h->kv_obs, st));
-  JobParams p = h->base;
+  Pick pk = pick_decomposition(h, samples);
+  JobParams p = *pk.base;
   // samples of one job must share a schedule: g divides N_obs
-  int g = p.g, shape = h->shape;
+  int g = p.g;
   while (g > 1 && N_obs % g) g >>= 1;
   if (g != p.g) {
     // fewer samples per job: the compiled shape for g, with its own ring geometry
     int slot = 0, nslot = 0;
-    shape = shape_find(h->cfg.dtype, h->E, h->cfg.n_head, h->H, p.C, g, &slot, &nslot);
-    if (shape < 0) return EVO_ERR_UNSUPPORTED;
+    pk.shape = shape_find(h->cfg.dtype, h->E, h->cfg.n_head, h->H, p.C, g, &slot, &nslot);
+    if (pk.shape < 0) return EVO_ERR_UNSUPPORTED;
     const int smem = plan(&h->cfg, p.C, g, slot, nslot, h->smem_limit, p);
     if (smem < 0) return EVO_ERR_UNSUPPORTED;
-    int mc = 0;
-    EVO_CUDA(job_kernel_prepare(shape, smem, &mc));
+    EVO_CUDA(job_kernel_prepare(pk.shape, smem, &pk.max_clusters));
     p.stab = h->stab;
     p.kv_time = h->kv_time;
     p.kv_obs = h->kv_obs;
@@ -944,7 +1041,7 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   p.noise = noise;
   p.out = h->pop_x;
   p.trace = nullptr;
-  EVO_CUDA(launch_loop(h, p, st, shape));
+  EVO_CUDA(launch_loop(h, p, st, pk));
   EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
   h->last_kernels += 1;
   if (out_actions)

@@ -192,13 +192,29 @@ def test_handles_with_different_plans_coexist(torch, B):
 
 @pytest.mark.parametrize("path", ["wide", "cluster"])
 def test_manip_batch64_heterogeneous(torch, B, path):
-    cfg, W, obs, noise, ev, d_obs, d_noise = setup("manip", 64, torch, B, wide_rows=0 if path == "wide" else -1)
+    cfg, W, obs, noise, ev, d_obs, d_noise = setup("manip", 64, torch, B, wide_rows=1024 if path == "wide" else -1)
     S = synth.heterogeneous_schedule(24, 100, 4)
     got = ev.denoise(d_obs, d_noise, S).cpu().numpy()
     assert ev.last_call()["path"] == path
     idx = [0, 17, 63]
     check(got[idx], oracle_subset(W, cfg, obs, noise, S, idx), TOL["bf16"], "manip")
     assert np.all(np.isfinite(got)) and np.all(np.abs(got) <= 1.5)
+
+
+def test_automatic_decomposition_by_batch(torch, B):
+    # with the cluster size left to the library, one handle holds the 16-, 8- and
+    # 4-CTA decompositions and a call takes the one with the fewest job rounds
+    cfg = synth.config("manip")
+    W = synth.make_weights(cfg, 0)
+    ev = B.Evo(cfg, W, 64)
+    S = synth.heterogeneous_schedule(24, 100, 4)
+    for n, C, idx in [(1, 16, [0]), (8, 8, [0, 7]), (64, 4, [0, 33, 63])]:
+        obs, noise = synth.make_obs(cfg, n, 1), synth.make_noise(cfg, n, 2)
+        got = ev.denoise(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(), S).cpu().numpy()
+        assert ev.last_call()["path"] == "cluster"
+        assert ev.launch_info()["cluster"] == C, (n, ev.launch_info())
+        check(got[idx], oracle_subset(W, cfg, obs, noise, S, idx), TOL["bf16"], f"batch {n}")
+    assert ev.status() == B.OK
 
 
 @pytest.mark.parametrize("n,frac", [(256, 0.125), (1024, 1.0)])
