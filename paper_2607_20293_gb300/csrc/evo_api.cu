@@ -304,9 +304,8 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   if (g * p.Cm * (dh / 4 + p.Ec / 4) > NCT) return -1;     // one memory key/value chunk per thread
   if (es == 2 && p.Cm > 16) return -1;                      // tensor-core attention pads memory keys to 16
   if (p.A > 16) return -1;                                  // action dimensions of the fused head
-  // head partials per row segment of min(Ec, 32) columns: sum, sum of squares, A dots
-  p.npr = rup((2 + p.A) * (p.Ec > 32 ? p.Ec / 32 : 1), 4);
-  if (p.C * (p.Ec > 32 ? p.Ec / 32 : 1) > 16) return -1;   // partials a head row sums
+  // head partials per row: sum, sum of squares, A dots (4-padded)
+  p.npr = rup(2 + p.A, 4);
   if (es == 2) {
     if (p.Mp > 32) return -1;
   } else {

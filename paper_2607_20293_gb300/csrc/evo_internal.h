@@ -61,7 +61,7 @@ struct JobParams {
   int sampler, force;
   int nslot, slot_bytes;
   int head_sep;                   // 1: head partials double-buffered by step parity; 0: one buffer + cluster barrier
-  int npr;                        // floats per row of a head partial block: (2 + A) per row segment, 4-padded
+  int npr;                        // floats per row of a head partial block: 2 + A, 4-padded
   // samples
   int samples;                    // real samples in this launch
   int per_sched;                  // samples that share one schedule

@@ -140,6 +140,15 @@ struct Loop {
   __host__ __device__ static constexpr int gemm_ntw() { return (S::pN(U, Q) / 8 + gemm_warps<U, Q>() - 1) / gemm_warps<U, Q>(); }
   static_assert(!MMA_ATT || S::G * att_sample_elems<0>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
   static_assert(!MMA_ATT || S::G * att_sample_elems<1>() * 2 <= S::Mp * S::lda * S::ES, "attention staging fits");
+  // With tensor-core attention the q / k / v tiles are staged in ablk, which is
+  // free between LayerNorm (its last reader) and the second GEMM's staging, so
+  // the first GEMM's epilogue needs no barrier after its k-loop (xln, its A
+  // operand, is not overwritten).
+  static_assert(!MMA_ATT || S::G * att_sample_elems<0>() * 2 <= C * S::blk * 4, "attention staging fits in ablk");
+  static_assert(!MMA_ATT || S::G * att_sample_elems<1>() * 2 <= C * S::blk * 4, "attention staging fits in ablk");
+  __device__ __forceinline__ static uint8_t* att_stage(const JobParams& p, Ctx& cx) {
+    return cx.smem + (MMA_ATT ? p.sm.ablk : p.sm.xln);
+  }
 
   // ---------------------------------------------------------------- rings and barriers
   // wait for the next slab not yet acquired (cx.qa); slabs are released in
@@ -464,7 +473,7 @@ struct Loop {
       }
       float acc[MT][NTW][4];
       gemm_bf16<U, 0>(p, cx, reinterpret_cast<const __nv_bfloat16*>(cx.smem + p.sm.xln), S::lda, slab0, acc);
-      bar_compute();
+      if constexpr (!(MMA_ATT && U != 2)) bar_compute();     // the output aliases xln
 #pragma unroll
       for (int i = 0; i < NTW; ++i) {
         const int nt = cx.warp + i * NWG;
@@ -482,7 +491,7 @@ struct Loop {
                       __floats2bfloat162_rn(gelu_erf(v0), gelu_erf(v1));
                 } else if constexpr (MMA_ATT) {
                   // q -> Q[i], k -> K[i], v -> V[i] of sample m / H
-                  __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) +
+                  __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(att_stage(p, cx)) +
                                       (m >> S::lH) * att_sample_elems<U>();
                   const int i = m & (H - 1);
                   __nv_bfloat16* dst = n < dh       ? st + i * LQ + n
@@ -584,7 +593,7 @@ struct Loop {
     constexpr int NK = att_keys<U>(), NKT = NK / 8, MTH = H / 16;
     if (cx.warp >= S::G) return;
     const int sm_ = cx.warp, lane = cx.lane;
-    __nv_bfloat16* Q = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) + sm_ * att_sample_elems<U>();
+    __nv_bfloat16* Q = reinterpret_cast<__nv_bfloat16*>(att_stage(p, cx)) + sm_ * att_sample_elems<U>();
     __nv_bfloat16* K = Q + H * LQ;
     __nv_bfloat16* V = K + NK * LQ;
     const int g = lane >> 2, tq = lane & 3;
@@ -699,7 +708,7 @@ struct Loop {
     constexpr int NK = att_keys<1>(), PK = NK * (dh / 2), PS = NK * ((dh + Ec) / 2);
     for (int c = cx.tid; c < S::G * PS; c += NCT) {
       const int s_ = c / PS, r = c - s_ * PS;
-      __nv_bfloat16* K = reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.xln) + s_ * att_sample_elems<1>() + H * LQ;
+      __nv_bfloat16* K = reinterpret_cast<__nv_bfloat16*>(att_stage(p, cx)) + s_ * att_sample_elems<1>() + H * LQ;
       const float* kv = kvs + s_ * p.Cm * S::kvw;
       const bool isk = r < PK;
       const int j = isk ? r / (dh / 2) : (r - PK) / (Ec / 2);
@@ -933,9 +942,6 @@ struct Loop {
   // Without head_sep the blocks land in ablk at c*blk: block c of CTA r last
   // held r's second-GEMM partials for this CTA, which this CTA has received.
   __device__ __forceinline__ static void head_step(const JobParams& p, Ctx& cx, int t) {
-    constexpr int L = Ec < 32 ? Ec : 32;             // lanes holding one row segment of this CTA's columns
-    constexpr int SEG = Ec / L;                      // segments per row
-    static_assert(C * SEG <= 16, "head: at most 16 partials per row");
     const float* ac = reinterpret_cast<const float*>(cx.smem + p.sm.ac);
     float* x = reinterpret_cast<float*>(cx.smem + p.sm.x);
     const float* z = reinterpret_cast<const float*>(cx.smem + p.sm.z);
@@ -949,31 +955,50 @@ struct Loop {
     float* ps = reinterpret_cast<float*>(cx.smem + p.sm.hsrc) + par * M * npr;
     const int hstr = p.head_sep ? M * npr : S::blk;   // landing stride between the C blocks
     const float* hb = reinterpret_cast<const float*>(cx.smem + p.sm.hblk) + par * C * M * npr;
-    // 1. this CTA's partials (MEc is a multiple of 64: the guard is warp-uniform)
+    // 1. this CTA's partials.  Up to 16 columns: one element per thread, reduced
+    //    over the Ec lanes of its row with shuffles; more columns: thread
+    //    o < M * NP takes quantity q of row m as one dot product over the
+    //    columns (a . 1, a . a, a . gw[q - 2]).  (Measured: the first is faster
+    //    on 16 columns, the second on 64.)
+    if constexpr (Ec <= 16) {
 #pragma unroll
-    for (int k = 0; k < EPT; ++k) {
-      const int e = cx.tid + k * NCT;
-      if (MEc % NCT == 0 || e < MEc) {
-        const int m = e >> S::lEc, j = e & (Ec - 1);
-        const bool lead = (j & (L - 1)) == 0;
-        float* dst = ps + m * npr + (j / L) * NP;
-        const float v = ac[e];
-        float s0 = v, s1 = v * v;
+      for (int k = 0; k < EPT; ++k) {
+        const int e = cx.tid + k * NCT;
+        if (MEc % NCT == 0 || e < MEc) {         // MEc is a multiple of 64: warp-uniform
+          const int m = e >> S::lEc, j = e & (Ec - 1);
+          const bool lead = j == 0;
+          float* dst = ps + m * npr;
+          const float v = ac[e];
+          float s0 = v, s1 = v * v;
 #pragma unroll
-        for (int o = L / 2; o > 0; o >>= 1) {
-          s0 += __shfl_xor_sync(0xffffffffu, s0, o);
-          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-        }
-        if (lead) {
-          dst[0] = s0;
-          dst[1] = s1;
-        }
-        for (int a = 0; a < p.A; ++a) {
-          float d = v * gw[a * Ec + j];
+          for (int o = Ec / 2; o > 0; o >>= 1) {
+            s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+            s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+          }
+          if (lead) {
+            dst[0] = s0;
+            dst[1] = s1;
+          }
+          for (int a = 0; a < p.A; ++a) {
+            float d = v * gw[a * Ec + j];
 #pragma unroll
-          for (int o = L / 2; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-          if (lead) dst[2 + a] = d;
+            for (int o = Ec / 2; o > 0; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+            if (lead) dst[2 + a] = d;
+          }
         }
+      }
+    } else {
+      for (int o = cx.tid; o < M * NP; o += NCT) {
+        const int m = o / NP, q = o - m * NP;
+        const float* arow = ac + m * Ec;
+        const float* wrow = gw + (q >= 2 ? q - 2 : 0) * Ec;
+        float acc = 0.f;
+#pragma unroll
+        for (int j = 0; j < Ec; ++j) {
+          const float a = arow[j];
+          acc = fmaf(a, q == 0 ? 1.f : (q == 1 ? a : wrow[j]), acc);
+        }
+        ps[m * npr + q] = acc;
       }
     }
     cp_async_wait_all();                 // z_t (issued after the previous step's head)
@@ -993,14 +1018,31 @@ struct Loop {
       if (M % (2 * NCW) == 0 || m0 + cx.warp * 2 < M) {
         const int m = m0 + cx.warp * 2 + half;
         float t0 = 0.f, t1 = 0.f;
+        if constexpr (Ec <= 16) {                 // (measured faster on 16 partials)
 #pragma unroll
-        for (int r = 0; r < C; ++r)
-#pragma unroll
-          for (int sg = 0; sg < SEG; ++sg) {
-            const float* src = hb + r * hstr + m * npr + sg * NP;
+          for (int r = 0; r < C; ++r) {
+            const float* src = hb + r * hstr + m * npr;
             if (hl < NP) t0 += src[hl];
             if (hl + 16 < NP) t1 += src[hl + 16];
           }
+        } else {
+          float v0[C], v1[C];
+#pragma unroll
+          for (int r = 0; r < C; ++r) {
+            const float* src = hb + r * hstr + m * npr;
+            v0[r] = hl < NP ? src[hl] : 0.f;
+            v1[r] = hl + 16 < NP ? src[hl + 16] : 0.f;
+          }
+#pragma unroll
+          for (int w = C / 2; w > 0; w >>= 1)
+#pragma unroll
+            for (int r = 0; r < w; ++r) {
+              v0[r] += v0[r + w];
+              v1[r] += v1[r + w];
+            }
+          t0 = v0[0];
+          t1 = v1[0];
+        }
         const float S0 = __shfl_sync(0xffffffffu, t0, 0, 16);
         const float S1 = __shfl_sync(0xffffffffu, t0, 1, 16);
         const int qd = 2 + hl;
