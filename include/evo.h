@@ -69,7 +69,9 @@ typedef struct evo_config {
   int32_t sampler;      /* EVO_SAMPLER_* */
   int32_t dtype;        /* EVO_DTYPE_*: arithmetic/storage type of weights, GEMM operands and caches */
   int32_t empty_cache;  /* EVO_EMPTY_* */
-  int32_t cluster;      /* CTAs that cooperate on one job; 0 = choose */
+  int32_t cluster;      /* CTAs that cooperate on one job; 0 = choose per call: the handle packs every
+                           compiled decomposition of the model (16, 8, 4 CTAs) and a call takes the one
+                           with the fewest estimated rounds of jobs for its batch */
   int32_t job_samples;  /* samples per job (rows = job_samples * horizon); 0 = choose */
   int32_t debug_sync;   /* 1: synchronize after each call and return the device status */
   int32_t wide_rows;    /* batch-wide tensor-core path for calls of at least this many action-token
