@@ -44,6 +44,11 @@ struct evo_handle {
   float* kv_time = nullptr;
   float* kv_obs = nullptr;
   float* cond_scratch = nullptr;   // 6E floats per condition token
+  // condition path of small calls (bf16 models): bf16 weight copy, k|v bias, partial sums, counters
+  __nv_bfloat16* cond_w16 = nullptr;
+  float* cond_bkv = nullptr;
+  float* cond_part = nullptr;
+  unsigned* cond_count = nullptr;
   void* cache = nullptr;
   uint8_t* sched = nullptr;
   size_t sched_cap = 0;
@@ -63,6 +68,7 @@ struct evo_handle {
   long long wide_rows = 1024;
   int last_path = 0;
   long long last_kernels = 0;
+  int last_cond_kernels = 4;          // kernels of the last call's condition path
   // Further cluster decompositions of the same model (automatic cluster size
   // only): a smaller cluster is slower per job but more clusters run at once,
   // so a call takes the decomposition with the fewest estimated job rounds.
@@ -417,6 +423,10 @@ evo_status evo_destroy(evo_handle* h) {
   cudaFree(h->kv_time);
   cudaFree(h->kv_obs);
   cudaFree(h->cond_scratch);
+  cudaFree(h->cond_w16);
+  cudaFree(h->cond_bkv);
+  cudaFree(h->cond_part);
+  cudaFree(h->cond_count);
   cudaFree(h->cache);
   cudaFree(h->sched);
   cudaFree(h->status);
@@ -675,6 +685,29 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
     return fail(EVO_ERR_CUDA);
 
   if (cudaMalloc(&h->kv_obs, cap_samples * cfg->n_obs * L * 2 * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (es == 2 && cond_fast_ok(E, L, 1)) {
+    // bf16 copy of the condition matmuls for calls of a few tokens
+    std::vector<uint16_t> w16((size_t)8 * E * E + (size_t)E * L * 2 * E);
+    std::vector<float> bkv((size_t)L * 2 * E);
+    const float* w1 = W(W_CM_W1);
+    const float* w2 = W(W_CM_W2);
+    for (size_t i = 0; i < (size_t)4 * E * E; ++i) w16[i] = f2bf(w1[i]);
+    for (size_t i = 0; i < (size_t)4 * E * E; ++i) w16[(size_t)4 * E * E + i] = f2bf(w2[i]);
+    uint16_t* wkv = w16.data() + (size_t)8 * E * E;
+    for (int l = 0; l < L; ++l) {
+      const float* src = WL(l, WL_CA_WKV);
+      for (int k = 0; k < E; ++k)
+        for (int j = 0; j < 2 * E; ++j) wkv[(size_t)k * L * 2 * E + (size_t)l * 2 * E + j] = f2bf(src[(size_t)k * 2 * E + j]);
+      std::memcpy(&bkv[(size_t)l * 2 * E], WL(l, WL_CA_BKV), (size_t)2 * E * 4);
+    }
+    if (cudaMalloc(&h->cond_w16, w16.size() * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMalloc(&h->cond_bkv, bkv.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMalloc(&h->cond_part, cond_fast_part_floats(E, L, 32) * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMalloc(&h->cond_count, 768 * sizeof(unsigned)) != cudaSuccess) return fail(EVO_ERR_OOM);
+    cudaMemcpy(h->cond_w16, w16.data(), w16.size() * 2, cudaMemcpyHostToDevice);
+    cudaMemcpy(h->cond_bkv, bkv.data(), bkv.size() * 4, cudaMemcpyHostToDevice);
+    cudaMemset(h->cond_count, 0, 768 * sizeof(unsigned));
+  }
   if (cudaMalloc(&h->cache, cap_samples * H * (size_t)U * E * es) != cudaSuccess) return fail(EVO_ERR_OOM);
   h->sched_cap = cap_samples * U * T;
   if (cudaMalloc(&h->sched, h->sched_cap) != cudaSuccess) return fail(EVO_ERR_OOM);
@@ -728,6 +761,19 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
 
 namespace {
 
+// The observation tokens' keys/values of a call: the spread-out bf16 kernels
+// for a few tokens, else the general ones.
+cudaError_t obs_cond(evo_handle* h, const float* obs, int N, float* scratch, float* kv_obs, cudaStream_t st) {
+  h->last_cond_kernels = 4;
+  if (h->cond_w16 && cond_fast_ok(h->E, h->L, (long long)N * h->cfg.n_obs)) {
+    h->last_cond_kernels = 3;
+    return launch_obs_cond_fast(h->wf32, h->woff, h->cond_w16, h->cond_bkv, obs, N, h->cfg.n_obs, h->cfg.obs_dim,
+                                h->L, h->E, scratch, h->cond_part, h->cond_count, kv_obs, st);
+  }
+  return launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E, scratch,
+                         kv_obs, st);
+}
+
 // Copy n_sched lattices (+ optionally an all-ones reference lattice) into the
 // handle's device buffer.  Host lattices are validated here; device lattices
 // are checked by a kernel that sets status[1].
@@ -762,8 +808,6 @@ evo_status stage_schedules(evo_handle* h, const uint8_t* S, int n_sched, int row
   return EVO_OK;
 }
 
-// kernels of the observation-condition path per call (embedding + three GEMVs)
-constexpr int COND_KERNELS = 4;
 
 // The decomposition a cluster-path call of `samples` samples takes: the fewest
 // estimated job rounds, weighting a round of a smaller cluster by (C_max/C)^0.4
@@ -802,7 +846,7 @@ cudaError_t launch_loop(evo_handle* h, const JobParams& p, cudaStream_t st, cons
   h->last_base = pk.base;
   h->last_mc = pk.max_clusters;
   h->last_path = 0;
-  h->last_kernels = COND_KERNELS + 1 + (p.sched_err ? 1 : 0);
+  h->last_kernels = h->last_cond_kernels + 1 + (p.sched_err ? 1 : 0);
   if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
   return cudaSuccess;
 }
@@ -853,7 +897,7 @@ cudaError_t launch_wide(evo_handle* h, const float* noise, float* out, int sampl
   const cudaError_t e = wide_run(h->wide, c);
   if (e != cudaSuccess) return e;
   h->last_path = 1;
-  h->last_kernels = COND_KERNELS + wide_last_launches(h->wide);
+  h->last_kernels = h->last_cond_kernels + wide_last_launches(h->wide);
   if (h->prof_start && h->prof_stop) return cudaEventRecord(h->prof_stop, st);
   return cudaSuccess;
 }
@@ -871,16 +915,14 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   if (!trace && use_wide(h, N)) {
     const evo_status s = stage_wide(h, S, 1, S_rows, false, st);
     if (s != EVO_OK) return s;
-    EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
-                             h->cond_scratch, h->kv_obs, st));
+    EVO_CUDA(obs_cond(h, obs, N, h->cond_scratch, h->kv_obs, st));
     EVO_CUDA(launch_wide(h, noise, out, N, N, 1, S_rows, st));
     return finish(h, st);
   }
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
-                           h->cond_scratch, h->kv_obs, st));
+  EVO_CUDA(obs_cond(h, obs, N, h->cond_scratch, h->kv_obs, st));
   const Pick pk = pick_decomposition(h, N);
   JobParams p = *pk.base;
   p.samples = N;
@@ -961,8 +1003,7 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S, 1, S_rows, false, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
-                           kv + kv_floats, kv, st));
+  EVO_CUDA(obs_cond(h, obs, N, kv + kv_floats, kv, st));
   const Pick pk = pick_decomposition(h, N);
   JobParams p = *pk.base;
   p.kv_obs = kv;
@@ -994,8 +1035,7 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   if (use_wide(h, samples)) {
     const evo_status s = stage_wide(h, S_pop, P, S_rows, true, st);
     if (s != EVO_OK) return s;
-    EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
-                             h->cond_scratch, h->kv_obs, st));
+    EVO_CUDA(obs_cond(h, obs, N_obs, h->cond_scratch, h->kv_obs, st));
     EVO_CUDA(launch_wide(h, noise, h->pop_x, (int)samples, N_obs, P + 1, S_rows, st));
     EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
     h->last_kernels += 1;
@@ -1006,8 +1046,7 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   const int* err = nullptr;
   evo_status s = stage_schedules(h, S_pop, P, S_rows, true, st, &err);
   if (s != EVO_OK) return s;
-  EVO_CUDA(launch_obs_cond(h->wf32, h->woff_d, h->woff, obs, N_obs, h->cfg.n_obs, h->cfg.obs_dim, h->L, h->E,
-                           h->cond_scratch, h->kv_obs, st));
+  EVO_CUDA(obs_cond(h, obs, N_obs, h->cond_scratch, h->kv_obs, st));
   Pick pk = pick_decomposition(h, samples);
   JobParams p = *pk.base;
   // samples of one job must share a schedule: g divides N_obs

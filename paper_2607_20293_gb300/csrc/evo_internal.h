@@ -103,6 +103,14 @@ cudaError_t launch_job(int shape, const JobParams& p, int n_clusters, cudaStream
 // condition path; scratch holds 6E floats per token
 cudaError_t launch_time_table(const float* wf32, const int* woff_dev, const int* woff, const float* kstep, int T,
                               int L, int E, float* scratch, float* kv_time, cudaStream_t s);
+// condition path for at most 32 tokens of a bf16 model (cond_fast_ok): bf16 weight copy w16 =
+// [E][4E] | [4E][E] | [E][L*2E] (row k holds every layer's [k | v] columns), bkv = [L*2E],
+// part = cond_fast_part_floats floats, count = 768 zeroed counters (reset by the kernels)
+bool cond_fast_ok(int E, int L, long long ntok);
+size_t cond_fast_part_floats(int E, int L, long long ntok);
+cudaError_t launch_obs_cond_fast(const float* wf32, const int* woff, const __nv_bfloat16* w16, const float* bkv,
+                                 const float* obs, int N, int n_obs, int D, int L, int E, float* scratch,
+                                 float* part, unsigned* count, float* kv_obs, cudaStream_t s);
 cudaError_t launch_obs_cond(const float* wf32, const int* woff_dev, const int* woff, const float* obs, int N,
                             int n_obs, int D, int L, int E, float* scratch, float* kv_obs, cudaStream_t s);
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s);

@@ -3,6 +3,8 @@
 // shared-memory plan of the loop kernel and the dispatch over its compiled
 // shapes (the loop kernel itself is in evo_loop.cuh).
 
+#include <algorithm>
+
 #include "evo_ptx.cuh"
 #include "evo_shapes.h"
 
@@ -113,6 +115,176 @@ static cudaError_t cond_tokens_to_kv(const float* w, const int* wo_dev, const in
       Md, ntok, E, L * 2 * E, w + wo[W_LAYER0] + wo[WL_CA_WKV], wo[W_LAYER_STRIDE], 2 * E, 2 * E,
       w + wo[W_LAYER0] + wo[WL_CA_BKV], wo[W_LAYER_STRIDE], kv, 0);
   (void)wo_dev;
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// condition path for a few tokens (bf16 models): every weight byte is read once
+// per call, so the three matmuls are spread over many blocks.  Block (g, kb, z)
+// takes columns g*256 .. +256 and rows kb*CK .. +CK of W (bf16, [K][N]) for the
+// tokens z*8 .. +8; warp w takes rows kb*CK + w, + 8, ..., lane l columns
+// 8l .. 8l+7 (one 16-byte load per row).  The block's partial sums go to
+// part[z][kb][t][N]; the last block of a column group (a counter, reset by that
+// block) adds the KB partials in order, adds the bias, applies the activation
+// and writes Y.  Stage 0 builds its input rows itself: the observation token
+// embedding obs W_obs + b_obs + cond_pos[1 + j].
+// ---------------------------------------------------------------------------
+
+constexpr int CG_COLS = 256, CG_TOK = 8, CG_ROWS = 16;   // columns per block, tokens per block, rows per block
+
+struct CondGemv {
+  const float* X;            // [ntok][K] (stage 0: null, obs below)
+  const float* obs;          // stage 0: [ntok][D]
+  const float* w_obs;        // stage 0: [D][K] fp32, + b_obs [K], cond_pos [1 + n_obs][K]
+  const float* b_obs;
+  const float* pos;
+  int D, n_obs;
+  int ntok, K, N;
+  const __nv_bfloat16* W;    // [K][N]
+  const float* bias;         // [N]
+  float* Y;                  // [ntok][N]
+  float* part;               // [ceil(ntok/8)][K/16][8][N]
+  unsigned* count;           // [ceil(ntok/8)][N/256]
+  int act;                   // 1 = Mish
+};
+
+__global__ void __launch_bounds__(256) cond_gemv_kernel(const CondGemv a) {
+  __shared__ float xs[CG_TOK][CG_ROWS];
+  __shared__ __align__(16) float red[8][CG_COLS];
+  __shared__ int last;
+  const int g = blockIdx.x, kb = blockIdx.y, z = blockIdx.z, KB = gridDim.y;
+  const int t0 = z * CG_TOK, nt = min(CG_TOK, a.ntok - t0), k0 = kb * CG_ROWS;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid < CG_TOK * CG_ROWS) {
+    const int t = tid / CG_ROWS, r = tid % CG_ROWS, k = k0 + r;
+    float v = 0.f;
+    if (t < nt) {
+      if (a.X) {
+        v = a.X[(long long)(t0 + t) * a.K + k];
+      } else {
+        const float* o = a.obs + (long long)(t0 + t) * a.D;
+        for (int d = 0; d < a.D; ++d) v = fmaf(o[d], a.w_obs[(long long)d * a.K + k], v);
+        v += a.b_obs[k] + a.pos[(1 + (t0 + t) % a.n_obs) * a.K + k];
+      }
+    }
+    xs[t][r] = v;
+  }
+  __syncthreads();
+  float acc[CG_TOK][8];
+#pragma unroll
+  for (int t = 0; t < CG_TOK; ++t)
+#pragma unroll
+    for (int c = 0; c < 8; ++c) acc[t][c] = 0.f;
+  const __nv_bfloat16* wp = a.W + (long long)k0 * a.N + g * CG_COLS + lane * 8;
+#pragma unroll
+  for (int r = warp; r < CG_ROWS; r += 8) {
+    const uint4 raw = __ldg(reinterpret_cast<const uint4*>(wp + (long long)r * a.N));
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&raw);
+    float w[8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = __bfloat1622float2(h[q]);
+      w[2 * q] = f.x;
+      w[2 * q + 1] = f.y;
+    }
+#pragma unroll
+    for (int t = 0; t < CG_TOK; ++t) {
+      const float xv = xs[t][r];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) acc[t][c] = fmaf(xv, w[c], acc[t][c]);
+    }
+  }
+  // the block's partial of column tid, token by token: the 8 warps in order
+  float* part = a.part + ((long long)z * KB + kb) * CG_TOK * a.N;
+  const int n = g * CG_COLS + tid;
+#pragma unroll
+  for (int t = 0; t < CG_TOK; ++t) {
+    if (t < nt) {                                   // block-uniform
+      float4* dst = reinterpret_cast<float4*>(&red[warp][lane * 8]);
+      dst[0] = make_float4(acc[t][0], acc[t][1], acc[t][2], acc[t][3]);
+      dst[1] = make_float4(acc[t][4], acc[t][5], acc[t][6], acc[t][7]);
+      __syncthreads();
+      float sum = 0.f;
+#pragma unroll
+      for (int w = 0; w < 8; ++w) sum += red[w][tid];
+      part[(long long)t * a.N + n] = sum;
+      __syncthreads();
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) {
+    unsigned* cnt = a.count + z * gridDim.x + g;
+    last = atomicAdd(cnt, 1u) == (unsigned)(KB - 1);
+    if (last) *cnt = 0u;                   // ready for the next launch (stream-ordered)
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  const float* p0 = a.part + (long long)z * KB * CG_TOK * a.N;
+  for (int t = 0; t < nt; ++t) {
+    float v = a.bias[n];
+    for (int b = 0; b < KB; ++b) v += __ldcg(p0 + ((long long)b * CG_TOK + t) * a.N + n);
+    if (a.act) v = mish(v);
+    a.Y[(long long)(t0 + t) * a.N + n] = v;
+  }
+}
+
+bool cond_fast_ok(int E, int L, long long ntok) {
+  return E % CG_COLS == 0 && E % CG_ROWS == 0 && ntok <= 4 * CG_TOK && L * 2 * E % CG_COLS == 0;
+}
+
+size_t cond_fast_part_floats(int E, int L, long long ntok) {
+  const long long zb = (ntok + CG_TOK - 1) / CG_TOK;
+  const long long a = (long long)(4 * E / CG_ROWS) * E, b = (long long)(E / CG_ROWS) * L * 2 * E;
+  return (size_t)(zb * CG_TOK * std::max(std::max(a, (long long)(E / CG_ROWS) * 4 * E), b));
+}
+
+// w16: [E][4E] | [4E][E] | [E][L*2E] bf16; bkv: [L*2E] fp32; scratch: 5E floats per token
+cudaError_t launch_obs_cond_fast(const float* w, const int* wo, const __nv_bfloat16* w16, const float* bkv,
+                                 const float* obs, int N, int n_obs, int D, int L, int E, float* scratch,
+                                 float* part, unsigned* count, float* kv_obs, cudaStream_t s) {
+  const int ntok = N * n_obs, zb = (ntok + CG_TOK - 1) / CG_TOK;
+  float* Hd = scratch;                          // [ntok][4E]
+  float* Md = scratch + (size_t)ntok * 4 * E;   // [ntok][E]
+  CondGemv a{};
+  a.ntok = ntok;
+  a.part = part;
+  a.count = count;
+  // stage 0: embedding + E -> 4E, Mish
+  a.X = nullptr;
+  a.obs = obs;
+  a.w_obs = w + wo[W_OBS_W];
+  a.b_obs = w + wo[W_OBS_B];
+  a.pos = w + wo[W_COND_POS];
+  a.D = D;
+  a.n_obs = n_obs;
+  a.K = E;
+  a.N = 4 * E;
+  a.W = w16;
+  a.bias = w + wo[W_CM_B1];
+  a.Y = Hd;
+  a.act = 1;
+  cond_gemv_kernel<<<dim3(a.N / CG_COLS, a.K / CG_ROWS, zb), 256, 0, s>>>(a);
+  // 4E -> E
+  a.X = Hd;
+  a.K = 4 * E;
+  a.N = E;
+  a.W = w16 + (size_t)E * 4 * E;
+  a.bias = w + wo[W_CM_B2];
+  a.Y = Md;
+  a.act = 0;
+  a.count = count + 256;
+  cond_gemv_kernel<<<dim3(a.N / CG_COLS, a.K / CG_ROWS, zb), 256, 0, s>>>(a);
+  // every layer's [k | v]
+  a.X = Md;
+  a.K = E;
+  a.N = L * 2 * E;
+  a.W = w16 + (size_t)8 * E * E;
+  a.bias = bkv;
+  a.Y = kv_obs;
+  a.count = count + 512;
+  cond_gemv_kernel<<<dim3(a.N / CG_COLS, a.K / CG_ROWS, zb), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 
