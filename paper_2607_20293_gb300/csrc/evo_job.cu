@@ -155,6 +155,10 @@ __global__ void __launch_bounds__(256) cond_gemv_kernel(const CondGemv a) {
   const int g = blockIdx.x, kb = blockIdx.y, z = blockIdx.z, KB = gridDim.y;
   const int t0 = z * CG_TOK, nt = min(CG_TOK, a.ntok - t0), k0 = kb * CG_ROWS;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // the next stage may launch now; this one touches memory only after the
+  // previous stage (its input, the shared partial sums) has completed
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (tid < CG_TOK * CG_ROWS) {
     const int t = tid / CG_ROWS, r = tid % CG_ROWS, k = k0 + r;
     float v = 0.f;
@@ -275,7 +279,17 @@ cudaError_t launch_obs_cond_fast(const float* w, const int* wo, const __nv_bfloa
   a.Y = Md;
   a.act = 0;
   a.count = count + 256;
-  cond_gemv_kernel<<<dim3(a.N / CG_COLS, a.K / CG_ROWS, zb), 256, 0, s>>>(a);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.blockDim = dim3(256);
+  cfg.stream = s;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3(a.N / CG_COLS, a.K / CG_ROWS, zb);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, cond_gemv_kernel, a);
+  if (e != cudaSuccess) return e;
   // every layer's [k | v]
   a.X = Md;
   a.K = E;
@@ -284,7 +298,9 @@ cudaError_t launch_obs_cond_fast(const float* w, const int* wo, const __nv_bfloa
   a.bias = bkv;
   a.Y = kv_obs;
   a.count = count + 512;
-  cond_gemv_kernel<<<dim3(a.N / CG_COLS, a.K / CG_ROWS, zb), 256, 0, s>>>(a);
+  cfg.gridDim = dim3(a.N / CG_COLS, a.K / CG_ROWS, zb);
+  e = cudaLaunchKernelEx(&cfg, cond_gemv_kernel, a);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
