@@ -8,7 +8,7 @@
   X(0, __nv_bfloat16, 256, 4, 16, 16, 1, 2, 32768, 4)          \
   X(1, __nv_bfloat16, 256, 4, 16, 16, 2, 2, 32768, 2)          \
   X(2, __nv_bfloat16, 256, 4, 16, 8, 1, 2, 32768, 4)           \
-  X(3, __nv_bfloat16, 256, 4, 16, 4, 1, 2, 32768, 4)           \
+  X(3, __nv_bfloat16, 256, 4, 16, 4, 1, 2, 24576, 3)           \
   X(4, __nv_bfloat16, 512, 8, 32, 16, 1, 2, 16384, 2)          \
   X(5, __nv_bfloat16, 64, 2, 8, 4, 1, 2, 32768, 4)             \
   X(6, float, 64, 2, 8, 2, 1, 4, 32768, 4)                     \
