@@ -452,9 +452,10 @@ struct Loop {
   }
 
   // ---------------------------------------------------------------- first GEMM
-  // A = xln.  SA / CA: f32 rows of q|k|v (SA) or q (CA) + bias; FFN:
-  // T(gelu(. + bias)).  The output region aliases xln, so all warps finish
-  // their k-loop before any epilogue writes.
+  // A = xln.  SA / CA: q|k|v (SA) or q (CA) + bias, as bf16 attention tiles in
+  // ablk (tensor-core attention) or f32 rows aliasing xln; FFN:
+  // T(gelu(. + bias)) aliasing xln.  Where the output aliases xln, all warps
+  // finish their k-loop before any epilogue writes.
   template <int U>
   __device__ __forceinline__ static void gemm1(const JobParams& p, Ctx& cx, const uint8_t* slab0) {
     constexpr int N = S::n1(U);
