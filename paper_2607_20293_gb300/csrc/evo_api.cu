@@ -80,6 +80,7 @@ struct evo_handle {
   Alt alt[2];
   int n_alt = 0;
   const JobParams* last_base = nullptr;   // decomposition of the last cluster launch
+  JobParams replan{};                     // a population call's plan with fewer samples per job
   int last_mc = 0;
 };
 
@@ -1067,6 +1068,8 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
     p.vec = h->vec;
     p.cache = h->cache;
     p.status = h->status;
+    h->replan = p;
+    pk.base = &h->replan;
   }
   p.samples = (int)samples;
   p.per_sched = N_obs;
