@@ -88,6 +88,15 @@ def dist_env():
     return world, rank, local
 
 
+def max_over_ranks(values, device: str):
+    """Element-wise maximum of per-rank timings (seconds) over the process group."""
+    import torch
+    import torch.distributed as tdist
+    t = torch.tensor([float(v) for v in values], device=device, dtype=torch.float64)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
 class Clocks:
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -281,9 +290,7 @@ def run_ours(args, world, rank, local):
     total_s = sum(headline["ms"]) / 1000.0
     total_e2e = sum(headline["e2e_ms"]) / 1000.0
     if dist:
-        t = torch.tensor([total_s, total_e2e], device="cuda")
-        tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
-        total_s, total_e2e = float(t[0]), float(t[1])
+        total_s, total_e2e = max_over_ranks([total_s, total_e2e], "cuda")
     if rank != 0:
         return None
     chunks = n * args.steps * world
