@@ -814,7 +814,7 @@ struct Loop {
   // the cached outputs of b+1..bnext-1 and, when bnext < U, prepares its gather.
   template <int U>
   __device__ __forceinline__ static void unit(const JobParams& p, Ctx& cx, int job, int b, int t, int sample0,
-                                              int bnext, uint64_t valid) {
+                                              int bnext) {
     const int l = b / 3;
     float* ac = reinterpret_cast<float*>(cx.smem + p.sm.ac);
     float* ablk = reinterpret_cast<float*>(cx.smem + p.sm.ablk);
@@ -895,7 +895,7 @@ struct Loop {
           if (s < p.samples)
             p.trace[(((long long)t * p.U + b) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] = r;
         }
-        const float a = add_cached(p, cx, job, b + 1, bnext, t, sample0, valid, e, ac[e] + r);
+        const float a = add_cached(p, cx, job, b + 1, bnext, t, sample0, e, ac[e] + r);
         ac[e] = a;
         if (BF && bnext < p.U) reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb)[e] = __float2bfloat16_rn(a);
       }
@@ -904,19 +904,20 @@ struct Loop {
 
   // ---------------------------------------------------------------- skipped units b0..b1-1 (Eq. 1: a += c_b)
   // Element e of this CTA's columns: a + the cached outputs of the skipped
-  // units b0..b1-1 whose caches hold a value (valid), loaded eight at a time and
-  // summed pairwise before the add.  Runs inside the per-element pass that
-  // precedes them (the embedding or a refreshed unit's finish).
+  // units b0..b1-1 (zero for a unit not refreshed yet in this query), loaded
+  // eight at a time and summed pairwise before the add.  Runs inside the
+  // per-element pass that precedes them (the embedding or a refreshed unit's
+  // finish).
   __device__ __forceinline__ static float add_cached(const JobParams& p, Ctx& cx, int job, int b0, int b1, int t,
-                                                     int sample0, uint64_t valid, int e, float a) {
+                                                     int sample0, int e, float a) {
     if (b0 >= b1) return a;
-    const T* cb = cache_ptr(p, cx, job, 0);
     const int cstride = p.sm.cs >= 0 ? MEc : C * MEc;
-    for (int b = b0; b < b1; b += 8) {
-      const uint32_t live = (uint32_t)(valid >> b) & (b1 - b >= 8 ? 0xffu : (1u << (b1 - b)) - 1u);
+    const T* cb = cache_ptr(p, cx, job, b0) + e;
+    for (int b = b0; b < b1; b += 8, cb += 8 * cstride) {
+      const int n = b1 - b;                           // uniform over the block
       float cv[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) cv[q] = ((live >> q) & 1u) ? to_f<T>(cb[(b + q) * cstride + e]) : 0.f;
+      for (int q = 0; q < 8; ++q) cv[q] = q < n ? to_f<T>(cb[q * cstride]) : 0.f;
       a += ((cv[0] + cv[1]) + (cv[2] + cv[3])) + ((cv[4] + cv[5]) + (cv[6] + cv[7]));
       if (p.trace) {
         const int m = e >> S::lEc, j = e & (Ec - 1);
@@ -1101,6 +1102,12 @@ struct Loop {
         x[v] = p.noise[((long long)(s % p.obs_mod) * H + (m & (H - 1))) * p.A + (v % p.A)];
       }
       stage_kv_job(p, cx, sample0);
+      // the job's caches start as zero tensors: under the zero policy a unit not
+      // yet refreshed adds nothing (Sec. 3.1 cache reset), so the skip adds need no mask
+      for (int b = 0; b < p.U; ++b) {
+        T* cb = cache_ptr(p, cx, job, b);
+        for (int e = cx.tid; e < MEc; e += NCT) cb[e] = from_f<T>(0.f);
+      }
       // DDPM noise: thread v < G*H*A/4 copies 16 bytes of z_t per step (one chunk per thread)
       const float* zsrc = nullptr;
       int zdst = 0;
@@ -1138,7 +1145,7 @@ struct Loop {
             const int m = e >> S::lEc, j = e & (Ec - 1);
             float acc = 0.f;
             for (int a = 0; a < p.A; ++a) acc = fmaf(x[m * p.A + a], c_inw[a * Ec + j], acc);
-            const float a = add_cached(p, cx, job, 0, b, t, sample0, valid, e, acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j]);
+            const float a = add_cached(p, cx, job, 0, b, t, sample0, e, acc + c_inb[j] + c_pos[(m & (H - 1)) * Ec + j]);
             ac[e] = a;
             if (BF && b < p.U) reinterpret_cast<__nv_bfloat16*>(cx.smem + p.sm.acb)[e] = __float2bfloat16_rn(a);
           }
@@ -1149,9 +1156,9 @@ struct Loop {
           const uint64_t later = b + 1 < 64 ? refresh >> (b + 1) : 0ull;
           const int bnext = later ? b + __ffsll((long long)later) : p.U;
           const int u = b % 3;
-          if (u == 0) unit<0>(p, cx, job, b, t, sample0, bnext, valid);
-          else if (u == 1) unit<1>(p, cx, job, b, t, sample0, bnext, valid);
-          else unit<2>(p, cx, job, b, t, sample0, bnext, valid);
+          if (u == 0) unit<0>(p, cx, job, b, t, sample0, bnext);
+          else if (u == 1) unit<1>(p, cx, job, b, t, sample0, bnext);
+          else unit<2>(p, cx, job, b, t, sample0, bnext);
           b = bnext;
         }
         head_step(p, cx, t);

@@ -217,6 +217,15 @@ def test_automatic_decomposition_by_batch(torch, B):
     assert ev.status() == B.OK
 
 
+def test_scaleup_cluster_path_global_caches(torch, B):
+    # n_emb 512 on a 16-CTA cluster keeps the unit caches in global memory
+    cfg, W, obs, noise, ev, d_obs, d_noise = setup("scale256", 2, torch, B, wide_rows=-1)
+    S = synth.bernoulli_schedule(36, 100, 0.2, 11)
+    got = ev.denoise(d_obs, d_noise, S).cpu().numpy()
+    assert ev.last_call()["path"] == "cluster"
+    check(got[[1]], oracle_subset(W, cfg, obs, noise, S, [1]), TOL["bf16"], "scale-up cluster")
+
+
 @pytest.mark.parametrize("n,frac", [(256, 0.125), (1024, 1.0)])
 def test_scaleup(torch, B, n, frac):
     name = "scale256" if n == 256 else "scale1024"
