@@ -169,23 +169,26 @@ evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise
  * kernel's own duration.  Pass NULL, NULL to turn it off. */
 evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop);
 
-/* evo_denoise for callers that must not allocate device memory when they run
- * a query: for example code that issues its work under CUDA stream capture
- * (where cudaMalloc is not allowed), a real-time control loop that forbids
- * allocation after start-up, or an application whose own allocator owns the
- * device memory.  The paper has no counterpart; this is an interface choice.
- * Arguments, layouts and results are those of evo_denoise.  The per-call
- * scratch (the observation tokens' cross-attention keys/values and the
- * condition MLP's intermediates) lives in one file-scope device array of
- * 8 MiB that every GPU which loads this library holds until the process
- * exits; N * n_obs * (2 * n_layer + 6) * n_emb * 4 bytes must fit in it, else
- * EVO_ERR_SHAPE and nothing is launched.  No cudaMalloc,
- * cudaFree or allocating library routine is called.  The first call on a
- * device looks up the array's device address (cudaGetSymbolAddress) and
- * keeps it, so make that first call before any stream capture.  All calls
- * share the array and every call overwrites what it reads, so nothing needs
- * clearing; calls that overlap on the GPU (other streams, other handles)
- * race on it.  The handle's device must be the current device. */
+/* evo_denoise for callers that cannot allocate device memory when they run a
+ * query: a real-time control loop that forbids allocation once it has
+ * started (an allocation can block for an unbounded time), or an application
+ * whose own allocator reserved the device's memory up front, so that a
+ * cudaMalloc behind its back would fail or fragment that pool.  The paper has
+ * no counterpart; this is an interface choice.  Arguments, layouts and
+ * results are those of evo_denoise, and it always takes the one-cluster-per-job
+ * path, so its output is bit-identical to an evo_denoise call that takes that
+ * path.  The per-call scratch (the observation tokens' cross-attention
+ * keys/values and the condition MLP's intermediates) lives in one file-scope
+ * device array of 8 MiB that every GPU which loads this library holds until
+ * the process exits; N * n_obs * (2 * n_layer + 6) * n_emb * 4 bytes must fit
+ * in it (186 samples of the Push-T-shaped model), else EVO_ERR_SHAPE and
+ * nothing is launched.  No cudaMalloc, cudaFree or allocating library routine
+ * is called.  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) and keeps it; make that first call before any stream
+ * capture.  All calls share the array and every call overwrites all of it
+ * that it reads, so nothing needs clearing; calls that overlap on the GPU
+ * (other streams, other handles) race on it.  The handle's device must be the
+ * current device (EVO_ERR_ARG otherwise). */
 evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noise,
                                const uint8_t* S, int32_t S_rows, int32_t N,
                                float* out_actions, void* stream);

@@ -140,7 +140,11 @@ def _ptr(x) -> int | None:
     if x is None:
         return None
     if isinstance(x, np.ndarray):
+        if not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("arrays passed to the C ABI must be C-contiguous")
         return x.ctypes.data
+    if not x.is_contiguous():
+        raise ValueError("tensors passed to the C ABI must be contiguous")
     return x.data_ptr()
 
 

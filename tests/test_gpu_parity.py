@@ -265,11 +265,21 @@ def test_population_64x16(torch, B, path):
     assert ev.last_call()["path"] == path
     host_dev = np.linalg.norm((x - full[None]).reshape(P, N, -1), axis=2).mean(1)
     assert np.allclose(dev, host_dev, rtol=1e-4, atol=1e-5)
-    # sampled chunks against the oracle, including the reference
-    for p, n in [(0, 0), (13, 5), (P - 1, N - 1)]:
-        want = O.denoise(W, cfg, obs[[n]], noise[:, [n]], pop[p])
-        check(x[p, n][None], want, TOL["bf16"], f"candidate {p} obs {n}")
-    check(full[[3]], O.denoise(W, cfg, obs[[3]], noise[:, [3]], np.ones((24, 100), np.uint8)), TOL["bf16"])
+    # sampled candidates on every observation against the oracle's population
+    # evaluation (its first candidate is the all-refresh lattice, so its actions
+    # are the oracle's reference x_full)
+    ones = np.ones_like(pop[0])
+    sel = [0, 13, P - 1]
+    xs_o, dev_o = O.population_deviation(W, cfg, obs, noise, np.stack([ones] + [pop[p] for p in sel]))
+    assert dev_o[0] == 0.0
+    full_err = np.linalg.norm((full - xs_o[0]).reshape(N, -1), axis=1)
+    check(full, xs_o[0], TOL["bf16"], "all-refresh reference")
+    for j, p in enumerate(sel):
+        check(x[p], xs_o[1 + j], TOL["bf16"], f"candidate {p}")
+        # |dev - dev_o| <= mean_n (||x_pn - x_pn^o|| + ||full_n - full_n^o||) by the triangle inequality
+        cand_err = np.linalg.norm((x[p] - xs_o[1 + j]).reshape(N, -1), axis=1)
+        bound = float(np.mean(cand_err + full_err)) + 1e-5
+        assert abs(float(dev[p]) - dev_o[1 + j]) <= bound, (p, dev[p], dev_o[1 + j], bound)
     # denser candidates deviate less on average
     dens = pop.reshape(P, -1).mean(1)
     assert np.corrcoef(dens, dev)[0, 1] < 0
