@@ -258,7 +258,7 @@ struct Loop {
                 const long long t0 = clock64();
                 while (!cx.dead && !mbar_try_wait(smem_u32(&cx.empty[slot]), ph ^ 1u)) {
                   __nanosleep(64);
-                  if (clock64() - t0 > WAIT_LIMIT) {
+                  if (clock64() - t0 > cx.wait_limit) {
                     atomicOr(p.status, ST_TIMEOUT);
                     cx.dead = 1;
                   }
@@ -990,6 +990,9 @@ struct Loop {
         }
       }
     } else {
+      // a thread reads a whole row of ac, written element by element by other
+      // threads (the last refreshed unit's finish, or the step's embedding)
+      bar_compute();
       for (int o = cx.tid; o < M * NP; o += NCT) {
         const int m = o / NP, q = o - m * NP;
         const float* arow = ac + m * Ec;
@@ -1195,6 +1198,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   cx.q = cx.qa = 0;
   cx.cph = cx.pg = cx.pr = cx.ph0 = cx.ph1 = 0;
   cx.dead = 0;
+  cx.wait_limit = p.wait_limit;
   {
     // staging map: chunk v = tid over [G][1+n_obs][k chunks (dh/4) | v chunks (Ec/4)]
     constexpr int kq = S::dh / 4, per_tok = kq + S::Ec / 4;
@@ -1268,6 +1272,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) job_kernel(const __grid_constant_
   }
   __syncwarp();
   hw_cluster_sync();
+  // In normal operation every exchange copy has been waited for by its
+  // receiver before the receiver arrives here, and a sender arrives only
+  // after its own waits, so no copy is in flight once all CTAs have passed
+  // this barrier.  After a timeout a CTA skips its remaining waits, so the
+  // last copies may still be landing (cluster barriers do not order the
+  // asynchronous copies): give them time before the shared memory is freed.
+  settle_after_timeout(p.status, cx.dead != 0);
 }
 
 // Host side of one shape: the plan must agree with the compile-time constants.
