@@ -46,7 +46,9 @@ typedef enum {
   EVO_ERR_CUDA = 4,         /* a CUDA runtime call failed */
   EVO_ERR_TIMEOUT = 5,      /* a device-side wait exceeded its iteration limit */
   EVO_ERR_OOM = 6,          /* device allocation failed */
-  EVO_ERR_UNSUPPORTED = 7   /* no GPU with cluster launch, or the shape does not fit on chip */
+  EVO_ERR_UNSUPPORTED = 7,  /* no GPU with cluster launch, or the shape does not fit on chip */
+  EVO_ERR_CORRUPT = 8       /* a guard band around an activation buffer was overwritten, or (debug
+                               build) a device-side index check failed */
 } evo_status;
 
 enum { EVO_SAMPLER_DDPM = 0, EVO_SAMPLER_DDIM = 1 };
@@ -158,7 +160,8 @@ evo_status evo_schedule_fixed_interval(int32_t n_units, int32_t T, int32_t M, ui
 
 /* Debug variant of evo_denoise that also records the residual added at every
  * lattice cell: trace device [T][3L][N][H][E] float32 (refreshed cells: r_{b,t};
- * skipped cells: the cached c_b as stored; empty cache under ZERO: 0). */
+ * skipped cells: the cached c_b as stored; empty cache under ZERO: 0).  Takes
+ * the same path (one cluster per job, or batch-wide) as evo_denoise would. */
 evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise,
                              const uint8_t* S, int32_t S_rows, int32_t N,
                              float* out_actions, float* trace, void* stream);
@@ -192,6 +195,25 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop);
 evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noise,
                                const uint8_t* S, int32_t S_rows, int32_t N,
                                float* out_actions, void* stream);
+
+/* Diagnostic of the device-side failure path (the paper has no counterpart).
+ * Every wait in the library's kernels is bounded: when it gives up, the kernel
+ * records EVO_ERR_TIMEOUT in the handle's status word and ends instead of
+ * hanging.  This entry point exercises that path safely: one thread of one
+ * block (no cluster, no asynchronous copy, no tensor memory) waits on a
+ * barrier that nothing arrives at, through the same wait helper as the
+ * denoising-loop kernel (helper 0, limit in SM cycles, 1..10^7) or the
+ * tensor-core kernels (helper 1, limit in polls, 1..10^5), so the wait runs
+ * out.  Afterwards evo_get_status() returns EVO_ERR_TIMEOUT once (and clears
+ * it); the handle stays usable.  EVO_ERR_ARG for other helpers or limits. */
+evo_status evo_test_wait_timeout(evo_handle* h, int32_t helper, int64_t limit, void* stream);
+
+/* Debug aid (the paper has no counterpart): every activation buffer of the
+ * handle (unit caches, and on the batch-wide path the residual stream and the
+ * GEMM operands) is allocated with a 4 KiB guard band of a fixed pattern on
+ * each side.  Synchronizes the handle's last stream and checks every band:
+ * EVO_OK if all are intact, EVO_ERR_CORRUPT if a kernel wrote past a buffer. */
+evo_status evo_check_guards(evo_handle* h);
 
 /* Synchronizes the handle's last stream, returns and clears the device status word. */
 evo_status evo_get_status(evo_handle* h);

@@ -9,13 +9,15 @@ from __future__ import annotations
 
 import ctypes
 import os
+import weakref
 
 import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libevo.so")
+LIB_PATH_DEBUG = os.path.join(HERE, "libevo_debug.so")
 
-OK, ERR_ARG, ERR_SHAPE, ERR_SCHEDULE, ERR_CUDA, ERR_TIMEOUT, ERR_OOM, ERR_UNSUPPORTED = range(8)
+OK, ERR_ARG, ERR_SHAPE, ERR_SCHEDULE, ERR_CUDA, ERR_TIMEOUT, ERR_OOM, ERR_UNSUPPORTED, ERR_CORRUPT = range(9)
 SAMPLERS = {"ddpm": 0, "ddim": 1}
 DTYPES = {"fp32": 0, "bf16": 1}
 EMPTY = {"zero": 0, "force": 1}
@@ -58,15 +60,23 @@ class EvoError(RuntimeError):
 
 
 _lib = None
+_lib_debug = None
+# handles alive in this process (their guard bands can be checked after a test)
+_live: "weakref.WeakSet[Evo]" = weakref.WeakSet()
+# guard failures found when a handle was closed
+guard_failures: list[str] = []
 
 
-def load() -> ctypes.CDLL:
-    global _lib
-    if _lib is not None:
-        return _lib
-    if not os.path.exists(LIB_PATH):
-        raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2607_20293_gb300.build.build()")
-    lib = ctypes.CDLL(LIB_PATH)
+def load(debug: bool = False) -> ctypes.CDLL:
+    """The library (debug=True: the build with device-side index checks)."""
+    global _lib, _lib_debug
+    if (_lib_debug if debug else _lib) is not None:
+        return _lib_debug if debug else _lib
+    path = LIB_PATH_DEBUG if debug else LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with paper_2607_20293_gb300.build.build("
+                           f"{'debug=True' if debug else ''})")
+    lib = ctypes.CDLL(path)
     P, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
     cfgp = ctypes.POINTER(EvoConfig)
     sig = {
@@ -76,6 +86,8 @@ def load() -> ctypes.CDLL:
         "evo_denoise": (I32, [P, P, P, P, I32, I32, P, P]),
         "evo_denoise_trace": (I32, [P, P, P, P, I32, I32, P, P, P]),
         "evo_denoise_noalloc": (I32, [P, P, P, P, I32, I32, P, P]),
+        "evo_test_wait_timeout": (I32, [P, I32, ctypes.c_int64, P]),
+        "evo_check_guards": (I32, [P]),
         "evo_denoise_population": (I32, [P, P, P, P, I32, I32, I32, P, P, P]),
         "evo_flops": (I32, [P, P, I32, ctypes.POINTER(I64)]),
         "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
@@ -97,7 +109,10 @@ def load() -> ctypes.CDLL:
         fn = getattr(lib, name)
         fn.restype = res
         fn.argtypes = args
-    _lib = lib
+    if debug:
+        _lib_debug = lib
+    else:
+        _lib = lib
     return lib
 
 
@@ -190,8 +205,8 @@ class Evo:
     """One evo_handle: packed weights, caches and workspace on the current GPU."""
 
     def __init__(self, cfg: dict, weights: dict, max_batch: int, cluster: int = 0, job_samples: int = 0,
-                 empty: str = "zero", debug_sync: bool = False, wide_rows: int = 0):
-        lib = load()
+                 empty: str = "zero", debug_sync: bool = False, wide_rows: int = 0, debug_lib: bool = False):
+        lib = self._lib = load(debug_lib)
         self.cfg = dict(cfg)
         self._c = make_config(cfg, cluster, job_samples, empty, debug_sync, wide_rows)
         self._blob = pack_blob(cfg, weights)
@@ -200,11 +215,17 @@ class Evo:
                               ctypes.byref(h)), "evo_create")
         self._h = h
         self.max_batch = max_batch
+        _live.add(self)
 
     def close(self):
         if getattr(self, "_h", None) and self._h.value:
-            load().evo_destroy(self._h)
+            rc = self._lib.evo_check_guards(self._h)
+            if rc != OK:
+                guard_failures.append(f"handle {self.cfg.get('n_emb')}x{self.cfg.get('n_layer')}: "
+                                      f"{status_string(rc)}")
+            self._lib.evo_destroy(self._h)
             self._h = ctypes.c_void_p()
+            _live.discard(self)
 
     def __del__(self):
         try:
@@ -214,13 +235,13 @@ class Evo:
 
     def launch_info(self) -> dict:
         v = [ctypes.c_int32() for _ in range(4)]
-        _check(load().evo_get_launch_info(self._h, *[ctypes.byref(x) for x in v]), "evo_get_launch_info")
+        _check(self._lib.evo_get_launch_info(self._h, *[ctypes.byref(x) for x in v]), "evo_get_launch_info")
         return dict(cluster=v[0].value, job_samples=v[1].value, max_clusters=v[2].value, smem_bytes=v[3].value)
 
     def last_call(self) -> dict:
         """path of the last call ("cluster" or "wide") and the kernels it launched"""
         path, k = ctypes.c_int32(), ctypes.c_int64()
-        _check(load().evo_get_last_call(self._h, ctypes.byref(path), ctypes.byref(k)), "evo_get_last_call")
+        _check(self._lib.evo_get_last_call(self._h, ctypes.byref(path), ctypes.byref(k)), "evo_get_last_call")
         return dict(path="wide" if path.value == 1 else "cluster", kernels=k.value)
 
     def denoise(self, obs, noise, S, out=None, stream=None, trace=None):
@@ -231,10 +252,10 @@ class Evo:
                               device=obs.device)
         S = _lattice(S)
         if trace is None:
-            rc = load().evo_denoise(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
+            rc = self._lib.evo_denoise(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
                                     _stream(stream))
         else:
-            rc = load().evo_denoise_trace(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
+            rc = self._lib.evo_denoise_trace(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], N, _ptr(out),
                                           _ptr(trace), _stream(stream))
         _check(rc, "evo_denoise")
         return out
@@ -243,7 +264,7 @@ class Evo:
         """evo_denoise with its per-call scratch in the library's static device
         array (no device allocation); `out` must be provided."""
         S = _lattice(S)
-        rc = load().evo_denoise_noalloc(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], obs.shape[0],
+        rc = self._lib.evo_denoise_noalloc(self._h, _ptr(obs), _ptr(noise), _ptr(S), S.shape[0], obs.shape[0],
                                         _ptr(out), _stream(stream))
         _check(rc, "evo_denoise_noalloc")
         return out
@@ -258,7 +279,7 @@ class Evo:
                               device=obs.device)
         if dev is None:
             dev = torch.empty((P,), dtype=torch.float32, device=obs.device)
-        rc = load().evo_denoise_population(self._h, _ptr(obs), _ptr(noise), _ptr(S_pop), P, S_pop.shape[1], N_obs,
+        rc = self._lib.evo_denoise_population(self._h, _ptr(obs), _ptr(noise), _ptr(S_pop), P, S_pop.shape[1], N_obs,
                                            _ptr(out), _ptr(dev), _stream(stream))
         _check(rc, "evo_denoise_population")
         return out, dev
@@ -266,7 +287,7 @@ class Evo:
     def flops(self, S) -> int:
         S = np.ascontiguousarray(S, dtype=np.uint8)
         out = ctypes.c_int64()
-        _check(load().evo_flops(self._h, S.ctypes.data, S.shape[0], ctypes.byref(out)), "evo_flops")
+        _check(self._lib.evo_flops(self._h, S.ctypes.data, S.shape[0], ctypes.byref(out)), "evo_flops")
         return out.value
 
     def set_profile_events(self, start=None, stop=None):
@@ -274,10 +295,19 @@ class Evo:
         (they must have been recorded once, so that their CUDA events exist)."""
         sp = start.cuda_event if start is not None else None
         ep = stop.cuda_event if stop is not None else None
-        _check(load().evo_set_profile_events(self._h, sp, ep), "evo_set_profile_events")
+        _check(self._lib.evo_set_profile_events(self._h, sp, ep), "evo_set_profile_events")
 
     def status(self) -> int:
-        return load().evo_get_status(self._h)
+        return self._lib.evo_get_status(self._h)
+
+    def check_guards(self) -> int:
+        """evo_check_guards: OK, or ERR_CORRUPT if a kernel wrote past an activation buffer."""
+        return self._lib.evo_check_guards(self._h)
+
+    def test_wait_timeout(self, helper: int, limit: int, stream=None):
+        """Run the bounded-wait helper of the loop kernel (0) or the tensor-core
+        kernels (1) on a barrier nothing arrives at, so that it gives up."""
+        _check(self._lib.evo_test_wait_timeout(self._h, helper, limit, _stream(stream)), "evo_test_wait_timeout")
 
 
 METRICS = {"cosine": 0, "mse": 1, "l1": 2, "w1": 3}

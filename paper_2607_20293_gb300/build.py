@@ -2,7 +2,9 @@
 
 Each .cu file is compiled in parallel with nvcc, then linked into one shared
 library next to this file.  No CMake, no torch extension machinery: the
-library exports only the C ABI of include/evo.h.
+library exports only the C ABI of include/evo.h.  build(debug=True) makes
+libevo_debug.so, the same library with device-side index checks
+(EVO_DEBUG_CHECKS: a failed check records a status bit and skips the access).
 """
 from __future__ import annotations
 
@@ -15,6 +17,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libevo.so")
+OUT_DEBUG = os.path.join(HERE, "libevo_debug.so")
 BUILD = os.path.join(ROOT, "_build")
 SOURCES = ["evo_api.cu", "evo_job.cu", "evo_loop_s01.cu", "evo_loop_s23.cu", "evo_loop_s45.cu", "evo_loop_f32.cu", "evo_wide.cu", "evo_redundancy.cu", "evo_search.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -36,8 +39,11 @@ def _stale(target: str, deps: list[str]) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(verbose: bool = False, extra: list[str] | None = None) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, extra: list[str] | None = None, debug: bool = False) -> str:
+    build_dir = os.path.join(BUILD, "debug") if debug else BUILD
+    out = OUT_DEBUG if debug else OUT
+    extra = list(extra or []) + (["-DEVO_DEBUG_CHECKS=1"] if debug else [])
+    os.makedirs(build_dir, exist_ok=True)
     nvcc = _nvcc()
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
     headers.append(os.path.join(ROOT, "include", "evo.h"))
@@ -45,10 +51,10 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
+        o = os.path.join(build_dir, os.path.splitext(src)[0] + ".o")
         objs.append(o)
         if _stale(o, [s] + headers):
-            jobs.append([nvcc, *ARCH, *FLAGS, *(extra or []), "-c", s, "-o", o])
+            jobs.append([nvcc, *ARCH, *FLAGS, *extra, "-c", s, "-o", o])
 
     def run(cmd):
         r = subprocess.run(cmd, capture_output=True, text=True)
@@ -59,9 +65,9 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
 
     with ThreadPoolExecutor(max_workers=len(jobs) or 1) as ex:
         list(ex.map(run, jobs))
-    if _stale(OUT, objs):
-        run([nvcc, *ARCH, "-shared", "-o", OUT, *objs, "-lcudart"])
-    return OUT
+    if _stale(out, objs):
+        run([nvcc, *ARCH, "-shared", "-o", out, *objs, "-lcudart"])
+    return out
 
 
 if __name__ == "__main__":

@@ -16,6 +16,8 @@
 #include "../../include/evo.h"
 #include "evo_internal.h"
 
+#include <nvtx3/nvToolsExt.h>
+
 #include <algorithm>
 #include <cmath>
 #include <cstring>
@@ -26,6 +28,7 @@ using namespace evo;
 
 struct evo_handle {
   evo_config cfg;
+  GuardList guards;             // guard bands of the handle's activation buffers
   int device = 0;
   int L = 0, E = 0, U = 0, T = 0, H = 0, A = 0;
   JobParams base{};
@@ -83,6 +86,53 @@ struct evo_handle {
   JobParams replan{};                     // a population call's plan with fewer samples per job
   int last_mc = 0;
 };
+
+namespace {
+
+// One NVTX range per public call (host side: covers staging and every launch
+// the call issues), so that a profiler timeline groups a call's kernels.  NVTX
+// is header-only and does nothing unless a tool is attached.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+
+}  // namespace
+
+namespace evo {
+
+cudaError_t guarded_malloc(void** user, size_t bytes, GuardList* list) {
+  unsigned char* base = nullptr;
+  cudaError_t e = cudaMalloc(&base, bytes + 2 * GUARD_BYTES);
+  if (e != cudaSuccess) return e;
+  e = cudaMemset(base, GUARD_FILL, GUARD_BYTES);
+  if (e == cudaSuccess) e = cudaMemset(base + GUARD_BYTES + bytes, GUARD_FILL, GUARD_BYTES);
+  if (e != cudaSuccess) {
+    cudaFree(base);
+    return e;
+  }
+  list->push_back({base, bytes});
+  *user = base + GUARD_BYTES;
+  return cudaSuccess;
+}
+
+void guarded_free(void* user) {
+  if (user) cudaFree(static_cast<unsigned char*>(user) - GUARD_BYTES);
+}
+
+int guards_check(const GuardList& list) {
+  std::vector<unsigned char> h(GUARD_BYTES);
+  for (const GuardedRegion& r : list)
+    for (int side = 0; side < 2; ++side) {
+      const unsigned char* g = r.base + (side ? GUARD_BYTES + r.bytes : 0);
+      if (cudaMemcpy(h.data(), g, GUARD_BYTES, cudaMemcpyDeviceToHost) != cudaSuccess) return -1;
+      for (unsigned char c : h)
+        if (c != GUARD_FILL) return 1;
+    }
+  return 0;
+}
+
+}  // namespace evo
 
 namespace {
 
@@ -325,6 +375,7 @@ int plan(const evo_config* c, int C, int g, int slot, int nslot, int smem_limit,
   if (slot < need) return -1;
   p.slot_bytes = slot;
   p.nslot = nslot;
+  p.wait_limit = WAIT_CYCLES_DEFAULT;
   // preference: caches on chip, per-step memory keys/values, double-buffered
   // head exchange, head weights on chip
   for (int cache_smem = 1; cache_smem >= 0; --cache_smem)
@@ -353,6 +404,7 @@ const char* evo_status_string(evo_status s) {
     case EVO_ERR_TIMEOUT: return "device wait timed out";
     case EVO_ERR_OOM: return "device out of memory";
     case EVO_ERR_UNSUPPORTED: return "unsupported on this device";
+    case EVO_ERR_CORRUPT: return "guard band overwritten or device index check failed";
   }
   return "unknown status";
 }
@@ -428,7 +480,7 @@ evo_status evo_destroy(evo_handle* h) {
   cudaFree(h->cond_bkv);
   cudaFree(h->cond_part);
   cudaFree(h->cond_count);
-  cudaFree(h->cache);
+  guarded_free(h->cache);
   cudaFree(h->sched);
   cudaFree(h->status);
   cudaFree(h->pop_x);
@@ -709,7 +761,8 @@ evo_status evo_create(const float* weights, size_t n_floats, const evo_config* c
     cudaMemcpy(h->cond_bkv, bkv.data(), bkv.size() * 4, cudaMemcpyHostToDevice);
     cudaMemset(h->cond_count, 0, 768 * sizeof(unsigned));
   }
-  if (cudaMalloc(&h->cache, cap_samples * H * (size_t)U * E * es) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (guarded_malloc(&h->cache, cap_samples * H * (size_t)U * E * es, &h->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
   h->sched_cap = cap_samples * U * T;
   if (cudaMalloc(&h->sched, h->sched_cap) != cudaSuccess) return fail(EVO_ERR_OOM);
   if (cudaMalloc(&h->status, 2 * sizeof(int)) != cudaSuccess) return fail(EVO_ERR_OOM);
@@ -875,7 +928,7 @@ evo_status stage_wide(evo_handle* h, const uint8_t* S, int n_sched, int rows, bo
 }
 
 cudaError_t launch_wide(evo_handle* h, const float* noise, float* out, int samples, int per_sched, int n_sched,
-                        int S_rows, cudaStream_t st) {
+                        int S_rows, cudaStream_t st, float* trace = nullptr) {
   WideCall c{};
   c.noise = noise;
   c.out = out;
@@ -889,6 +942,7 @@ cudaError_t launch_wide(evo_handle* h, const float* noise, float* out, int sampl
   c.S_dev = h->sched;
   c.n_sched = n_sched;
   c.S_rows = S_rows;
+  c.trace = trace;
   c.status = h->status;
   c.st = st;
   if (h->prof_start && h->prof_stop) {
@@ -913,11 +967,11 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
   if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (!trace && use_wide(h, N)) {
+  if (use_wide(h, N)) {
     const evo_status s = stage_wide(h, S, 1, S_rows, false, st);
     if (s != EVO_OK) return s;
     EVO_CUDA(obs_cond(h, obs, N, h->cond_scratch, h->kv_obs, st));
-    EVO_CUDA(launch_wide(h, noise, out, N, N, 1, S_rows, st));
+    EVO_CUDA(launch_wide(h, noise, out, N, N, 1, S_rows, st, trace));
     return finish(h, st);
   }
   const int* err = nullptr;
@@ -947,12 +1001,14 @@ extern "C" {
 
 evo_status evo_denoise(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
                        int32_t N, float* out_actions, void* stream) {
+  NvtxRange range("evo_denoise");
   return run(h, obs, noise, S, S_rows, N, out_actions, nullptr, stream);
 }
 
 evo_status evo_denoise_trace(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
                              int32_t N, float* out_actions, float* trace, void* stream) {
   if (!trace) return EVO_ERR_ARG;
+  NvtxRange range("evo_denoise_trace");
   return run(h, obs, noise, S, S_rows, N, out_actions, trace, stream);
 }
 
@@ -987,6 +1043,7 @@ extern "C" {
 
 evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noise, const uint8_t* S, int32_t S_rows,
                                int32_t N, float* out_actions, void* stream) {
+  NvtxRange range("evo_denoise_noalloc");
   if (!h || !obs || !noise || !S || !out_actions) return EVO_ERR_ARG;
   if (N <= 0 || N > h->max_batch) return EVO_ERR_SHAPE;
   if (S_rows != h->U && S_rows != h->L) return EVO_ERR_SCHEDULE;
@@ -1026,6 +1083,7 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
 evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* noise, const uint8_t* S_pop,
                                   int32_t P, int32_t S_rows, int32_t N_obs, float* out_actions, float* dev_l2,
                                   void* stream) {
+  NvtxRange range("evo_denoise_population");
   if (!h || !obs || !noise || !S_pop || !dev_l2) return EVO_ERR_ARG;
   if (P <= 0 || N_obs <= 0) return EVO_ERR_SHAPE;
   const long long samples = (long long)(P + 1) * N_obs;
@@ -1090,6 +1148,24 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   return finish(h, st);
 }
 
+evo_status evo_check_guards(evo_handle* h) {
+  if (!h) return EVO_ERR_ARG;
+  if (cudaStreamSynchronize(h->last_stream) != cudaSuccess) return EVO_ERR_CUDA;
+  int r = guards_check(h->guards);
+  if (r == 0 && h->wide) r = guards_check(*wide_guards(h->wide));
+  return r == 0 ? EVO_OK : (r > 0 ? EVO_ERR_CORRUPT : EVO_ERR_CUDA);
+}
+
+evo_status evo_test_wait_timeout(evo_handle* h, int32_t helper, int64_t limit, void* stream) {
+  if (!h || (helper != 0 && helper != 1)) return EVO_ERR_ARG;
+  // bounded so that the probe ends within milliseconds: 10^7 cycles or 10^5 polls
+  if (limit < 1 || limit > (helper == 0 ? 10000000 : 100000)) return EVO_ERR_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  EVO_CUDA(launch_wait_probe(helper, limit, h->status, st));
+  h->last_stream = st;
+  return EVO_OK;
+}
+
 evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
   if (!h || (start == nullptr) != (stop == nullptr)) return EVO_ERR_ARG;
   h->prof_start = reinterpret_cast<cudaEvent_t>(start);
@@ -1134,6 +1210,7 @@ evo_status evo_get_status(evo_handle* h) {
   if (cudaMemcpy(st, h->status, sizeof(st), cudaMemcpyDeviceToHost) != cudaSuccess) return EVO_ERR_CUDA;
   if (st[0] || st[1]) cudaMemset(h->status, 0, sizeof(st));
   if (st[1]) return EVO_ERR_SCHEDULE;
+  if (st[0] & ST_INDEX) return EVO_ERR_CORRUPT;
   if (st[0] & ST_TIMEOUT) return EVO_ERR_TIMEOUT;
   if (st[0] & ST_SCHEDULE) return EVO_ERR_SCHEDULE;
   return EVO_OK;

@@ -5,6 +5,7 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <vector>
 
 #include "evo.h"
 
@@ -19,6 +20,52 @@ constexpr int PLD = 33;             // row stride (floats) of the attention-prob
 // error bits written to the device status word
 constexpr int ST_SCHEDULE = 1;
 constexpr int ST_TIMEOUT = 2;
+constexpr int ST_INDEX = 4;         // a device-side index check failed (debug builds)
+
+// Device-side index checks of the debug build (EVO_DEBUG_CHECKS): a failed
+// check records ST_INDEX in the status word and the caller skips the access
+// (no trap, so the context stays usable).  In the normal build it is a
+// constant true and costs nothing.
+#ifdef EVO_DEBUG_CHECKS
+__device__ __forceinline__ bool dcheck(bool ok, int* status) {
+  if (!ok) atomicOr(status, ST_INDEX);
+  return ok;
+}
+#else
+__device__ __forceinline__ constexpr bool dcheck(bool, int*) { return true; }
+#endif
+
+// Guard bands around the activation buffers: GUARD_BYTES of a fixed pattern
+// before and after each one, so that a kernel writing past either end is
+// caught by evo_check_guards (a stand-in for a memory checker).
+constexpr size_t GUARD_BYTES = 4096;
+constexpr unsigned char GUARD_FILL = 0xA7;
+struct GuardedRegion {
+  unsigned char* base;   // allocation start: [guard | user bytes | guard]
+  size_t bytes;          // user bytes
+};
+using GuardList = std::vector<GuardedRegion>;
+// cudaMalloc of bytes + 2 guards; *user = the first byte after the leading guard
+cudaError_t guarded_malloc(void** user, size_t bytes, GuardList* list);
+void guarded_free(void* user);
+// 0: every guard intact; 1: a guard was overwritten; -1: a CUDA call failed
+int guards_check(const GuardList& list);
+
+// Limits of the bounded waits (kernel parameters, so that a diagnostic can run
+// the same helpers with a tiny limit): the loop kernel gives up after this many
+// SM cycles (~2 s), the tensor-core kernels after this many polls.
+constexpr long long WAIT_CYCLES_DEFAULT = 4000000000LL;
+constexpr long long WAIT_POLLS_DEFAULT = 1ll << 26;
+// After a wait gave up, copies issued by other threads or CTAs may still be in
+// flight into this CTA's shared memory (or reading from it): before the CTA
+// exits it gives them this many cycles (~0.2 ms) to land.
+constexpr long long SETTLE_CYCLES = 400000LL;
+
+__device__ __forceinline__ void settle_after_timeout(const int* status, bool dead) {
+  if (!dead && !(*reinterpret_cast<const volatile int*>(status) & ST_TIMEOUT)) return;
+  const long long t0 = clock64();
+  while (clock64() - t0 < SETTLE_CYCLES) __nanosleep(1000);
+}
 
 // Byte offsets of the regions of one CTA's dynamic shared memory.
 struct SmemLayout {
@@ -60,6 +107,7 @@ struct JobParams {
   int n_jobs;
   int sampler, force;
   int nslot, slot_bytes;
+  long long wait_limit;           // SM cycles before a wait gives up (WAIT_CYCLES_DEFAULT)
   int head_sep;                   // 1: head partials double-buffered by step parity; 0: one buffer + cluster barrier
   int npr;                        // floats per row of a head partial block: 2 + A, 4-padded
   // samples
@@ -114,6 +162,10 @@ cudaError_t launch_obs_cond_fast(const float* wf32, const int* woff, const __nv_
 cudaError_t launch_obs_cond(const float* wf32, const int* woff_dev, const int* woff, const float* obs, int N,
                             int n_obs, int D, int L, int E, float* scratch, float* kv_obs, cudaStream_t s);
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s);
+// one CTA, no cluster, no copies: waits on an mbarrier nothing arrives at through
+// the loop kernel's helper (helper 0, limit in cycles) or the tensor-core
+// kernels' helper (helper 1, limit in polls); the wait gives up and sets ST_TIMEOUT
+cudaError_t launch_wait_probe(int helper, long long limit, int* status, cudaStream_t s);
 cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev, cudaStream_t s);
 
 // batch-wide path (evo_wide.cu)
@@ -128,6 +180,7 @@ struct WideCall {
   const uint8_t* S_host;          // [n_sched][S_rows][T], validated
   const uint8_t* S_dev;           // the same lattices on the device
   int n_sched, S_rows;
+  float* trace;                   // [T][U][samples][H][E] or null: the residual added at every lattice cell
   int* status;
   cudaStream_t st;
 };
@@ -136,6 +189,7 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
                 long long max_rows, int max_sched);   // evo_status
 void wide_destroy(WideState* w);
 long long wide_rows_capacity(const WideState* w);
+const GuardList* wide_guards(const WideState* w);
 long long wide_last_launches(const WideState* w);
 cudaError_t wide_run(WideState* w, const WideCall& c);
 

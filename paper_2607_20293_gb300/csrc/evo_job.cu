@@ -6,6 +6,7 @@
 #include <algorithm>
 
 #include "evo_ptx.cuh"
+#include "evo_tc.cuh"
 #include "evo_shapes.h"
 
 namespace evo {
@@ -454,6 +455,34 @@ cudaError_t launch_obs_cond(const float* w, const int* wo_dev, const int* wo, co
   float* X = scratch + (size_t)ntok * 5 * E;
   cond_embed_kernel<<<ntok, 256, 0, s>>>(w, wo_dev, obs, nullptr, n_obs, D, E, 0, X);
   return cond_tokens_to_kv(w, wo_dev, wo, L, E, ntok, X, scratch, kv_obs, s);
+}
+
+// Diagnostic of the device-side failure path: one thread waits on an mbarrier
+// that nothing arrives at, through the same bounded-wait helper the loop kernel
+// (helper 0) or the tensor-core kernels (helper 1) use.  No cluster, no copy and
+// no tensor memory are involved, so giving up leaves nothing in flight.
+__global__ void wait_probe_kernel(int helper, long long limit, int* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (helper == 0) {
+      Ctx cx{};
+      cx.dead = 0;
+      cx.wait_limit = limit;
+      wait_parity(smem_u32(&bar), 0u, false, cx, status);
+    } else {
+      tc::mbar_wait(&bar, 0u, status, limit);
+    }
+  }
+}
+
+cudaError_t launch_wait_probe(int helper, long long limit, int* status, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(helper, limit, status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s) {

@@ -892,7 +892,7 @@ struct Loop {
         if (p.trace) {
           const int m = e >> S::lEc, j = e & (Ec - 1);
           const int s = sample0 + (m >> S::lH);
-          if (s < p.samples)
+          if (s < p.samples && dcheck(t < p.T && b < p.U && cx.c * Ec + j < E, p.status))
             p.trace[(((long long)t * p.U + b) * p.samples + s) * H * E + (m & (H - 1)) * E + cx.c * Ec + j] = r;
         }
         const float a = add_cached(p, cx, job, b + 1, bnext, t, sample0, e, ac[e] + r);
@@ -1172,7 +1172,8 @@ struct Loop {
       if (cx.c == 0) {
         for (int v = cx.tid; v < M * p.A; v += NCT) {
           const int s = sample0 + v / (H * p.A);
-          if (s < p.samples) p.out[(long long)sample0 * H * p.A + v] = x[v];
+          if (s < p.samples && dcheck((long long)sample0 * H * p.A + v < (long long)p.samples * H * p.A, p.status))
+            p.out[(long long)sample0 * H * p.A + v] = x[v];
         }
       }
       bar_compute();

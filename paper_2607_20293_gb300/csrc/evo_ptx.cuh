@@ -198,10 +198,10 @@ __device__ __forceinline__ float mish(float x) {
   return x * tanhf(sp);
 }
 
-// A bounded wait: after ~2 s of SM cycles the wait gives up, records
-// ST_TIMEOUT and lets the thread continue so that every CTA still reaches the
-// same synchronisation points and the kernel ends.
-constexpr long long WAIT_LIMIT = 4000000000LL;
+// A bounded wait: after cx.wait_limit SM cycles (JobParams::wait_limit, ~2 s
+// by default) the wait gives up, records ST_TIMEOUT and lets the thread
+// continue so that every CTA still reaches the same synchronisation points and
+// the kernel ends.
 
 struct Ctx {
   uint8_t* smem;
@@ -215,6 +215,7 @@ struct Ctx {
   uint32_t qa;     // next slab to acquire (qa - q slabs are held)
   uint32_t cph, pg, pr, ph0, ph1;   // phase parities
   int dead;
+  long long wait_limit;
   int c, tid, warp, lane;
   // this thread's 16-byte chunk of a memory key/value staging (kv_i < 0: none):
   // sample kv_i of the job, token kv_tok, float offset kv_src within the token's
@@ -230,7 +231,7 @@ __device__ __forceinline__ void wait_parity(uint32_t addr, uint32_t parity, bool
   if (cluster_acq ? mbar_try_wait_acq_cluster(addr, parity) : mbar_try_wait(addr, parity)) return;
   const long long t0 = clock64();
   while (!(cluster_acq ? mbar_try_wait_acq_cluster(addr, parity) : mbar_try_wait(addr, parity))) {
-    if (clock64() - t0 > WAIT_LIMIT) {
+    if (clock64() - t0 > cx.wait_limit) {
       atomicOr(status, ST_TIMEOUT);
       cx.dead = 1;
       return;

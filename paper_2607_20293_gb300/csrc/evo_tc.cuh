@@ -13,8 +13,8 @@
 //     accumulator to the epilogue;
 //   * warps 2-9: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
 //     quadrant 32 (w % 4) .. +31 and one half of the tile's columns, 32 at a
-//     time (tcgen05.ld), applies bias / GELU / residual-and-cache, stores, and
-//     releases the accumulator.
+//     time (tcgen05.ld), applies bias (and GELU), stores bf16, and releases the
+//     accumulator.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
 // next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
@@ -35,7 +35,6 @@ constexpr int BM = 128, BK = 64;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int EPI_WARPS = 8;                                    // two per TMEM lane quadrant
 constexpr int NTHREADS_GEMM = 32 * (2 + EPI_WARPS);             // producer, MMA, epilogue warps
-constexpr long long TC_WAIT_LIMIT = 1ll << 26;                  // polls before a wait gives up
 
 template <int BN>
 struct TileCfg {
@@ -50,17 +49,14 @@ struct TileCfg {
       (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 };
 
-enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2 };
+enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1 };
 
 struct GemmArgs {
   int K;                      // multiple of BK
   int b_row0;                 // first row of B (its tensor map spans every layer's matrices)
   const float* bias;          // [N] fp32
-  __nv_bfloat16* out;         // EPI_BF16 / EPI_GELU_BF16: out[row * ldo + n]
+  __nv_bfloat16* out;         // out[row * ldo + n]
   int ldo;
-  float* resid;               // EPI_RESID: residual stream [rows][ldr] fp32, += r
-  __nv_bfloat16* cache;       // EPI_RESID: unit cache [rows][ldr], <- bf16(r)
-  int ldr;
   int rows;                   // real rows; rows >= this are padding
   // refresh gate (null: every row refreshes): row -> sample row / H -> lattice
   // (sample / per_sched); refresh = S[lattice * S_stride + srow * T + t]
@@ -68,6 +64,7 @@ struct GemmArgs {
   long long S_stride;
   int srow, T, t, H, per_sched, force;
   int* status;
+  long long wait_limit;       // polls before a wait gives up (WAIT_POLLS_DEFAULT)
 };
 
 // ---------------------------------------------------------------- PTX wrappers
@@ -87,11 +84,12 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// bounded wait for the phase of `parity` to complete
-__device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, int* status) {
+// bounded wait for the phase of `parity` to complete: gives up after `limit`
+// polls and records ST_TIMEOUT
+__device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, int* status, long long limit) {
   const uint32_t a = su32(bar);
   if (mbar_test(a, parity)) return;
-  for (long long i = 0; i < TC_WAIT_LIMIT; ++i) {
+  for (long long i = 0; i < limit; ++i) {
     if (mbar_test(a, parity)) return;
     if (i > 64) __nanosleep(32);
   }
@@ -175,14 +173,6 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ bool row_refreshes(const GemmArgs& g, int row) {
-  if (row >= g.rows) return false;
-  if (!g.S) return true;
-  if (g.force && g.t == 0) return true;
-  const int sample = row / g.H;
-  return g.S[(long long)(sample / g.per_sched) * g.S_stride + (long long)g.srow * g.T + g.t] != 0;
-}
-
 __device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
 
 // does any row of the tile starting at m0 refresh?  (the same answer in every role)
@@ -206,48 +196,21 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n
     v[4 * q + 2] += bb.z;
     v[4 * q + 3] += bb.w;
   }
-  if constexpr (MODE == EPI_RESID) {
-    float4* a4 = reinterpret_cast<float4*>(g.resid + (long long)row * g.ldr + n);
-    uint4* c4 = reinterpret_cast<uint4*>(g.cache + (long long)row * g.ldr + n);
-    float4 av[8];
+  if constexpr (MODE == EPI_GELU_BF16) {
 #pragma unroll
-    for (int q = 0; q < 8; ++q) av[q] = a4[q];
+    for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
+  }
+  uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      uint4 pk;
-      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+  for (int q = 0; q < 4; ++q) {
+    uint4 pk;
+    uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
-        pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-      }
-      c4[q] = pk;
+    for (int j = 0; j < 4; ++j) {
+      __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
+      pw[j] = *reinterpret_cast<uint32_t*>(&h2);
     }
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      av[q].x += v[4 * q];
-      av[q].y += v[4 * q + 1];
-      av[q].z += v[4 * q + 2];
-      av[q].w += v[4 * q + 3];
-      a4[q] = av[q];
-    }
-  } else {
-    if constexpr (MODE == EPI_GELU_BF16) {
-#pragma unroll
-      for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
-    }
-    uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      uint4 pk;
-      uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
-        pw[j] = *reinterpret_cast<uint32_t*>(&h2);
-      }
-      o4[q] = pk;
-    }
+    o4[q] = pk;
   }
 }
 
@@ -295,7 +258,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
         if (!tile_live(g, m0)) continue;
         for (int kb = 0; kb < KB; ++kb, ++q) {
           const int s = q % C::STAGES;
-          mbar_wait(&empty[s], ((q / C::STAGES) & 1u) ^ 1u, g.status);
+          mbar_wait(&empty[s], ((q / C::STAGES) & 1u) ^ 1u, g.status, g.wait_limit);
           uint8_t* sa = smem + s * C::STAGE_BYTES;
           mbar_expect_tx(&full[s], C::STAGE_BYTES);
           tma_load_2d(sa, &tmA, kb * BK, m0, &full[s]);
@@ -309,12 +272,12 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
         if (!tile_live(g, (tile / n_tiles) * BM)) continue;
         const uint32_t acc = it & 1u;
-        mbar_wait(&tempty[acc], ((it >> 1) & 1u) ^ 1u, g.status);
+        mbar_wait(&tempty[acc], ((it >> 1) & 1u) ^ 1u, g.status, g.wait_limit);
         tc_fence_after();
         const uint32_t d = tmem + acc * BN;
         for (int kb = 0; kb < KB; ++kb, ++q) {
           const int s = q % C::STAGES;
-          mbar_wait(&full[s], (q / C::STAGES) & 1u, g.status);
+          mbar_wait(&full[s], (q / C::STAGES) & 1u, g.status, g.wait_limit);
           tc_fence_after();
           const uint32_t sa = su32(smem + s * C::STAGE_BYTES);
           const uint64_t da = sw128_desc(sa), db = sw128_desc(sa + A_BYTES);
@@ -336,10 +299,10 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
       if (!tile_live(g, m0)) continue;
       const uint32_t acc = it & 1u;
-      mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status);
+      mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status, g.wait_limit);
       tc_fence_after();
       const int row = m0 + quad * 32 + lane;
-      const bool live = MODE == EPI_RESID ? row_refreshes(g, row) : row < g.rows;
+      const bool live = row < g.rows;
 #pragma unroll 1
       for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
         float v[32];
@@ -354,6 +317,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
   }
   __syncwarp();
   pdl_trigger();                           // the next kernel may launch while this one drains
+  settle_after_timeout(g.status, false);   // after a timeout, copies and MMAs may still be in flight
   tc_fence_before();
   __syncthreads();
   if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);

@@ -6,21 +6,22 @@
 //
 // Per call:
 //   first_kernel      for every lattice and unit, the first step that refreshes it
-//   init_kernel       x <- noise[0]; a <- x W_in + b_in + P_pos
-//   for t in 0..T-1:
-//     for every unit b that some lattice refreshes at t (Eq. 1, (b,t) in S):
-//       prep_kernel   rows: a += c_k for the units k since the previous prep that
-//                     the row's lattice skipped (a cache that was never written
-//                     holds zero: skipped); then LN_b(a) -> xln for refreshing rows
-//       SA:  GEMM xln W_qkv (bf16 out) -> attention (causal) -> GEMM attn W_o (+= a, -> c_b)
-//       CA:  GEMM xln W_q -> attention (memory tokens) -> GEMM attn W_o (+= a, -> c_b)
-//       FFN: GEMM xln W_1 (GELU, bf16 out) -> GEMM h W_2 (+= a, -> c_b)
-//     head_kernel     pending skips, LN_f, eps = . W_head + b_head, sampler step
-//                     (DDPM / DDIM), next step's input embedding
-// A tile of rows none of whose lattices refresh the unit is skipped inside the
-// GEMM; the residual epilogue touches only refreshing rows.  Rows of one
-// lattice are contiguous (samples are ordered by lattice), so with the batch
-// sizes this path serves a 128-row tile rarely mixes lattices.
+//   walk_kernel       (start) x <- noise[0]; a <- x W_in + b_in + P_pos; walk to
+//                     the first refreshed cell
+//   for every cell (t, b) that some lattice refreshes (Eq. 1, (b,t) in S), in loop order:
+//     SA:  GEMM xln W_qkv (bf16 out) -> attention (causal) -> resid_kernel -> walk_kernel
+//     CA:  GEMM xln W_q -> attention (memory tokens) -> resid_kernel -> walk_kernel
+//     FFN: GEMM xln W_1 (GELU, bf16 out) -> resid_kernel (W_2) -> walk_kernel
+//   resid_kernel      the unit's output projection over whole rows: a += r and
+//                     c_b <- bf16(r) for the rows that refresh the unit
+//   walk_kernel       one warp per row, from the unit just computed to the next
+//                     refreshed cell: the skipped units' cache adds, at step ends
+//                     LN_f, eps = . W_head + b_head, the sampler step (DDPM /
+//                     DDIM) and the next step's input embedding, and finally the
+//                     LayerNorm of the next refreshed unit -> xln (bf16)
+// The GEMMs skip 128-row tiles none of whose lattices refresh the unit.  Rows
+// of one lattice are contiguous (samples are ordered by lattice), so with the
+// batch sizes this path serves a 128-row tile rarely mixes lattices.
 
 #include <cuda.h>
 
@@ -116,19 +117,26 @@ __global__ void first_kernel(Lat L, int n_sched, int* first) {
   (void)n_sched;
 }
 
-// ---------------------------------------------------------------- row kernels (one warp per row)
-struct RowArgs {
+// ---------------------------------------------------------------- the row walk (one warp per row)
+// Between two refreshed lattice cells nothing but per-row work happens: the
+// skipped units' cached outputs are added (Eq. 1), and at the end of a step
+// the final LayerNorm, the output projection, the sampler step and the next
+// step's input embedding.  The walk does all of it for one action-token row
+// held in registers -- lane l owns columns 4 l + 128 j (j < NV = E / 128), one
+// float4 each -- from the position after the unit just computed up to the next
+// cell that some lattice refreshes (or the end of the call), then writes the
+// stream back and, if the row's lattice refreshes that cell, the LayerNorm of
+// its unit as the next GEMM's bf16 operand.
+struct Walk {
   Lat lat;
-  int rows, E, A, t;
-  float* a;                       // [rows][E]
-  const __nv_bfloat16* cache;     // [U][rmax][E]
+  int rows, E, A;
+  float* a;                       // [rows][E] residual stream, fp32
+  __nv_bfloat16* cache;           // [U][rmax][E]
   long long cache_unit;           // elements per unit
-  int lo, b;                      // pending skips over units [lo, b); b < U: LayerNorm of unit b
-  const float* gamma;
-  const float* beta;
   __nv_bfloat16* xln;             // [rows][E]
-  // head / embedding
-  float* x;                       // [samples][H][A] (= rows x A)
+  const float* ln_g;              // [U][E]: LayerNorm gain of every unit's branch
+  const float* ln_b;              // [U][E]
+  float* x;                       // [samples][H][A] (= rows x A): running sample, final actions
   const float* noise;             // [n_noise][obs_mod][H][A]
   int obs_mod;
   const float* stab;              // [T][8]
@@ -140,56 +148,12 @@ struct RowArgs {
   const float* in_w;              // [A][E]
   const float* in_b;              // [E]
   const float* pos;               // [H][E]
+  const float* bias;              // [E]: output bias of the unit computed by the launch (resid kernel)
+  float* trace;                   // [T][U][rows][E] or null: the residual added at every cell (debug)
+  int* status;                    // device status word (index checks of the debug build)
+  int t0, b0;                     // the unit whose output the launch adds (b0 < 0: start of the call)
+  int t1, b1;                     // the next cell some lattice refreshes (t1 = T: none, the call ends)
 };
-
-// Row layout of the warp-per-row kernels: lane owns columns
-// [256 j + 8 lane, 256 j + 8 lane + 8) for j < NV = E / 256, so a row of the
-// fp32 stream is two float4 per lane and chunk, a bf16 cache row one uint4.
-template <int NV>
-struct RowV {
-  float v[NV][8];
-};
-
-template <int NV>
-__device__ __forceinline__ void load_row(const float* src, int lane, RowV<NV>& r) {
-#pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    const float4* s4 = reinterpret_cast<const float4*>(src + 256 * j + 8 * lane);
-    const float4 a = s4[0], b = s4[1];
-    r.v[j][0] = a.x; r.v[j][1] = a.y; r.v[j][2] = a.z; r.v[j][3] = a.w;
-    r.v[j][4] = b.x; r.v[j][5] = b.y; r.v[j][6] = b.z; r.v[j][7] = b.w;
-  }
-}
-
-template <int NV>
-__device__ __forceinline__ void store_row(float* dst, int lane, const RowV<NV>& r) {
-#pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    float4* d4 = reinterpret_cast<float4*>(dst + 256 * j + 8 * lane);
-    d4[0] = make_float4(r.v[j][0], r.v[j][1], r.v[j][2], r.v[j][3]);
-    d4[1] = make_float4(r.v[j][4], r.v[j][5], r.v[j][6], r.v[j][7]);
-  }
-}
-
-__device__ __forceinline__ void add_bf16x8(float* v, uint4 raw) {
-  const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
-    v[2 * i] += f.x;
-    v[2 * i + 1] += f.y;
-  }
-}
-
-__device__ __forceinline__ uint4 pack_bf16x8(const float* v) {
-  uint32_t w[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-    w[i] = *reinterpret_cast<uint32_t*>(&h);
-  }
-  return make_uint4(w[0], w[1], w[2], w[3]);
-}
 
 __device__ __forceinline__ float warp_sum(float s) {
 #pragma unroll
@@ -197,167 +161,167 @@ __device__ __forceinline__ float warp_sum(float s) {
   return s;
 }
 
-// a += c_k for the pending units [lo, b) this row's lattice skipped and that
-// hold a value; the cache rows of up to four units are in flight at once
 template <int NV>
-__device__ __forceinline__ bool pending_skips(const RowArgs& p, int row, int sample, int lane, RowV<NV>& r) {
+__device__ __forceinline__ void ld4(float4 (&v)[NV], const float* src, int lane) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) v[j] = *reinterpret_cast<const float4*>(src + 128 * j + 4 * lane);
+}
+
+template <int NV>
+__device__ __forceinline__ void st4(float* dst, int lane, const float4 (&v)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) *reinterpret_cast<float4*>(dst + 128 * j + 4 * lane) = v[j];
+}
+
+__device__ __forceinline__ void add_bf16x4(float4& v, uint2 raw) {
+  const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
+  const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
+  v.x += lo.x;
+  v.y += lo.y;
+  v.z += hi.x;
+  v.w += hi.y;
+}
+
+__device__ __forceinline__ uint2 pack_bf16x4(float4 v) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(v.x, v.y), hi = __floats2bfloat162_rn(v.z, v.w);
+  return make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
+}
+
+// v += c_k for the units k in [b, bend) that the row's lattice skips at step t
+// and whose cache holds a value, in unit order, up to eight cache rows in flight
+template <int NV>
+__device__ __forceinline__ float* trace_row(const Walk& p, int t, int k, int row) {
+  return p.trace + (((long long)t * p.lat.U + k) * p.rows + row) * p.E;
+}
+
+template <int NV>
+__device__ __forceinline__ void skip_run(const Walk& p, int sample, int row, int lane, int t, int b, int bend,
+                                         float4 (&v)[NV]) {
   uint64_t m = 0;
-  for (int k = p.lo; k < p.b; ++k)
-    if (!lat_refresh(p.lat, sample, k, p.t) && lat_valid(p.lat, sample, k, p.t)) m |= 1ull << k;
-  if (!m) return false;
-  const __nv_bfloat16* base = p.cache + (long long)row * p.E + 8 * lane;
+  for (int k = b; k < bend; ++k)
+    if (!lat_refresh(p.lat, sample, k, t) && lat_valid(p.lat, sample, k, t)) m |= 1ull << k;
+  if (p.trace) {
+    // debug: the value every skipped cell adds, as stored (a cache never written adds 0)
+    for (int k = b; k < bend; ++k) {
+      if (lat_refresh(p.lat, sample, k, t)) continue;
+      float4 c[NV];
+#pragma unroll
+      for (int j = 0; j < NV; ++j) {
+        c[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if ((m >> k) & 1ull)
+          add_bf16x4(c[j], *reinterpret_cast<const uint2*>(p.cache + k * p.cache_unit + (long long)row * p.E +
+                                                          128 * j + 4 * lane));
+      }
+      st4<NV>(trace_row<NV>(p, t, k, row), lane, c);
+    }
+  }
+  const __nv_bfloat16* base = p.cache + (long long)row * p.E + 4 * lane;
+  if (!dcheck(bend <= p.lat.U && (long long)row * p.E < p.cache_unit, p.status)) return;
   while (m) {
-    int ks[4];
+    constexpr int BATCH = NV >= 4 ? 4 : 8;   // cache rows in flight (registers: BATCH x NV x 8 bytes per lane)
+    uint2 raw[BATCH][NV];
     int nk = 0;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      ks[q] = m ? __ffsll((long long)m) - 1 : -1;
+    for (int q = 0; q < BATCH; ++q) {
       if (m) {
+        const int k = __ffsll((long long)m) - 1;
         m &= m - 1;
         ++nk;
+#pragma unroll
+        for (int j = 0; j < NV; ++j) raw[q][j] = *reinterpret_cast<const uint2*>(base + k * p.cache_unit + 128 * j);
       }
     }
-    uint4 raw[4][NV];
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
-#pragma unroll
-      for (int j = 0; j < NV; ++j)
-        raw[q][j] = ks[q] >= 0 ? *reinterpret_cast<const uint4*>(base + ks[q] * p.cache_unit + 256 * j)
-                               : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int q = 0; q < BATCH; ++q)
       if (q < nk)
 #pragma unroll
-        for (int j = 0; j < NV; ++j) add_bf16x8(r.v[j], raw[q][j]);
-  }
-  return true;
-}
-
-template <int NV>
-__device__ __forceinline__ void layer_norm(RowV<NV>& r, const float* g, const float* bb, int lane, float invE) {
-  float s = 0.f, s2 = 0.f;
-#pragma unroll
-  for (int j = 0; j < NV; ++j)
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      s += r.v[j][i];
-      s2 += r.v[j][i] * r.v[j][i];
-    }
-  s = warp_sum(s);
-  s2 = warp_sum(s2);
-  const float mean = s * invE;
-  const float rstd = rsqrtf(fmaxf(s2 * invE - mean * mean, 0.f) + 1e-5f);
-#pragma unroll
-  for (int j = 0; j < NV; ++j) {
-    const int col = 256 * j + 8 * lane;
-    const float4 g0 = *reinterpret_cast<const float4*>(g + col), g1 = *reinterpret_cast<const float4*>(g + col + 4);
-    const float4 b0 = *reinterpret_cast<const float4*>(bb + col), b1 = *reinterpret_cast<const float4*>(bb + col + 4);
-    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-    const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) r.v[j][i] = (r.v[j][i] - mean) * rstd * gg[i] + bv[i];
+        for (int j = 0; j < NV; ++j) add_bf16x4(v[j], raw[q][j]);
   }
 }
 
+// mean and 1/sqrt(var + eps) of the row (two passes over the registers)
 template <int NV>
-__global__ void __launch_bounds__(256) prep_kernel(const RowArgs p) {
-  tc::pdl_trigger();
-  tc::pdl_wait();
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (row >= p.rows) return;
-  const int sample = row / p.lat.H;
-  const bool ln = lat_refresh(p.lat, sample, p.b, p.t);
-  RowV<NV> r;
-  float* arow = p.a + (long long)row * p.E;
-  load_row<NV>(arow, lane, r);
-  if (pending_skips<NV>(p, row, sample, lane, r)) store_row<NV>(arow, lane, r);
-  if (!ln) return;
-  layer_norm<NV>(r, p.gamma, p.beta, lane, 1.f / (float)p.E);
-  __nv_bfloat16* dst = p.xln + (long long)row * p.E + 8 * lane;
+__device__ __forceinline__ void row_stats(const float4 (&v)[NV], float invE, float& mean, float& rstd) {
+  float s = 0.f;
 #pragma unroll
-  for (int j = 0; j < NV; ++j) *reinterpret_cast<uint4*>(dst + 256 * j) = pack_bf16x8(r.v[j]);
-}
-
-// a <- sum_a x[a] W_in[a] + b_in + P_pos[token] for this row
-template <int NV>
-__device__ __forceinline__ void embed_row(const RowArgs& p, int row, int lane, float xa_lane) {
-  const int tok = row % p.lat.H;
-  RowV<NV> r;
-  load_row<NV>(p.pos + (long long)tok * p.E, lane, r);
+  for (int j = 0; j < NV; ++j) s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+  mean = warp_sum(s) * invE;
+  float s2 = 0.f;
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
-    const int col = 256 * j + 8 * lane;
-    const float4 b0 = *reinterpret_cast<const float4*>(p.in_b + col), b1 = *reinterpret_cast<const float4*>(p.in_b + col + 4);
-    r.v[j][0] += b0.x; r.v[j][1] += b0.y; r.v[j][2] += b0.z; r.v[j][3] += b0.w;
-    r.v[j][4] += b1.x; r.v[j][5] += b1.y; r.v[j][6] += b1.z; r.v[j][7] += b1.w;
+    const float dx = v[j].x - mean, dy = v[j].y - mean, dz = v[j].z - mean, dw = v[j].w - mean;
+    s2 += (dx * dx + dy * dy) + (dz * dz + dw * dw);
+  }
+  rstd = rsqrtf(warp_sum(s2) * invE + 1e-5f);
+}
+
+template <int NV>
+__device__ __forceinline__ void ln_apply(float4 (&y)[NV], const float4 (&v)[NV], float mean, float rstd,
+                                         const float* g, const float* bb, int lane) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const float4 gg = *reinterpret_cast<const float4*>(g + 128 * j + 4 * lane);
+    const float4 be = *reinterpret_cast<const float4*>(bb + 128 * j + 4 * lane);
+    y[j].x = (v[j].x - mean) * rstd * gg.x + be.x;
+    y[j].y = (v[j].y - mean) * rstd * gg.y + be.y;
+    y[j].z = (v[j].z - mean) * rstd * gg.z + be.z;
+    y[j].w = (v[j].w - mean) * rstd * gg.w + be.w;
+  }
+}
+
+// v <- x W_in + b_in + P_pos[tok] for this row (x: lane a < A holds x_a)
+template <int NV>
+__device__ __forceinline__ void embed(const Walk& p, int tok, int lane, float xa_lane, float4 (&v)[NV]) {
+  float4 pp[NV];
+  ld4<NV>(v, p.in_b, lane);
+  ld4<NV>(pp, p.pos + (long long)tok * p.E, lane);
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    v[j].x += pp[j].x;
+    v[j].y += pp[j].y;
+    v[j].z += pp[j].z;
+    v[j].w += pp[j].w;
   }
   for (int a = 0; a < p.A; ++a) {
     const float xa = __shfl_sync(0xffffffffu, xa_lane, a);
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
-      const float* w = p.in_w + (long long)a * p.E + 256 * j + 8 * lane;
-      const float4 w0 = *reinterpret_cast<const float4*>(w), w1 = *reinterpret_cast<const float4*>(w + 4);
-      r.v[j][0] = fmaf(xa, w0.x, r.v[j][0]); r.v[j][1] = fmaf(xa, w0.y, r.v[j][1]);
-      r.v[j][2] = fmaf(xa, w0.z, r.v[j][2]); r.v[j][3] = fmaf(xa, w0.w, r.v[j][3]);
-      r.v[j][4] = fmaf(xa, w1.x, r.v[j][4]); r.v[j][5] = fmaf(xa, w1.y, r.v[j][5]);
-      r.v[j][6] = fmaf(xa, w1.z, r.v[j][6]); r.v[j][7] = fmaf(xa, w1.w, r.v[j][7]);
+      const float4 w = *reinterpret_cast<const float4*>(p.in_w + (long long)a * p.E + 128 * j + 4 * lane);
+      v[j].x = fmaf(xa, w.x, v[j].x);
+      v[j].y = fmaf(xa, w.y, v[j].y);
+      v[j].z = fmaf(xa, w.z, v[j].z);
+      v[j].w = fmaf(xa, w.w, v[j].w);
     }
   }
-  store_row<NV>(p.a + (long long)row * p.E, lane, r);
 }
 
+// end of step t for this row: eps = LN_f(a) W_head + b_head, the sampler step
+// (x is updated in place), and -- unless t is the last step -- the input
+// embedding of step t + 1 in v.  Returns false after the last step.
 template <int NV>
-__global__ void __launch_bounds__(256) init_kernel(const RowArgs p) {
-  tc::pdl_trigger();
-  tc::pdl_wait();
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (row >= p.rows) return;
-  const int H = p.lat.H, sample = row / H, tok = row % H;
-  float xv = 0.f;
-  if (lane < p.A) {
-    xv = p.noise[((long long)(sample % p.obs_mod) * H + tok) * p.A + lane];
-    p.x[(long long)row * p.A + lane] = xv;
-  }
-  embed_row<NV>(p, row, lane, xv);
-}
-
-constexpr int MAXA = 16;
-
-template <int NV>
-__global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
-  tc::pdl_trigger();
-  tc::pdl_wait();
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (row >= p.rows) return;
-  const int H = p.lat.H, sample = row / H, tok = row % H, t = p.t, A = p.A;
-  RowV<NV> r;
-  load_row<NV>(p.a + (long long)row * p.E, lane, r);
-  pending_skips<NV>(p, row, sample, lane, r);        // a is rebuilt from x for the next step
-  layer_norm<NV>(r, p.lnf_g, p.lnf_b, lane, 1.f / (float)p.E);
-  // eps[a] = sum_e v[e] W_head[e][a] over this lane's columns (coalesced rows
-  // of W_head^T), then one reduction per action dimension
+__device__ __forceinline__ bool head_step(const Walk& p, int row, int sample, int tok, int lane, int t,
+                                          float4 (&v)[NV]) {
+  const int A = p.A, H = p.lat.H;
+  float mean, rstd;
+  row_stats<NV>(v, 1.f / (float)p.E, mean, rstd);
+  float4 y[NV];
+  ln_apply<NV>(y, v, mean, rstd, p.lnf_g, p.lnf_b, lane);
   float eps = 0.f;
   for (int a = 0; a < A; ++a) {
-    const float* w = p.head_wt + (long long)a * p.E + 8 * lane;
     float part = 0.f;
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
-      const float4 w0 = *reinterpret_cast<const float4*>(w + 256 * j);
-      const float4 w1 = *reinterpret_cast<const float4*>(w + 256 * j + 4);
-      part = fmaf(r.v[j][0], w0.x, part);
-      part = fmaf(r.v[j][1], w0.y, part);
-      part = fmaf(r.v[j][2], w0.z, part);
-      part = fmaf(r.v[j][3], w0.w, part);
-      part = fmaf(r.v[j][4], w1.x, part);
-      part = fmaf(r.v[j][5], w1.y, part);
-      part = fmaf(r.v[j][6], w1.z, part);
-      part = fmaf(r.v[j][7], w1.w, part);
+      const float4 w = *reinterpret_cast<const float4*>(p.head_wt + (long long)a * p.E + 128 * j + 4 * lane);
+      part = fmaf(y[j].x, w.x, part);
+      part = fmaf(y[j].y, w.y, part);
+      part = fmaf(y[j].z, w.z, part);
+      part = fmaf(y[j].w, w.w, part);
     }
     part = warp_sum(part);
     if (lane == a) eps = part + p.head_b[a];
   }
   float xn = 0.f;
-  if (lane < A) {
+  if (lane < A && dcheck(row < p.rows && t < p.lat.T, p.status)) {
     const float* tb = p.stab + t * 8;
     const float inv_sa = tb[0], s1 = tb[1], cx0 = tb[2], cxt = tb[3], sig = tb[4], sab = tb[5], sabp = tb[6],
                 s1p = tb[7];
@@ -372,7 +336,239 @@ __global__ void __launch_bounds__(256) head_kernel(const RowArgs p) {
     }
     p.x[(long long)row * A + lane] = xn;
   }
-  if (t + 1 < p.lat.T) embed_row<NV>(p, row, lane, xn);
+  if (t + 1 >= p.lat.T) return false;
+  embed<NV>(p, tok, lane, xn, v);
+  return true;
+}
+
+// Walk the row from step t, unit b (v = the stream before unit b) to the
+// launch's next refreshed cell (t1, b1), or to the end of the call.
+template <int NV>
+__device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t, int b, float4 (&v)[NV]) {
+  const int sample = row / p.lat.H, tok = row - sample * p.lat.H;
+  for (;;) {
+    const bool last = t == p.t1;
+    const int bend = last ? p.b1 : p.lat.U;
+    if (b < bend) skip_run<NV>(p, sample, row, lane, t, b, bend, v);
+    if (last) break;
+    if (!head_step<NV>(p, row, sample, tok, lane, t, v)) return;   // the call's last step: x is final
+    ++t;
+    b = 0;
+  }
+  if (!dcheck(row < p.rows && p.b1 < p.lat.U && p.t1 < p.lat.T, p.status)) return;
+  st4<NV>(p.a + (long long)row * p.E, lane, v);
+  if (lat_refresh(p.lat, sample, p.b1, p.t1)) {
+    float mean, rstd;
+    row_stats<NV>(v, 1.f / (float)p.E, mean, rstd);
+    float4 y[NV];
+    ln_apply<NV>(y, v, mean, rstd, p.ln_g + (long long)p.b1 * p.E, p.ln_b + (long long)p.b1 * p.E, lane);
+    __nv_bfloat16* dst = p.xln + (long long)row * p.E + 4 * lane;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) *reinterpret_cast<uint2*>(dst + 128 * j) = pack_bf16x4(y[j]);
+  }
+}
+
+// One warp per row: the walk from the launch's position to the next refreshed
+// cell.  b0 < 0: the start of a call (x <- noise[0]; a <- x W_in + b_in +
+// P_pos).  Otherwise the stream already holds unit b0's output for the rows
+// that refresh it (resid_kernel); the walk starts at b0, so rows that skip b0
+// add its cache.
+template <int NV>
+__global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (row >= p.rows) return;
+  float4 v[NV];
+  if (p.b0 < 0) {
+    const int H = p.lat.H, sample = row / H, tok = row % H;
+    float xv = 0.f;
+    if (lane < p.A) {
+      xv = p.noise[((long long)(sample % p.obs_mod) * H + tok) * p.A + lane];
+      p.x[(long long)row * p.A + lane] = xv;
+    }
+    embed<NV>(p, tok, lane, xv, v);
+    walk_row<NV>(p, row, lane, 0, 0, v);
+  } else {
+    ld4<NV>(v, p.a + (long long)row * p.E, lane);
+    walk_row<NV>(p, row, lane, p.t0, p.b0, v);
+  }
+}
+
+// ---------------------------------------------------------------- residual GEMM
+// r = att W_o + b_o (attention units) or h W_2 + b_2 (FFN) for a 128-row tile
+// and ALL n_emb columns: the accumulator is one 128 x E block of tensor memory
+// (E / 256 MMAs of N = 256 per k-step).  The epilogue drains 32 rows at a time
+// into a padded shared-memory tile (thread = row), then the eight epilogue
+// warps take the rows (warp = row, coalesced): a += r and c_b <- bf16(r) for
+// the rows that refresh the unit.  Each warp loads its rows of the stream
+// before the accumulator is ready.  Tiles where no row refreshes the unit are
+// skipped; the row walk that follows adds c_b for rows that skip it.
+template <int E>
+struct ResidCfg {
+  static constexpr int NV = E / 128;
+  static constexpr int B_BYTES = E * tc::BK * 2;
+  static constexpr int STAGE_BYTES = tc::A_BYTES + B_BYTES;
+  static constexpr int STAGES = E == 512 ? 2 : 4;
+  static constexpr int STG_LD = E + 4;                       // staging row stride (floats): conflict-free float4
+  static constexpr int STG_BYTES = 32 * STG_LD * 4;
+  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + STG_BYTES + 256;
+  static constexpr uint32_t IDESC = tc::TileCfg<256>::IDESC;  // M = 128, N = 256
+};
+
+template <int E>
+__global__ void __launch_bounds__(tc::NTHREADS_GEMM, 1) resid_kernel(const __grid_constant__ CUtensorMap tmA,
+                                                                     const __grid_constant__ CUtensorMap tmB,
+                                                                     const tc::GemmArgs g, const Walk p,
+                                                                     int m_tiles) {
+  using C = ResidCfg<E>;
+  constexpr int NV = C::NV;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  float* stg = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES + C::STG_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint64_t* tempty = tfull + 1;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tempty + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp == 1) tc::tmem_alloc(tslot, E);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      tc::mbar_init1(&full[s], 1);
+      tc::mbar_init1(&empty[s], 1);
+    }
+    tc::mbar_init1(tfull, 1);
+    tc::mbar_init1(tempty, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  tc::pdl_wait();                          // A, the residual stream, caches and lattices come from earlier kernels
+  const uint32_t tmem = *tslot;
+  const int KB = g.K / tc::BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t q = 0;
+      for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
+        const int m0 = tile * tc::BM;
+        if (!tc::tile_live(g, m0)) continue;
+        for (int kb = 0; kb < KB; ++kb, ++q) {
+          const int s = q % C::STAGES;
+          tc::mbar_wait(&empty[s], ((q / C::STAGES) & 1u) ^ 1u, g.status, g.wait_limit);
+          uint8_t* sa = smem + s * C::STAGE_BYTES;
+          tc::mbar_expect_tx(&full[s], C::STAGE_BYTES);
+          tc::tma_load_2d(sa, &tmA, kb * tc::BK, m0, &full[s]);
+#pragma unroll
+          for (int h = 0; h < E / 256; ++h)
+            tc::tma_load_2d(sa + tc::A_BYTES + h * 256 * tc::BK * 2, &tmB, kb * tc::BK, g.b_row0 + h * 256, &full[s]);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      uint32_t q = 0, it = 0;
+      for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
+        if (!tc::tile_live(g, tile * tc::BM)) continue;
+        tc::mbar_wait(tempty, (it & 1u) ^ 1u, g.status, g.wait_limit);
+        tc::tc_fence_after();
+        for (int kb = 0; kb < KB; ++kb, ++q) {
+          const int s = q % C::STAGES;
+          tc::mbar_wait(&full[s], (q / C::STAGES) & 1u, g.status, g.wait_limit);
+          tc::tc_fence_after();
+          const uint32_t sa = tc::su32(smem + s * C::STAGE_BYTES);
+          const uint64_t da = tc::sw128_desc(sa);
+#pragma unroll
+          for (int h = 0; h < E / 256; ++h) {
+            const uint64_t db = tc::sw128_desc(sa + tc::A_BYTES + h * 256 * tc::BK * 2);
+#pragma unroll
+            for (int k = 0; k < tc::BK / 16; ++k)   // +32 bytes along K = +2 in the encoded start address
+              tc::mma_f16(tmem + h * 256, da + 2 * k, db + 2 * k, C::IDESC, (kb | k) != 0);
+          }
+          tc::mma_commit(&empty[s]);
+        }
+        tc::mma_commit(tfull);
+        ++it;
+      }
+    }
+  } else {
+    // epilogue warps 2..9: TMEM lane quadrant (warp % 4), column half (warp - 2) / 4;
+    // in the row phase warp ew takes rows ew, ew + 8, ew + 16, ew + 24 of the group
+    const int ew = warp - 2, quad = warp & 3, half = ew >> 2;
+    uint32_t it = 0;
+    for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
+      const int m0 = tile * tc::BM;
+      if (!tc::tile_live(g, m0)) continue;   // no row refreshes the unit: the walk adds its cache
+      for (int grp = 0; grp < 4; ++grp) {
+        // this warp's rows of the group: which refresh the unit, and their stream
+        // (loaded before the accumulator is drained; the loads do not depend on it)
+        float4 v[4][NV];
+        bool ref[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int row = m0 + grp * 32 + ew + 8 * i;
+          ref[i] = row < p.rows && lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0);
+          if (ref[i]) ld4<NV>(v[i], p.a + (long long)row * E, lane);
+        }
+        if (grp == 0) {
+          tc::mbar_wait(tfull, it & 1u, g.status, g.wait_limit);
+          tc::tc_fence_after();
+        }
+        if (quad == grp) {
+          // thread = tile row 32 grp + lane: its half of the columns into the staging tile
+#pragma unroll 1
+          for (int c = half * (E / 64); c < (half + 1) * (E / 64); ++c) {
+            float r[32];
+            tc::tmem_ld32(tmem + ((uint32_t)(grp * 32) << 16) + (uint32_t)(c * 32), r);
+            float4* d = reinterpret_cast<float4*>(stg + lane * C::STG_LD + c * 32);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) d[q] = make_float4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
+          }
+          tc::tc_fence_before();
+        }
+        asm volatile("bar.sync 1, 256;" ::: "memory");
+        if (grp == 3 && ew == 0 && lane == 0) {
+          tc::tc_fence_after();
+          tc::mbar_arrive1(tempty);          // the accumulator is drained: the next tile's MMAs may start
+        }
+        float4 bb[NV];
+        ld4<NV>(bb, p.bias, lane);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if (!ref[i]) continue;
+          const int rr = ew + 8 * i, row = m0 + grp * 32 + rr;
+          if (!dcheck(p.b0 >= 0 && p.b0 < p.lat.U && (long long)row * E < p.cache_unit, g.status)) continue;
+          __nv_bfloat16* crow = p.cache + (long long)p.b0 * p.cache_unit + (long long)row * E + 4 * lane;
+#pragma unroll
+          for (int j = 0; j < NV; ++j) {
+            float4 r = *reinterpret_cast<const float4*>(stg + rr * C::STG_LD + 128 * j + 4 * lane);
+            r.x += bb[j].x;
+            r.y += bb[j].y;
+            r.z += bb[j].z;
+            r.w += bb[j].w;
+            *reinterpret_cast<uint2*>(crow + 128 * j) = pack_bf16x4(r);
+            if (p.trace) *reinterpret_cast<float4*>(trace_row<NV>(p, p.t0, p.b0, row) + 128 * j + 4 * lane) = r;
+            v[i][j].x += r.x;
+            v[i][j].y += r.y;
+            v[i][j].z += r.z;
+            v[i][j].w += r.w;
+          }
+          st4<NV>(p.a + (long long)row * E, lane, v[i]);
+        }
+        asm volatile("bar.sync 1, 256;" ::: "memory");   // the staging tile is free for the next group
+      }
+      ++it;
+    }
+  }
+  __syncwarp();
+  tc::pdl_trigger();                       // the next kernel may launch while this one drains
+  settle_after_timeout(g.status, false);   // after a timeout, copies and MMAs may still be in flight
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) tc::tmem_dealloc(tmem, E);
 }
 
 // ---------------------------------------------------------------- attention
@@ -604,10 +800,12 @@ struct WideState {
   __nv_bfloat16* cache = nullptr;   // [U][rmax][E]
   float* a = nullptr;               // [rmax][E]
   float* head_wt = nullptr;         // [A][E]
+  float* ln_gb = nullptr;           // [2][U][E]: LayerNorm gain and shift of every unit's branch
   int* first = nullptr;             // [max_sched][U]
   CUtensorMap mA_xln, mA_att, mA_hid;
   BMaps mB_e, mB_4e;
   int num_sms = 0;
+  GuardList guards;                 // guard bands of the activation buffers
   std::vector<uint8_t> any;         // [U][T] scratch: some lattice refreshes (b, t)
   long long launches = 0;
 };
@@ -660,23 +858,33 @@ cudaError_t gemm_attr() {
                               tc::TileCfg<BN>::SMEM_BYTES);
 }
 
-template <int NV>
-cudaError_t launch_rows(int which, const RowArgs& p, bool pdl, cudaStream_t st) {
-  const int blocks = (p.rows + 7) / 8;
-  if (which == 0) return launch_pdl(pdl, init_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
-  if (which == 1) return launch_pdl(pdl, prep_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
-  return launch_pdl(pdl, head_kernel<NV>, dim3(blocks), dim3(256), 0, st, p);
+cudaError_t walk(const Walk& p, bool pdl, cudaStream_t st) {
+  const dim3 grid((p.rows + 7) / 8), block(256);
+  if (p.E == 256) return launch_pdl(pdl, walk_kernel<2>, grid, block, 0, st, p);
+  if (p.E == 512) return launch_pdl(pdl, walk_kernel<4>, grid, block, 0, st, p);
+  return cudaErrorInvalidValue;
 }
 
-cudaError_t rows_kernel(int which, const RowArgs& p, bool pdl, cudaStream_t st) {
-  switch (p.E / 256) {
-    case 1: return launch_rows<1>(which, p, pdl, st);
-    case 2: return launch_rows<2>(which, p, pdl, st);
-    default: return cudaErrorInvalidValue;
-  }
+template <int E>
+cudaError_t resid_attr() {
+  return cudaFuncSetAttribute(resid_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, ResidCfg<E>::SMEM_BYTES);
+}
+
+// the residual GEMM of one refreshed unit and the walk to the next refreshed cell
+cudaError_t resid(const CUtensorMap& ma, const BMaps& mb, const tc::GemmArgs& g, const Walk& p, int rows_p,
+                  int num_sms, bool pdl, cudaStream_t st) {
+  const int m_tiles = rows_p / tc::BM;
+  const dim3 grid(std::min(m_tiles, num_sms)), block(tc::NTHREADS_GEMM);
+  if (p.E == 256)
+    return launch_pdl(pdl, resid_kernel<256>, grid, block, ResidCfg<256>::SMEM_BYTES, st, ma, mb.n256, g, p, m_tiles);
+  if (p.E == 512)
+    return launch_pdl(pdl, resid_kernel<512>, grid, block, ResidCfg<512>::SMEM_BYTES, st, ma, mb.n256, g, p, m_tiles);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
+
+constexpr int MAXA = 16;
 
 bool wide_supported(const evo_config* c) {
   const int E = c->n_emb, dh = E / c->n_head;
@@ -752,12 +960,31 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     if (cudaMemcpy(w->head_wt, ht.data(), ht.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(EVO_ERR_CUDA);
   }
-  if (cudaMalloc(&w->xln, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMalloc(&w->qkv, R * 3 * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMalloc(&w->att, R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMalloc(&w->hid, R * 4 * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMalloc(&w->cache, (size_t)w->U * R * E * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
-  if (cudaMalloc(&w->a, R * E * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+  {
+    static const int ln_g[3] = {WL_LN1G, WL_LN2G, WL_LN3G}, ln_b[3] = {WL_LN1B, WL_LN2B, WL_LN3B};
+    const int U = w->U;
+    std::vector<float> gb((size_t)2 * U * E);
+    for (int b = 0; b < U; ++b) {
+      const float* base = weights + woff[W_LAYER0] + (size_t)(b / 3) * woff[W_LAYER_STRIDE];
+      std::memcpy(&gb[(size_t)b * E], base + woff[ln_g[b % 3]], (size_t)E * 4);
+      std::memcpy(&gb[((size_t)U + b) * E], base + woff[ln_b[b % 3]], (size_t)E * 4);
+    }
+    if (cudaMalloc(&w->ln_gb, gb.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMemcpy(w->ln_gb, gb.data(), gb.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(EVO_ERR_CUDA);
+  }
+  if (guarded_malloc(reinterpret_cast<void**>(&w->xln), R * E * 2, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
+  if (guarded_malloc(reinterpret_cast<void**>(&w->qkv), R * 3 * E * 2, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
+  if (guarded_malloc(reinterpret_cast<void**>(&w->att), R * E * 2, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
+  if (guarded_malloc(reinterpret_cast<void**>(&w->hid), R * 4 * E * 2, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
+  if (guarded_malloc(reinterpret_cast<void**>(&w->cache), (size_t)w->U * R * E * 2, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
+  if (guarded_malloc(reinterpret_cast<void**>(&w->a), R * E * 4, &w->guards) != cudaSuccess)
+    return fail(EVO_ERR_OOM);
   if (cudaMalloc(&w->first, (size_t)max_sched * w->U * sizeof(int)) != cudaSuccess) return fail(EVO_ERR_OOM);
   // operand rows that no call writes (padding up to a tile) read as zero
   cudaMemset(w->xln, 0, R * E * 2);
@@ -772,7 +999,7 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     return fail(EVO_ERR_CUDA);
   if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
       gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
-      gemm_attr<tc::EPI_RESID, 128>() != cudaSuccess || gemm_attr<tc::EPI_RESID, 256>() != cudaSuccess)
+      resid_attr<256>() != cudaSuccess || resid_attr<512>() != cudaSuccess)
     return fail(EVO_ERR_CUDA);
   {
     int dev = 0;
@@ -792,18 +1019,20 @@ void wide_destroy(WideState* w) {
   if (!w) return;
   cudaFree(w->wt_e);
   cudaFree(w->wt_4e);
-  cudaFree(w->xln);
-  cudaFree(w->qkv);
-  cudaFree(w->att);
-  cudaFree(w->hid);
-  cudaFree(w->cache);
-  cudaFree(w->a);
+  guarded_free(w->xln);
+  guarded_free(w->qkv);
+  guarded_free(w->att);
+  guarded_free(w->hid);
+  guarded_free(w->cache);
+  guarded_free(w->a);
   cudaFree(w->first);
   cudaFree(w->head_wt);
+  cudaFree(w->ln_gb);
   delete w;
 }
 
 long long wide_rows_capacity(const WideState* w) { return w ? w->rmax : 0; }
+const GuardList* wide_guards(const WideState* w) { return &w->guards; }
 long long wide_last_launches(const WideState* w) { return w ? w->launches : 0; }
 
 cudaError_t wide_run(WideState* w, const WideCall& c) {
@@ -846,28 +1075,51 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   lat.force = w->force;
   WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first));
 
-  RowArgs rp{};
-  rp.lat = lat;
-  rp.rows = (int)R;
-  rp.E = E;
-  rp.A = w->A;
-  rp.a = w->a;
-  rp.cache = w->cache;
-  rp.cache_unit = w->rmax * E;
-  rp.xln = w->xln;
-  rp.x = c.out;
-  rp.noise = c.noise;
-  rp.obs_mod = c.obs_mod;
-  rp.stab = c.stab;
-  rp.sampler = w->sampler;
-  rp.lnf_g = w->wf32 + w->woff[W_LNF_G];
-  rp.lnf_b = w->wf32 + w->woff[W_LNF_B];
-  rp.head_wt = w->head_wt;
-  rp.head_b = w->wf32 + w->woff[W_HEAD_B];
-  rp.in_w = w->wf32 + w->woff[W_IN_W];
-  rp.in_b = w->wf32 + w->woff[W_IN_B];
-  rp.pos = w->wf32 + w->woff[W_POS];
-  WCK(rows_kernel(0, rp, pdl, st));
+  Walk wp{};
+  wp.lat = lat;
+  wp.rows = (int)R;
+  wp.E = E;
+  wp.A = w->A;
+  wp.a = w->a;
+  wp.cache = w->cache;
+  wp.cache_unit = w->rmax * E;
+  wp.xln = w->xln;
+  wp.ln_g = w->ln_gb;
+  wp.ln_b = w->ln_gb + (long long)U * E;
+  wp.x = c.out;
+  wp.noise = c.noise;
+  wp.obs_mod = c.obs_mod;
+  wp.stab = c.stab;
+  wp.sampler = w->sampler;
+  wp.lnf_g = w->wf32 + w->woff[W_LNF_G];
+  wp.lnf_b = w->wf32 + w->woff[W_LNF_B];
+  wp.head_wt = w->head_wt;
+  wp.head_b = w->wf32 + w->woff[W_HEAD_B];
+  wp.in_w = w->wf32 + w->woff[W_IN_W];
+  wp.in_b = w->wf32 + w->woff[W_IN_B];
+  wp.pos = w->wf32 + w->woff[W_POS];
+  wp.trace = c.trace;
+  wp.status = c.status;
+
+  // the cells some lattice refreshes, in loop order; each launch chain walks
+  // from one to the next
+  std::vector<int> cells;
+  for (int t = 0; t < T; ++t)
+    for (int b = 0; b < U; ++b)
+      if (w->any[(size_t)b * T + t]) cells.push_back(t * U + b);
+  auto set_next = [&](size_t i) {
+    if (i < cells.size()) {
+      wp.t1 = cells[i] / U;
+      wp.b1 = cells[i] % U;
+    } else {
+      wp.t1 = T;
+      wp.b1 = 0;
+    }
+  };
+  wp.t0 = 0;
+  wp.b0 = -1;
+  set_next(0);
+  WCK(walk(wp, pdl, st));
 
   tc::GemmArgs g{};
   g.rows = (int)R;
@@ -878,8 +1130,7 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   g.per_sched = c.per_sched;
   g.force = w->force;
   g.status = c.status;
-  g.ldr = E;
-  g.resid = w->a;
+  g.wait_limit = WAIT_POLLS_DEFAULT;
 
   AttnArgs ap{};
   ap.lat = lat;
@@ -898,68 +1149,58 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   const size_t sa_smem = attn_smem_bytes(H, false), ca_smem = attn_smem_bytes(H, true);
   const dim3 attn_grid(c.samples, (w->nh + SA_WARPS - 1) / SA_WARPS);
 
-  for (int t = 0; t < T; ++t) {
-    int lo = 0;
-    rp.t = t;
+  for (size_t i = 0; i < cells.size(); ++i) {
+    const int t = cells[i] / U, b = cells[i] % U, l = b / 3, u = b % 3;
     g.t = t;
+    g.srow = c.S_rows == U ? b : b / 3;
     ap.t = t;
-    for (int b = 0; b < U; ++b) {
-      if (!w->any[(size_t)b * T + t]) continue;
-      const int l = b / 3, u = b % 3;
-      static const int ln_g[3] = {WL_LN1G, WL_LN2G, WL_LN3G}, ln_b[3] = {WL_LN1B, WL_LN2B, WL_LN3B};
-      rp.lo = lo;
-      rp.b = b;
-      rp.gamma = wl(w, l, ln_g[u]);
-      rp.beta = wl(w, l, ln_b[u]);
-      WCK(rows_kernel(1, rp, pdl, st));
-      lo = b;
-      g.srow = c.S_rows == U ? b : b / 3;
-      g.cache = w->cache + (long long)b * w->rmax * E;
-      ap.b = b;
-      ap.l = l;
-      const int rowE = l * 10 * E;
-      if (u == 0) {
-        g.K = E;
-        g.b_row0 = rowE;
-        g.bias = wl(w, l, WL_SA_BQKV);
-        g.out = w->qkv;
-        g.ldo = 3 * E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, pdl, st));
-        ap.qkv = w->qkv;
-        WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, false> : attn_mma_kernel<1, false>, attn_grid,
-                       dim3(SA_WARPS * 32), sa_smem, st, ap));
-        g.b_row0 = rowE + 3 * E;
-        g.bias = wl(w, l, WL_SA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
-      } else if (u == 1) {
-        g.K = E;
-        g.b_row0 = rowE + 4 * E;
-        g.bias = wl(w, l, WL_CA_BQ);
-        g.out = w->qkv;
-        g.ldo = E;
-        WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
-        ap.qkv = w->qkv;
-        WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, true> : attn_mma_kernel<1, true>, attn_grid,
-                       dim3(SA_WARPS * 32), ca_smem, st, ap));
-        g.b_row0 = rowE + 5 * E;
-        g.bias = wl(w, l, WL_CA_BO);
-        WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
-      } else {
-        g.K = E;
-        g.b_row0 = rowE + 6 * E;
-        g.bias = wl(w, l, WL_FF_B1);
-        g.out = w->hid;
-        g.ldo = 4 * E;
-        WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, pdl, st));
-        g.K = 4 * E;
-        g.b_row0 = l * E;
-        g.bias = wl(w, l, WL_FF_B2);
-        WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, pdl, st));
-      }
+    ap.b = b;
+    ap.l = l;
+    wp.t0 = t;
+    wp.b0 = b;
+    set_next(i + 1);
+    const int rowE = l * 10 * E;
+    if (u == 0) {
+      g.K = E;
+      g.b_row0 = rowE;
+      g.bias = wl(w, l, WL_SA_BQKV);
+      g.out = w->qkv;
+      g.ldo = 3 * E;
+      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, pdl, st));
+      ap.qkv = w->qkv;
+      WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, false> : attn_mma_kernel<1, false>, attn_grid,
+                     dim3(SA_WARPS * 32), sa_smem, st, ap));
+      g.b_row0 = rowE + 3 * E;
+      wp.bias = wl(w, l, WL_SA_BO);
+      WCK(resid(w->mA_att, w->mB_e, g, wp, Rp, w->num_sms, pdl, st));
+      WCK(walk(wp, pdl, st));
+    } else if (u == 1) {
+      g.K = E;
+      g.b_row0 = rowE + 4 * E;
+      g.bias = wl(w, l, WL_CA_BQ);
+      g.out = w->qkv;
+      g.ldo = E;
+      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
+      ap.qkv = w->qkv;
+      WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, true> : attn_mma_kernel<1, true>, attn_grid,
+                     dim3(SA_WARPS * 32), ca_smem, st, ap));
+      g.b_row0 = rowE + 5 * E;
+      wp.bias = wl(w, l, WL_CA_BO);
+      WCK(resid(w->mA_att, w->mB_e, g, wp, Rp, w->num_sms, pdl, st));
+      WCK(walk(wp, pdl, st));
+    } else {
+      g.K = E;
+      g.b_row0 = rowE + 6 * E;
+      g.bias = wl(w, l, WL_FF_B1);
+      g.out = w->hid;
+      g.ldo = 4 * E;
+      WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, pdl, st));
+      g.K = 4 * E;
+      g.b_row0 = l * E;
+      wp.bias = wl(w, l, WL_FF_B2);
+      WCK(resid(w->mA_hid, w->mB_4e, g, wp, Rp, w->num_sms, pdl, st));
+      WCK(walk(wp, pdl, st));
     }
-    rp.lo = lo;
-    rp.b = U;
-    WCK(rows_kernel(2, rp, pdl, st));
   }
 #undef WCK
   w->launches = n;

@@ -12,6 +12,8 @@ import pytest
 from oracle import evo_oracle as O
 from paper_2607_20293_gb300 import synth
 
+from eq1_trace import check_reuse
+
 pytestmark = pytest.mark.gpu
 
 TOL = {"fp32": 1e-4, "bf16": 3e-2}
@@ -111,6 +113,23 @@ def test_tiny_trace_eq1(torch, B):
             else:
                 assert not tr[t, b].any()                     # reset cache contributes zero
     assert n_skip > 5
+
+
+@pytest.mark.parametrize("name,n", [("tiny", 2), ("pusht", 1)])
+def test_bf16_trace_eq1_bitwise(torch, B, name, n):
+    """bf16 caches on the cluster path: every skipped cell adds exactly the bf16
+    value stored at that unit's last refresh (Eq. 1), bit for bit."""
+    cfg = synth.config(name, dtype="bf16")
+    W = synth.make_weights(cfg, 0)
+    obs, noise = synth.make_obs(cfg, n, 1), synth.make_noise(cfg, n, 2)
+    ev = B.Evo(cfg, W, n, wide_rows=-1)
+    U, T, H, E = 3 * cfg["n_layer"], cfg["n_steps"], cfg["horizon"], cfg["n_emb"]
+    S = synth.bernoulli_schedule(U, T, 0.3, 22)
+    trace = torch.zeros((T, U, n, H, E), dtype=torch.float32, device="cuda")
+    got = ev.denoise(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(), S, trace=trace).cpu().numpy()
+    assert ev.last_call()["path"] == "cluster"
+    assert check_reuse(trace.cpu().numpy(), S, bf16=True) > 20
+    check(got, O.denoise(W, cfg, obs, noise, S), TOL["bf16"], name)
 
 
 # ------------------------------------------------------------------ Push-T shaped (bf16, DDPM, batch 1)

@@ -12,6 +12,8 @@ import pytest
 from oracle import evo_oracle as O
 from paper_2607_20293_gb300 import synth
 
+from eq1_trace import check_reuse
+
 pytestmark = pytest.mark.gpu
 
 TOL = 3e-2
@@ -124,3 +126,20 @@ def test_wide_population_tiles_mix_lattices(torch, B):
     ref_dev = np.linalg.norm((x - full[None]).reshape(P, N, -1), axis=2).mean(1)
     assert np.allclose(dev, ref_dev, atol=2 * TOL)
     assert dev[5] < 1e-6 * max(1.0, float(dev.max()))      # the all-ones candidate is the reference itself
+
+
+@pytest.mark.parametrize("force", [False, True])
+def test_wide_trace_eq1_bitwise(torch, B, force):
+    """bf16 caches on the batch-wide path: every skipped cell adds exactly the
+    bf16 value stored at the unit's last refresh (Eq. 1), bit for bit, and a
+    unit not refreshed yet adds zero (or, under FORCE, is computed at t = 0)."""
+    kw = {"empty": "force"} if force else {}
+    cfg, W, obs, noise, ev, d_obs, d_noise = make("pusht", 9, torch, B, **kw)
+    S = synth.bernoulli_schedule(24, 100, 0.2, 23)
+    if force:
+        S[:, 0] = 0
+    trace = torch.zeros((100, 24, 9, 16, 256), dtype=torch.float32, device="cuda")
+    got = ev.denoise(d_obs, d_noise, S, trace=trace).cpu().numpy()
+    assert ev.last_call()["path"] == "wide"
+    assert check_reuse(trace.cpu().numpy(), S, bf16=True, force=force) > 100
+    check(got, O.denoise(W, cfg, obs, noise, S, "force" if force else "zero"), "wide trace")
