@@ -13,8 +13,13 @@
 //     accumulator to the epilogue;
 //   * warps 2-9: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
 //     quadrant 32 (w % 4) .. +31 and one half of the tile's columns, 32 at a
-//     time (tcgen05.ld), applies bias (and GELU), stores bf16, and releases the
-//     accumulator.
+//     time (tcgen05.ld), applies bias (and GELU), packs bf16 into its staging
+//     rows in shared memory, and stores 64 columns at a time as whole 128-byte
+//     row segments (a warp-per-row store: the thread-per-row layout of the
+//     accumulator would scatter every store over 32 rows), then releases the
+//     accumulator.  The residual mode (the output projection of a refreshed
+//     unit) stages fp32 and, row by row, adds r to the residual stream and
+//     writes the unit's bf16 cache (Eq. 1) for the rows that refresh the unit.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
 // next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
@@ -36,12 +41,18 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int EPI_WARPS = 8;                                    // two per TMEM lane quadrant
 constexpr int NTHREADS_GEMM = 32 * (2 + EPI_WARPS);             // producer, MMA, epilogue warps
 
+// epilogue staging: per epilogue warp 32 rows x 64 bf16 columns (128-byte rows,
+// 16-byte chunks XOR-swizzled by row so that both the thread-per-row writes and
+// the warp-per-row reads are free of bank conflicts)
+constexpr int EPI_STG_BYTES = EPI_WARPS * 32 * 128;
+
 template <int BN>
 struct TileCfg {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = BN == 256 ? 4 : 6;
-  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;   // alignment slack, stages, barriers
+  // alignment slack, stages, epilogue staging, barriers
+  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_STG_BYTES + 256;
   static constexpr int TMEM_COLS = 2 * BN;                                // two accumulators
   // instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
   // K-major, M = BM, N = BN
@@ -49,14 +60,18 @@ struct TileCfg {
       (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 };
 
-enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1 };
+enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2 };
 
 struct GemmArgs {
   int K;                      // multiple of BK
   int b_row0;                 // first row of B (its tensor map spans every layer's matrices)
   const float* bias;          // [N] fp32
-  __nv_bfloat16* out;         // out[row * ldo + n]
+  __nv_bfloat16* out;         // EPI_BF16 / EPI_GELU_BF16: out[row * ldo + n]
   int ldo;
+  float* resid;               // EPI_RESID: residual stream [rows][ldr] fp32, += r for refreshing rows
+  __nv_bfloat16* cache;       // EPI_RESID: the unit's cache [rows][ldr], <- bf16(r) for refreshing rows
+  float* trace;               // EPI_RESID: [rows][ldr] or null: r of refreshing rows (debug trace)
+  int ldr;
   int rows;                   // real rows; rows >= this are padding
   // refresh gate (null: every row refreshes): row -> sample row / H -> lattice
   // (sample / per_sched); refresh = S[lattice * S_stride + srow * T + t]
@@ -173,6 +188,14 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// the row's lattice refreshes the unit (EPI_RESID writes only such rows)
+__device__ __forceinline__ bool row_refreshes(const GemmArgs& g, int row) {
+  if (row >= g.rows) return false;
+  if (!g.S || (g.force && g.t == 0)) return true;
+  const int sample = row / g.H;
+  return g.S[(long long)(sample / g.per_sched) * g.S_stride + (long long)g.srow * g.T + g.t] != 0;
+}
+
 __device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
 
 // does any row of the tile starting at m0 refresh?  (the same answer in every role)
@@ -185,8 +208,12 @@ __device__ __forceinline__ bool tile_live(const GemmArgs& g, int m0) {
   return false;
 }
 
+// bias (and GELU) on 32 accumulator columns n .. n + 31 of this thread's row,
+// packed to bf16 and written as 64 bytes of the thread's staging row (chunks
+// j4 .. j4 + 3 of 16 bytes, swizzled by the row within the 8-row group)
 template <int MODE>
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n, float (&v)[32]) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int n, float (&v)[32], uint8_t* srow, int lane,
+                                               int j4) {
   const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
@@ -200,7 +227,6 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
   }
-  uint4* o4 = reinterpret_cast<uint4*>(g.out + (long long)row * g.ldo + n);
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     uint4 pk;
@@ -210,8 +236,58 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n
       __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
       pw[j] = *reinterpret_cast<uint32_t*>(&h2);
     }
-    o4[q] = pk;
+    *reinterpret_cast<uint4*>(srow + (((j4 + q) ^ (lane & 7)) << 4)) = pk;
   }
+}
+
+// the warp's staged 32 rows x 64 columns to global memory: 4 rows of 128
+// contiguous bytes per store instruction
+__device__ __forceinline__ void epilogue_flush(const GemmArgs& g, const uint8_t* stg, int row0, int n, int lane) {
+  const int cc = lane & 7;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int r = 4 * i + (lane >> 3);
+    const uint4 val = *reinterpret_cast<const uint4*>(stg + r * 128 + ((cc ^ (r & 7)) << 4));
+    if (row0 + r < g.rows) *reinterpret_cast<uint4*>(g.out + (long long)(row0 + r) * g.ldo + n + 8 * cc) = val;
+  }
+}
+
+// EPI_RESID, one chunk of 32 columns n .. n + 31: r = acc + bias goes to the
+// warp's staging rows (fp32, thread = row), then the warp takes the rows one
+// at a time (lane = column, 128 contiguous bytes): a += r, c_b <- bf16(r) for
+// the rows whose lattice refreshes the unit (bit r of rmask); the stream of 16
+// rows at a time is loaded before any is written.
+__device__ __forceinline__ void epilogue_resid(const GemmArgs& g, int row0, int n, float (&v)[32], uint8_t* stg,
+                                               int lane, unsigned rmask) {
+  const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
+  uint8_t* srow = stg + lane * 128;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 bb = __ldg(b4 + q);
+    *reinterpret_cast<float4*>(srow + ((q ^ (lane & 7)) << 4)) =
+        make_float4(v[4 * q] + bb.x, v[4 * q + 1] + bb.y, v[4 * q + 2] + bb.z, v[4 * q + 3] + bb.w);
+  }
+  __syncwarp();
+  const long long col = n + lane;
+#pragma unroll
+  for (int h = 0; h < 32; h += 16) {
+    float av[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+      av[r] = (rmask >> (h + r)) & 1u ? g.resid[(long long)(row0 + h + r) * g.ldr + col] : 0.f;
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      if (!((rmask >> (h + r)) & 1u)) continue;
+      const int rr = h + r;
+      const float rv =
+          *reinterpret_cast<const float*>(stg + rr * 128 + (((lane >> 2) ^ (rr & 7)) << 4) + (lane & 3) * 4);
+      const long long o = (long long)(row0 + rr) * g.ldr + col;
+      g.resid[o] = av[r] + rv;
+      g.cache[o] = __float2bfloat16_rn(rv);
+      if (g.trace) g.trace[o] = rv;
+    }
+  }
+  __syncwarp();
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -225,7 +301,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES + EPI_STG_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;     // [2]: accumulator ready for the epilogue
   uint64_t* tempty = tfull + 2;            // [2]: accumulator drained by the epilogue
@@ -292,8 +368,9 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
     }
   } else {
     // epilogue warps: TMEM lane quadrant (warp % 4) = tile rows 32 (warp % 4) ..,
-    // column half (warp - 2) / 4
+    // column half (warp - 2) / 4; 64 columns at a time through the warp's staging
     const int quad = warp & 3, half = (warp - 2) >> 2;
+    uint8_t* stg = smem + C::STAGES * C::STAGE_BYTES + (warp - 2) * 32 * 128;
     uint32_t it = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
       const int m0 = (tile / n_tiles) * BM, n0 = (tile % n_tiles) * BN;
@@ -301,13 +378,31 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       const uint32_t acc = it & 1u;
       mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status, g.wait_limit);
       tc_fence_after();
-      const int row = m0 + quad * 32 + lane;
-      const bool live = row < g.rows;
+      if constexpr (MODE == EPI_RESID) {
+        const unsigned rmask = __ballot_sync(0xffffffffu, row_refreshes(g, m0 + quad * 32 + lane));
 #pragma unroll 1
-      for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
-        float v[32];
-        tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
-        if (live) epilogue_chunk<MODE>(g, row, n0 + c * 32, v);
+        for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
+          float v[32];
+          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
+          epilogue_resid(g, m0 + quad * 32, n0 + c * 32, v, stg, lane, rmask);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive1(&tempty[acc]);
+        ++it;
+        continue;
+      }
+#pragma unroll 1
+      for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); c += 2) {
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          float v[32];
+          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)((c + j) * 32), v);
+          epilogue_chunk<MODE>(g, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
+        }
+        __syncwarp();
+        epilogue_flush(g, stg, m0 + quad * 32, n0 + c * 32, lane);
+        __syncwarp();
       }
       tc_fence_before();
       __syncwarp();

@@ -9,11 +9,11 @@
 //   walk_kernel       (start) x <- noise[0]; a <- x W_in + b_in + P_pos; walk to
 //                     the first refreshed cell
 //   for every cell (t, b) that some lattice refreshes (Eq. 1, (b,t) in S), in loop order:
-//     SA:  GEMM xln W_qkv (bf16 out) -> attention (causal) -> resid_kernel -> walk_kernel
-//     CA:  GEMM xln W_q -> attention (memory tokens) -> resid_kernel -> walk_kernel
-//     FFN: GEMM xln W_1 (GELU, bf16 out) -> resid_kernel (W_2) -> walk_kernel
-//   resid_kernel      the unit's output projection over whole rows: a += r and
-//                     c_b <- bf16(r) for the rows that refresh the unit
+//     SA:  GEMM xln W_qkv (bf16 out) -> attention (causal) -> GEMM W_o (residual) -> walk_kernel
+//     CA:  GEMM xln W_q -> attention (memory tokens) -> GEMM W_o (residual) -> walk_kernel
+//     FFN: GEMM xln W_1 (GELU, bf16 out) -> GEMM W_2 (residual) -> walk_kernel
+//   GEMM (residual)   the unit's output projection: a += r and c_b <- bf16(r)
+//                     for the rows that refresh the unit (evo_tc.cuh, EPI_RESID)
 //   walk_kernel       one warp per row, from the unit just computed to the next
 //                     refreshed cell: the skipped units' cache adds, at step ends
 //                     LN_f, eps = . W_head + b_head, the sampler step (DDPM /
@@ -81,6 +81,7 @@ struct Lat {
   const uint8_t* S;     // [n_sched][S_rows][T]
   long long stride;     // bytes per lattice
   const int* first;     // [n_sched][U]: first step that refreshes the unit (T: never)
+  const uint64_t* mask; // [n_sched][T][2]: bit b of [0] = unit b refreshed at t, of [1] = its cache holds a value
   int S_rows, U, T, H, per_sched, force;
 };
 
@@ -95,9 +96,12 @@ __device__ __forceinline__ bool lat_valid(const Lat& L, int sample, int b, int t
   return L.first[(sample / L.per_sched) * L.U + b] < t;
 }
 
-__global__ void first_kernel(Lat L, int n_sched, int* first) {
+// per lattice: the first step that refreshes each unit, and per step the
+// bitmasks of the units it refreshes and of the units whose cache holds a value
+__global__ void first_kernel(Lat L, int n_sched, int* first, uint64_t* mask) {
   tc::pdl_trigger();
   tc::pdl_wait();
+  __shared__ int fs[64];
   const int s = blockIdx.x;
   for (int b = threadIdx.x; b < L.U; b += blockDim.x) {
     int f = L.T;
@@ -113,6 +117,18 @@ __global__ void first_kernel(Lat L, int n_sched, int* first) {
         }
     }
     first[s * L.U + b] = f;
+    fs[b] = f;
+  }
+  __syncthreads();
+  for (int t = threadIdx.x; t < L.T; t += blockDim.x) {
+    uint64_t ref = 0, val = 0;
+    for (int b = 0; b < L.U; ++b) {
+      const int r = L.S_rows == L.U ? b : b / 3;
+      if ((L.force && t == 0) || L.S[(long long)s * L.stride + (long long)r * L.T + t]) ref |= 1ull << b;
+      if (fs[b] < t) val |= 1ull << b;
+    }
+    mask[((long long)s * L.T + t) * 2] = ref;
+    mask[((long long)s * L.T + t) * 2 + 1] = val;
   }
   (void)n_sched;
 }
@@ -148,7 +164,6 @@ struct Walk {
   const float* in_w;              // [A][E]
   const float* in_b;              // [E]
   const float* pos;               // [H][E]
-  const float* bias;              // [E]: output bias of the unit computed by the launch (resid kernel)
   float* trace;                   // [T][U][rows][E] or null: the residual added at every cell (debug)
   int* status;                    // device status word (index checks of the debug build)
   int t0, b0;                     // the unit whose output the launch adds (b0 < 0: start of the call)
@@ -197,9 +212,9 @@ __device__ __forceinline__ float* trace_row(const Walk& p, int t, int k, int row
 template <int NV>
 __device__ __forceinline__ void skip_run(const Walk& p, int sample, int row, int lane, int t, int b, int bend,
                                          float4 (&v)[NV]) {
-  uint64_t m = 0;
-  for (int k = b; k < bend; ++k)
-    if (!lat_refresh(p.lat, sample, k, t) && lat_valid(p.lat, sample, k, t)) m |= 1ull << k;
+  const uint64_t* mk = p.lat.mask + ((long long)(sample / p.lat.per_sched) * p.lat.T + t) * 2;
+  const uint64_t range = (bend >= 64 ? ~0ull : (1ull << bend) - 1ull) & ~((1ull << b) - 1ull);
+  uint64_t m = ~mk[0] & mk[1] & range;                // skipped units whose cache holds a value
   if (p.trace) {
     // debug: the value every skipped cell adds, as stored (a cache never written adds 0)
     for (int k = b; k < bend; ++k) {
@@ -371,8 +386,8 @@ __device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t
 // One warp per row: the walk from the launch's position to the next refreshed
 // cell.  b0 < 0: the start of a call (x <- noise[0]; a <- x W_in + b_in +
 // P_pos).  Otherwise the stream already holds unit b0's output for the rows
-// that refresh it (resid_kernel); the walk starts at b0, so rows that skip b0
-// add its cache.
+// that refresh it (the residual GEMM); the walk starts at b0, so rows that skip
+// b0 add its cache.
 template <int NV>
 __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
   tc::pdl_trigger();
@@ -393,182 +408,6 @@ __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
     ld4<NV>(v, p.a + (long long)row * p.E, lane);
     walk_row<NV>(p, row, lane, p.t0, p.b0, v);
   }
-}
-
-// ---------------------------------------------------------------- residual GEMM
-// r = att W_o + b_o (attention units) or h W_2 + b_2 (FFN) for a 128-row tile
-// and ALL n_emb columns: the accumulator is one 128 x E block of tensor memory
-// (E / 256 MMAs of N = 256 per k-step).  The epilogue drains 32 rows at a time
-// into a padded shared-memory tile (thread = row), then the eight epilogue
-// warps take the rows (warp = row, coalesced): a += r and c_b <- bf16(r) for
-// the rows that refresh the unit.  Each warp loads its rows of the stream
-// before the accumulator is ready.  Tiles where no row refreshes the unit are
-// skipped; the row walk that follows adds c_b for rows that skip it.
-template <int E>
-struct ResidCfg {
-  static constexpr int NV = E / 128;
-  static constexpr int B_BYTES = E * tc::BK * 2;
-  static constexpr int STAGE_BYTES = tc::A_BYTES + B_BYTES;
-  static constexpr int STAGES = E == 512 ? 2 : 4;
-  static constexpr int STG_LD = E + 4;                       // staging row stride (floats): conflict-free float4
-  static constexpr int STG_BYTES = 32 * STG_LD * 4;
-  static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + STG_BYTES + 256;
-  static constexpr uint32_t IDESC = tc::TileCfg<256>::IDESC;  // M = 128, N = 256
-};
-
-template <int E>
-__global__ void __launch_bounds__(tc::NTHREADS_GEMM, 1) resid_kernel(const __grid_constant__ CUtensorMap tmA,
-                                                                     const __grid_constant__ CUtensorMap tmB,
-                                                                     const tc::GemmArgs g, const Walk p,
-                                                                     int m_tiles) {
-  using C = ResidCfg<E>;
-  constexpr int NV = C::NV;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  float* stg = reinterpret_cast<float*>(smem + C::STAGES * C::STAGE_BYTES);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES + C::STG_BYTES);
-  uint64_t* empty = full + C::STAGES;
-  uint64_t* tfull = empty + C::STAGES;
-  uint64_t* tempty = tfull + 1;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(tempty + 1);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (warp == 1) tc::tmem_alloc(tslot, E);
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < C::STAGES; ++s) {
-      tc::mbar_init1(&full[s], 1);
-      tc::mbar_init1(&empty[s], 1);
-    }
-    tc::mbar_init1(tfull, 1);
-    tc::mbar_init1(tempty, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  tc::tc_fence_after();
-  tc::pdl_wait();                          // A, the residual stream, caches and lattices come from earlier kernels
-  const uint32_t tmem = *tslot;
-  const int KB = g.K / tc::BK;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      uint32_t q = 0;
-      for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
-        const int m0 = tile * tc::BM;
-        if (!tc::tile_live(g, m0)) continue;
-        for (int kb = 0; kb < KB; ++kb, ++q) {
-          const int s = q % C::STAGES;
-          tc::mbar_wait(&empty[s], ((q / C::STAGES) & 1u) ^ 1u, g.status, g.wait_limit);
-          uint8_t* sa = smem + s * C::STAGE_BYTES;
-          tc::mbar_expect_tx(&full[s], C::STAGE_BYTES);
-          tc::tma_load_2d(sa, &tmA, kb * tc::BK, m0, &full[s]);
-#pragma unroll
-          for (int h = 0; h < E / 256; ++h)
-            tc::tma_load_2d(sa + tc::A_BYTES + h * 256 * tc::BK * 2, &tmB, kb * tc::BK, g.b_row0 + h * 256, &full[s]);
-        }
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      uint32_t q = 0, it = 0;
-      for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
-        if (!tc::tile_live(g, tile * tc::BM)) continue;
-        tc::mbar_wait(tempty, (it & 1u) ^ 1u, g.status, g.wait_limit);
-        tc::tc_fence_after();
-        for (int kb = 0; kb < KB; ++kb, ++q) {
-          const int s = q % C::STAGES;
-          tc::mbar_wait(&full[s], (q / C::STAGES) & 1u, g.status, g.wait_limit);
-          tc::tc_fence_after();
-          const uint32_t sa = tc::su32(smem + s * C::STAGE_BYTES);
-          const uint64_t da = tc::sw128_desc(sa);
-#pragma unroll
-          for (int h = 0; h < E / 256; ++h) {
-            const uint64_t db = tc::sw128_desc(sa + tc::A_BYTES + h * 256 * tc::BK * 2);
-#pragma unroll
-            for (int k = 0; k < tc::BK / 16; ++k)   // +32 bytes along K = +2 in the encoded start address
-              tc::mma_f16(tmem + h * 256, da + 2 * k, db + 2 * k, C::IDESC, (kb | k) != 0);
-          }
-          tc::mma_commit(&empty[s]);
-        }
-        tc::mma_commit(tfull);
-        ++it;
-      }
-    }
-  } else {
-    // epilogue warps 2..9: TMEM lane quadrant (warp % 4), column half (warp - 2) / 4;
-    // in the row phase warp ew takes rows ew, ew + 8, ew + 16, ew + 24 of the group
-    const int ew = warp - 2, quad = warp & 3, half = ew >> 2;
-    uint32_t it = 0;
-    for (int tile = blockIdx.x; tile < m_tiles; tile += gridDim.x) {
-      const int m0 = tile * tc::BM;
-      if (!tc::tile_live(g, m0)) continue;   // no row refreshes the unit: the walk adds its cache
-      for (int grp = 0; grp < 4; ++grp) {
-        // this warp's rows of the group: which refresh the unit, and their stream
-        // (loaded before the accumulator is drained; the loads do not depend on it)
-        float4 v[4][NV];
-        bool ref[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int row = m0 + grp * 32 + ew + 8 * i;
-          ref[i] = row < p.rows && lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0);
-          if (ref[i]) ld4<NV>(v[i], p.a + (long long)row * E, lane);
-        }
-        if (grp == 0) {
-          tc::mbar_wait(tfull, it & 1u, g.status, g.wait_limit);
-          tc::tc_fence_after();
-        }
-        if (quad == grp) {
-          // thread = tile row 32 grp + lane: its half of the columns into the staging tile
-#pragma unroll 1
-          for (int c = half * (E / 64); c < (half + 1) * (E / 64); ++c) {
-            float r[32];
-            tc::tmem_ld32(tmem + ((uint32_t)(grp * 32) << 16) + (uint32_t)(c * 32), r);
-            float4* d = reinterpret_cast<float4*>(stg + lane * C::STG_LD + c * 32);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) d[q] = make_float4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
-          }
-          tc::tc_fence_before();
-        }
-        asm volatile("bar.sync 1, 256;" ::: "memory");
-        if (grp == 3 && ew == 0 && lane == 0) {
-          tc::tc_fence_after();
-          tc::mbar_arrive1(tempty);          // the accumulator is drained: the next tile's MMAs may start
-        }
-        float4 bb[NV];
-        ld4<NV>(bb, p.bias, lane);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          if (!ref[i]) continue;
-          const int rr = ew + 8 * i, row = m0 + grp * 32 + rr;
-          if (!dcheck(p.b0 >= 0 && p.b0 < p.lat.U && (long long)row * E < p.cache_unit, g.status)) continue;
-          __nv_bfloat16* crow = p.cache + (long long)p.b0 * p.cache_unit + (long long)row * E + 4 * lane;
-#pragma unroll
-          for (int j = 0; j < NV; ++j) {
-            float4 r = *reinterpret_cast<const float4*>(stg + rr * C::STG_LD + 128 * j + 4 * lane);
-            r.x += bb[j].x;
-            r.y += bb[j].y;
-            r.z += bb[j].z;
-            r.w += bb[j].w;
-            *reinterpret_cast<uint2*>(crow + 128 * j) = pack_bf16x4(r);
-            if (p.trace) *reinterpret_cast<float4*>(trace_row<NV>(p, p.t0, p.b0, row) + 128 * j + 4 * lane) = r;
-            v[i][j].x += r.x;
-            v[i][j].y += r.y;
-            v[i][j].z += r.z;
-            v[i][j].w += r.w;
-          }
-          st4<NV>(p.a + (long long)row * E, lane, v[i]);
-        }
-        asm volatile("bar.sync 1, 256;" ::: "memory");   // the staging tile is free for the next group
-      }
-      ++it;
-    }
-  }
-  __syncwarp();
-  tc::pdl_trigger();                       // the next kernel may launch while this one drains
-  settle_after_timeout(g.status, false);   // after a timeout, copies and MMAs may still be in flight
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 1) tc::tmem_dealloc(tmem, E);
 }
 
 // ---------------------------------------------------------------- attention
@@ -802,6 +641,7 @@ struct WideState {
   float* head_wt = nullptr;         // [A][E]
   float* ln_gb = nullptr;           // [2][U][E]: LayerNorm gain and shift of every unit's branch
   int* first = nullptr;             // [max_sched][U]
+  uint64_t* mask = nullptr;         // [max_sched][T][2]
   CUtensorMap mA_xln, mA_att, mA_hid;
   BMaps mB_e, mB_4e;
   int num_sms = 0;
@@ -862,23 +702,6 @@ cudaError_t walk(const Walk& p, bool pdl, cudaStream_t st) {
   const dim3 grid((p.rows + 7) / 8), block(256);
   if (p.E == 256) return launch_pdl(pdl, walk_kernel<2>, grid, block, 0, st, p);
   if (p.E == 512) return launch_pdl(pdl, walk_kernel<4>, grid, block, 0, st, p);
-  return cudaErrorInvalidValue;
-}
-
-template <int E>
-cudaError_t resid_attr() {
-  return cudaFuncSetAttribute(resid_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, ResidCfg<E>::SMEM_BYTES);
-}
-
-// the residual GEMM of one refreshed unit and the walk to the next refreshed cell
-cudaError_t resid(const CUtensorMap& ma, const BMaps& mb, const tc::GemmArgs& g, const Walk& p, int rows_p,
-                  int num_sms, bool pdl, cudaStream_t st) {
-  const int m_tiles = rows_p / tc::BM;
-  const dim3 grid(std::min(m_tiles, num_sms)), block(tc::NTHREADS_GEMM);
-  if (p.E == 256)
-    return launch_pdl(pdl, resid_kernel<256>, grid, block, ResidCfg<256>::SMEM_BYTES, st, ma, mb.n256, g, p, m_tiles);
-  if (p.E == 512)
-    return launch_pdl(pdl, resid_kernel<512>, grid, block, ResidCfg<512>::SMEM_BYTES, st, ma, mb.n256, g, p, m_tiles);
   return cudaErrorInvalidValue;
 }
 
@@ -986,6 +809,7 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
   if (guarded_malloc(reinterpret_cast<void**>(&w->a), R * E * 4, &w->guards) != cudaSuccess)
     return fail(EVO_ERR_OOM);
   if (cudaMalloc(&w->first, (size_t)max_sched * w->U * sizeof(int)) != cudaSuccess) return fail(EVO_ERR_OOM);
+  if (cudaMalloc(&w->mask, (size_t)max_sched * w->T * 2 * sizeof(uint64_t)) != cudaSuccess) return fail(EVO_ERR_OOM);
   // operand rows that no call writes (padding up to a tile) read as zero
   cudaMemset(w->xln, 0, R * E * 2);
   cudaMemset(w->att, 0, R * E * 2);
@@ -999,7 +823,7 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     return fail(EVO_ERR_CUDA);
   if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
       gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
-      resid_attr<256>() != cudaSuccess || resid_attr<512>() != cudaSuccess)
+      gemm_attr<tc::EPI_RESID, 128>() != cudaSuccess || gemm_attr<tc::EPI_RESID, 256>() != cudaSuccess)
     return fail(EVO_ERR_CUDA);
   {
     int dev = 0;
@@ -1026,6 +850,7 @@ void wide_destroy(WideState* w) {
   guarded_free(w->cache);
   guarded_free(w->a);
   cudaFree(w->first);
+  cudaFree(w->mask);
   cudaFree(w->head_wt);
   cudaFree(w->ln_gb);
   delete w;
@@ -1067,13 +892,14 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   lat.S = c.S_dev;
   lat.stride = one;
   lat.first = w->first;
+  lat.mask = w->mask;
   lat.S_rows = c.S_rows;
   lat.U = U;
   lat.T = T;
   lat.H = H;
   lat.per_sched = c.per_sched;
   lat.force = w->force;
-  WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first));
+  WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first, w->mask));
 
   Walk wp{};
   wp.lat = lat;
@@ -1131,6 +957,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
   g.force = w->force;
   g.status = c.status;
   g.wait_limit = WAIT_POLLS_DEFAULT;
+  g.resid = w->a;
+  g.ldr = E;
 
   AttnArgs ap{};
   ap.lat = lat;
@@ -1156,6 +984,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
     ap.t = t;
     ap.b = b;
     ap.l = l;
+    g.cache = w->cache + (long long)b * w->rmax * E;
+    g.trace = c.trace ? c.trace + ((long long)t * U + b) * R * E : nullptr;
     wp.t0 = t;
     wp.b0 = b;
     set_next(i + 1);
@@ -1171,8 +1001,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
       WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, false> : attn_mma_kernel<1, false>, attn_grid,
                      dim3(SA_WARPS * 32), sa_smem, st, ap));
       g.b_row0 = rowE + 3 * E;
-      wp.bias = wl(w, l, WL_SA_BO);
-      WCK(resid(w->mA_att, w->mB_e, g, wp, Rp, w->num_sms, pdl, st));
+      g.bias = wl(w, l, WL_SA_BO);
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else if (u == 1) {
       g.K = E;
@@ -1185,8 +1015,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
       WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, true> : attn_mma_kernel<1, true>, attn_grid,
                      dim3(SA_WARPS * 32), ca_smem, st, ap));
       g.b_row0 = rowE + 5 * E;
-      wp.bias = wl(w, l, WL_CA_BO);
-      WCK(resid(w->mA_att, w->mB_e, g, wp, Rp, w->num_sms, pdl, st));
+      g.bias = wl(w, l, WL_CA_BO);
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else {
       g.K = E;
@@ -1197,8 +1027,8 @@ cudaError_t wide_run(WideState* w, const WideCall& c) {
       WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, pdl, st));
       g.K = 4 * E;
       g.b_row0 = l * E;
-      wp.bias = wl(w, l, WL_FF_B2);
-      WCK(resid(w->mA_hid, w->mB_4e, g, wp, Rp, w->num_sms, pdl, st));
+      g.bias = wl(w, l, WL_FF_B2);
+      WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     }
   }
