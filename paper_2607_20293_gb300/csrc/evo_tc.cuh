@@ -18,8 +18,8 @@
 //     row segments (a warp-per-row store: the thread-per-row layout of the
 //     accumulator would scatter every store over 32 rows), then releases the
 //     accumulator.  The residual mode (the output projection of a refreshed
-//     unit) stages fp32 and, row by row, adds r to the residual stream and
-//     writes the unit's bf16 cache (Eq. 1) for the rows that refresh the unit.
+//     unit) stages fp32 and, row by row, stores r and the unit's bf16 cache
+//     (Eq. 1) for the rows that refresh the unit.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
 // next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
@@ -68,7 +68,7 @@ struct GemmArgs {
   const float* bias;          // [N] fp32
   __nv_bfloat16* out;         // EPI_BF16 / EPI_GELU_BF16: out[row * ldo + n]
   int ldo;
-  float* resid;               // EPI_RESID: residual stream [rows][ldr] fp32, += r for refreshing rows
+  float* rout;                // EPI_RESID: the branch output r [rows][ldr] fp32, for refreshing rows
   __nv_bfloat16* cache;       // EPI_RESID: the unit's cache [rows][ldr], <- bf16(r) for refreshing rows
   float* trace;               // EPI_RESID: [rows][ldr] or null: r of refreshing rows (debug trace)
   int ldr;
@@ -254,9 +254,9 @@ __device__ __forceinline__ void epilogue_flush(const GemmArgs& g, const uint8_t*
 
 // EPI_RESID, one chunk of 32 columns n .. n + 31: r = acc + bias goes to the
 // warp's staging rows (fp32, thread = row), then the warp takes the rows one
-// at a time (lane = column, 128 contiguous bytes): a += r, c_b <- bf16(r) for
-// the rows whose lattice refreshes the unit (bit r of rmask); the stream of 16
-// rows at a time is loaded before any is written.
+// at a time (lane = column, 128 contiguous bytes) and, for the rows whose
+// lattice refreshes the unit (bit r of rmask), stores r and c_b <- bf16(r)
+// (Eq. 1).  The row walk that follows adds r to the residual stream.
 __device__ __forceinline__ void epilogue_resid(const GemmArgs& g, int row0, int n, float (&v)[32], uint8_t* stg,
                                                int lane, unsigned rmask) {
   const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
@@ -269,23 +269,14 @@ __device__ __forceinline__ void epilogue_resid(const GemmArgs& g, int row0, int 
   }
   __syncwarp();
   const long long col = n + lane;
-#pragma unroll
-  for (int h = 0; h < 32; h += 16) {
-    float av[16];
-#pragma unroll
-    for (int r = 0; r < 16; ++r)
-      av[r] = (rmask >> (h + r)) & 1u ? g.resid[(long long)(row0 + h + r) * g.ldr + col] : 0.f;
-#pragma unroll
-    for (int r = 0; r < 16; ++r) {
-      if (!((rmask >> (h + r)) & 1u)) continue;
-      const int rr = h + r;
-      const float rv =
-          *reinterpret_cast<const float*>(stg + rr * 128 + (((lane >> 2) ^ (rr & 7)) << 4) + (lane & 3) * 4);
-      const long long o = (long long)(row0 + rr) * g.ldr + col;
-      g.resid[o] = av[r] + rv;
-      g.cache[o] = __float2bfloat16_rn(rv);
-      if (g.trace) g.trace[o] = rv;
-    }
+#pragma unroll 8
+  for (int r = 0; r < 32; ++r) {
+    if (!((rmask >> r) & 1u)) continue;
+    const float rv = *reinterpret_cast<const float*>(stg + r * 128 + (((lane >> 2) ^ (r & 7)) << 4) + (lane & 3) * 4);
+    const long long o = (long long)(row0 + r) * g.ldr + col;
+    g.rout[o] = rv;
+    g.cache[o] = __float2bfloat16_rn(rv);
+    if (g.trace) g.trace[o] = rv;
   }
   __syncwarp();
 }

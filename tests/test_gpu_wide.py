@@ -143,3 +143,27 @@ def test_wide_trace_eq1_bitwise(torch, B, force):
     assert ev.last_call()["path"] == "wide"
     assert check_reuse(trace.cpu().numpy(), S, bf16=True, force=force) > 100
     check(got, O.denoise(W, cfg, obs, noise, S, "force" if force else "zero"), "wide trace")
+
+
+def test_repeated_calls_replay_the_captured_sequence(torch, B):
+    """A call that repeats the previous one (same lattice, sizes and buffers) is
+    captured into a CUDA graph and replayed: the first, second (captured) and
+    third (replayed) calls give bit-identical actions; a new lattice, or new
+    inputs in the same buffers, give that call's own result."""
+    cfg, W, obs, noise, ev, d_obs, d_noise = make("pusht", 9, torch, B)
+    out = torch.empty((9, 16, 2), device="cuda")
+    S = synth.bernoulli_schedule(24, 100, 0.2, 31)
+    runs = [ev.denoise(d_obs, d_noise, S, out=out).cpu().numpy() for _ in range(3)]
+    assert ev.last_call()["path"] == "wide"
+    assert np.array_equal(runs[0], runs[1]) and np.array_equal(runs[0], runs[2])
+    check(runs[0], O.denoise(W, cfg, obs, noise, S), "replayed")
+    S2 = synth.bernoulli_schedule(24, 100, 0.2, 32)
+    got2 = ev.denoise(d_obs, d_noise, S2, out=out).cpu().numpy()
+    check(got2, O.denoise(W, cfg, obs, noise, S2), "new lattice")
+    assert not np.array_equal(got2, runs[0])
+    obs3 = synth.make_obs(cfg, 9, 77)
+    d_obs.copy_(torch.from_numpy(obs3))                 # same buffer, new contents
+    for _ in range(3):
+        got3 = ev.denoise(d_obs, d_noise, S2, out=out).cpu().numpy()
+    check(got3, O.denoise(W, cfg, obs3, noise, S2), "new inputs in the same buffers")
+    assert ev.status() == B.OK
