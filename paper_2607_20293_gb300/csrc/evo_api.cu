@@ -927,9 +927,10 @@ evo_status stage_wide(evo_handle* h, const uint8_t* S, int n_sched, int rows, bo
   return stage_schedules(h, S, n_sched, rows, add_ones, st, &err);   // host lattice: validated, cached
 }
 
-cudaError_t launch_wide(evo_handle* h, const float* noise, float* out, int samples, int per_sched, int n_sched,
-                        int S_rows, cudaStream_t st, float* trace = nullptr) {
+cudaError_t launch_wide(evo_handle* h, const float* obs, const float* noise, float* out, int samples, int per_sched,
+                        int n_sched, int S_rows, cudaStream_t st, float* trace = nullptr) {
   WideCall c{};
+  c.obs = obs;
   c.noise = noise;
   c.out = out;
   c.kv_obs = h->kv_obs;
@@ -970,8 +971,8 @@ evo_status run(evo_handle* h, const float* obs, const float* noise, const uint8_
   if (use_wide(h, N)) {
     const evo_status s = stage_wide(h, S, 1, S_rows, false, st);
     if (s != EVO_OK) return s;
-    EVO_CUDA(obs_cond(h, obs, N, h->cond_scratch, h->kv_obs, st));
-    EVO_CUDA(launch_wide(h, noise, out, N, N, 1, S_rows, st, trace));
+    h->last_cond_kernels = 0;                  // the batch-wide sequence computes kv_obs itself
+    EVO_CUDA(launch_wide(h, obs, noise, out, N, N, 1, S_rows, st, trace));
     return finish(h, st);
   }
   const int* err = nullptr;
@@ -1094,8 +1095,8 @@ evo_status evo_denoise_population(evo_handle* h, const float* obs, const float* 
   if (use_wide(h, samples)) {
     const evo_status s = stage_wide(h, S_pop, P, S_rows, true, st);
     if (s != EVO_OK) return s;
-    EVO_CUDA(obs_cond(h, obs, N_obs, h->cond_scratch, h->kv_obs, st));
-    EVO_CUDA(launch_wide(h, noise, h->pop_x, (int)samples, N_obs, P + 1, S_rows, st));
+    h->last_cond_kernels = 0;                  // the batch-wide sequence computes kv_obs itself
+    EVO_CUDA(launch_wide(h, obs, noise, h->pop_x, (int)samples, N_obs, P + 1, S_rows, st));
     EVO_CUDA(launch_pop_dev(h->pop_x, P, N_obs, HA, dev_l2, st));
     h->last_kernels += 1;
     if (out_actions)

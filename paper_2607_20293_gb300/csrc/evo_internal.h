@@ -171,9 +171,10 @@ cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev,
 // batch-wide path (evo_wide.cu)
 struct WideState;
 struct WideCall {
+  const float* obs;               // [obs_mod][n_obs][obs_dim]: the path computes kv_obs from these
   const float* noise;             // [n_noise][obs_mod][H][A]
   float* out;                     // [samples][H][A]: running x, final actions
-  const float* kv_obs;            // [obs_mod][n_obs][L][2E]
+  float* kv_obs;                  // [obs_mod][n_obs][L][2E] (output of the condition GEMMs)
   const float* kv_time;           // [T][L][2E]
   const float* stab;              // [T][8]
   int samples, per_sched, obs_mod;

@@ -60,7 +60,7 @@ struct TileCfg {
       (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 };
 
-enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2 };
+enum EpiMode { EPI_BF16 = 0, EPI_GELU_BF16 = 1, EPI_RESID = 2, EPI_MISH_BF16 = 3, EPI_F32 = 4 };
 
 struct GemmArgs {
   int K;                      // multiple of BK
@@ -72,6 +72,9 @@ struct GemmArgs {
   __nv_bfloat16* cache;       // EPI_RESID: the unit's cache [rows][ldr], <- bf16(r) for refreshing rows
   float* trace;               // EPI_RESID: [rows][ldr] or null: r of refreshing rows (debug trace)
   int ldr;
+  float* out32;               // EPI_F32: out32[row * ldo + n]
+  const float* rbias;         // bf16 modes, or null: + rbias[(row % rbias_mod) * ldo + n] (a per-row bias)
+  int rbias_mod;
   int rows;                   // real rows; rows >= this are padding
   // refresh gate (null: every row refreshes): row -> sample row / H -> lattice
   // (sample / per_sched); refresh = S[lattice * S_stride + srow * T + t]
@@ -196,6 +199,11 @@ __device__ __forceinline__ bool row_refreshes(const GemmArgs& g, int row) {
   return g.S[(long long)(sample / g.per_sched) * g.S_stride + (long long)g.srow * g.T + g.t] != 0;
 }
 
+__device__ __forceinline__ float mish_f(float v) {
+  const float sp = v > 20.f ? v : log1pf(expf(v));
+  return v * tanhf(sp);
+}
+
 __device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
 
 // does any row of the tile starting at m0 refresh?  (the same answer in every role)
@@ -212,8 +220,8 @@ __device__ __forceinline__ bool tile_live(const GemmArgs& g, int m0) {
 // packed to bf16 and written as 64 bytes of the thread's staging row (chunks
 // j4 .. j4 + 3 of 16 bytes, swizzled by the row within the 8-row group)
 template <int MODE>
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int n, float (&v)[32], uint8_t* srow, int lane,
-                                               int j4) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n, float (&v)[32], uint8_t* srow,
+                                               int lane, int j4) {
   const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
@@ -223,9 +231,24 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int n, float (
     v[4 * q + 2] += bb.z;
     v[4 * q + 3] += bb.w;
   }
+  if (g.rbias) {
+    const float4* r4 = reinterpret_cast<const float4*>(g.rbias + (long long)(row % g.rbias_mod) * g.ldo + n);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 bb = __ldg(r4 + q);
+      v[4 * q] += bb.x;
+      v[4 * q + 1] += bb.y;
+      v[4 * q + 2] += bb.z;
+      v[4 * q + 3] += bb.w;
+    }
+  }
   if constexpr (MODE == EPI_GELU_BF16) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
+  }
+  if constexpr (MODE == EPI_MISH_BF16) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = mish_f(v[i]);
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -277,6 +300,28 @@ __device__ __forceinline__ void epilogue_resid(const GemmArgs& g, int row0, int 
     g.rout[o] = rv;
     g.cache[o] = __float2bfloat16_rn(rv);
     if (g.trace) g.trace[o] = rv;
+  }
+  __syncwarp();
+}
+
+// EPI_F32, one chunk of 32 columns: acc + bias staged as fp32 (thread = row),
+// then stored row by row (lane = column, 128 contiguous bytes) for rows < rows
+__device__ __forceinline__ void epilogue_f32(const GemmArgs& g, int row0, int n, float (&v)[32], uint8_t* stg,
+                                             int lane) {
+  const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
+  uint8_t* srow = stg + lane * 128;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 bb = __ldg(b4 + q);
+    *reinterpret_cast<float4*>(srow + ((q ^ (lane & 7)) << 4)) =
+        make_float4(v[4 * q] + bb.x, v[4 * q + 1] + bb.y, v[4 * q + 2] + bb.z, v[4 * q + 3] + bb.w);
+  }
+  __syncwarp();
+#pragma unroll 8
+  for (int r = 0; r < 32; ++r) {
+    if (row0 + r >= g.rows) break;
+    g.out32[(long long)(row0 + r) * g.ldo + n + lane] =
+        *reinterpret_cast<const float*>(stg + r * 128 + (((lane >> 2) ^ (r & 7)) << 4) + (lane & 3) * 4);
   }
   __syncwarp();
 }
@@ -369,6 +414,19 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       const uint32_t acc = it & 1u;
       mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status, g.wait_limit);
       tc_fence_after();
+      if constexpr (MODE == EPI_F32) {
+#pragma unroll 1
+        for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
+          float v[32];
+          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
+          epilogue_f32(g, m0 + quad * 32, n0 + c * 32, v, stg, lane);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive1(&tempty[acc]);
+        ++it;
+        continue;
+      }
       if constexpr (MODE == EPI_RESID) {
         const unsigned rmask = __ballot_sync(0xffffffffu, row_refreshes(g, m0 + quad * 32 + lane));
 #pragma unroll 1
@@ -389,7 +447,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
         for (int j = 0; j < 2; ++j) {
           float v[32];
           tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)((c + j) * 32), v);
-          epilogue_chunk<MODE>(g, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
+          epilogue_chunk<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
         }
         __syncwarp();
         epilogue_flush(g, stg, m0 + quad * 32, n0 + c * 32, lane);

@@ -134,6 +134,19 @@ __global__ void first_kernel(Lat L, int n_sched, int* first, uint64_t* mask) {
   (void)n_sched;
 }
 
+// observation features fp32 [ntok][D] -> bf16 [ntok][Dp] (zero padding), the
+// A operand of the condition path's first GEMM
+__global__ void obs_to_bf16_kernel(const float* obs, int ntok, int D, int Dp, __nv_bfloat16* out) {
+  tc::pdl_trigger();
+  tc::pdl_wait();
+  const long long n = (long long)ntok * Dp;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+    const long long tok = i / Dp;
+    const int d = (int)(i - tok * Dp);
+    out[i] = __float2bfloat16_rn(d < D ? obs[tok * D + d] : 0.f);
+  }
+}
+
 // ---------------------------------------------------------------- the row walk (one warp per row)
 // Between two refreshed lattice cells nothing but per-row work happens: the
 // skipped units' cached outputs are added (Eq. 1), and at the end of a step
@@ -654,16 +667,28 @@ struct WideState {
   float* rbuf = nullptr;            // [rmax][E]: output of the unit just computed
   float* head_wt = nullptr;         // [A][E]
   float* ln_gb = nullptr;           // [2][U][E]: LayerNorm gain and shift of every unit's branch
+  // observation conditioning on the tensor cores: embedding, MLP (Mish), keys|values
+  int D = 0, Dp = 0;                // observation dim, padded to a multiple of BK
+  long long tokcap = 0;             // rows of the condition buffers (multiple of BM)
+  __nv_bfloat16* obs16 = nullptr;   // [tokcap][Dp]
+  __nv_bfloat16* cx16 = nullptr;    // [tokcap][E]
+  __nv_bfloat16* ch16 = nullptr;    // [tokcap][4E]
+  __nv_bfloat16* cm16 = nullptr;    // [tokcap][E]
+  __nv_bfloat16* cw_t = nullptr;    // W_obs^T [E][Dp] | W1^T [4E][E] | W2^T [E][4E] | Wkv^T [L*2E][E]
+  float* bkv = nullptr;             // [L*2E]
   int* first = nullptr;             // [max_sched][U]
   uint64_t* mask = nullptr;         // [max_sched][T][2]
   CUtensorMap mA_xln, mA_att, mA_hid;
   BMaps mB_e, mB_4e;
+  CUtensorMap mA_obs, mA_cx, mA_ch, mA_cm;
+  BMaps mB_obs, mB_cw1, mB_cw2, mB_kv;
   int num_sms = 0;
   GuardList guards;                 // guard bands of the activation buffers
   // replay of a repeated call's launch sequence (wide_run)
   struct GraphKey {
     bool valid = false;
-    const void *noise = nullptr, *out = nullptr, *kv_obs = nullptr, *kv_time = nullptr, *stab = nullptr;
+    const void *obs = nullptr, *noise = nullptr, *out = nullptr, *kv_obs = nullptr, *kv_time = nullptr;
+    const void *stab = nullptr;
     const void *trace = nullptr, *status = nullptr, *S_dev = nullptr;
     int samples = 0, per_sched = 0, obs_mod = 0, n_sched = 0, S_rows = 0;
     std::vector<uint8_t> S;
@@ -823,6 +848,61 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     if (cudaMemcpy(w->ln_gb, gb.data(), gb.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(EVO_ERR_CUDA);
   }
+  {
+    // condition path: transposed bf16 weights [N][K] and the stacked key|value bias
+    w->D = c->obs_dim;
+    w->Dp = (c->obs_dim + tc::BK - 1) / tc::BK * tc::BK;
+    const int Dp = w->Dp, KV = L * 2 * E;
+    std::vector<uint16_t> cw((size_t)E * Dp + (size_t)4 * E * E * 2 + (size_t)KV * E, 0);
+    uint16_t* wo_t = cw.data();
+    uint16_t* w1_t = wo_t + (size_t)E * Dp;
+    uint16_t* w2_t = w1_t + (size_t)4 * E * E;
+    uint16_t* kv_t = w2_t + (size_t)4 * E * E;
+    const float* wobs = weights + woff[W_OBS_W];
+    const float* w1 = weights + woff[W_CM_W1];
+    const float* w2 = weights + woff[W_CM_W2];
+    for (int d = 0; d < w->D; ++d)
+      for (int e = 0; e < E; ++e) wo_t[(size_t)e * Dp + d] = bf16_bits(wobs[(size_t)d * E + e]);
+    for (int k = 0; k < E; ++k)
+      for (int n = 0; n < 4 * E; ++n) w1_t[(size_t)n * E + k] = bf16_bits(w1[(size_t)k * 4 * E + n]);
+    for (int k = 0; k < 4 * E; ++k)
+      for (int n = 0; n < E; ++n) w2_t[(size_t)n * 4 * E + k] = bf16_bits(w2[(size_t)k * E + n]);
+    std::vector<float> bkv((size_t)KV);
+    for (int l = 0; l < L; ++l) {
+      const float* base = weights + woff[W_LAYER0] + (size_t)l * woff[W_LAYER_STRIDE];
+      const float* wkv = base + woff[WL_CA_WKV];
+      for (int k = 0; k < E; ++k)
+        for (int j = 0; j < 2 * E; ++j) kv_t[((size_t)l * 2 * E + j) * E + k] = bf16_bits(wkv[(size_t)k * 2 * E + j]);
+      std::memcpy(&bkv[(size_t)l * 2 * E], base + woff[WL_CA_BKV], (size_t)2 * E * 4);
+    }
+    if (cudaMalloc(&w->cw_t, cw.size() * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMalloc(&w->bkv, bkv.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMemcpy(w->cw_t, cw.data(), cw.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(w->bkv, bkv.data(), bkv.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(EVO_ERR_CUDA);
+    const long long toks = (max_rows / w->H) * (long long)c->n_obs;
+    w->tokcap = (toks + tc::BM - 1) / tc::BM * tc::BM;
+    const long long TC = w->tokcap;
+    if (cudaMalloc(&w->obs16, TC * Dp * 2) != cudaSuccess || cudaMalloc(&w->cx16, TC * E * 2) != cudaSuccess ||
+        cudaMalloc(&w->ch16, TC * 4 * E * 2) != cudaSuccess || cudaMalloc(&w->cm16, TC * E * 2) != cudaSuccess)
+      return fail(EVO_ERR_OOM);
+    cudaMemset(w->obs16, 0, TC * Dp * 2);
+    cudaMemset(w->cx16, 0, TC * E * 2);
+    cudaMemset(w->ch16, 0, TC * 4 * E * 2);
+    cudaMemset(w->cm16, 0, TC * E * 2);
+    const __nv_bfloat16* cwd = w->cw_t;
+    const __nv_bfloat16* d_wo = cwd;
+    const __nv_bfloat16* d_w1 = d_wo + (size_t)E * Dp;
+    const __nv_bfloat16* d_w2 = d_w1 + (size_t)4 * E * E;
+    const __nv_bfloat16* d_kv = d_w2 + (size_t)4 * E * E;
+    if (!make_map(&w->mA_obs, w->obs16, TC, Dp, tc::BM) || !make_map(&w->mA_cx, w->cx16, TC, E, tc::BM) ||
+        !make_map(&w->mA_ch, w->ch16, TC, 4 * E, tc::BM) || !make_map(&w->mA_cm, w->cm16, TC, E, tc::BM) ||
+        !make_map(&w->mB_obs.n128, d_wo, E, Dp, 128) || !make_map(&w->mB_obs.n256, d_wo, E, Dp, 256) ||
+        !make_map(&w->mB_cw1.n128, d_w1, 4 * E, E, 128) || !make_map(&w->mB_cw1.n256, d_w1, 4 * E, E, 256) ||
+        !make_map(&w->mB_cw2.n128, d_w2, E, 4 * E, 128) || !make_map(&w->mB_cw2.n256, d_w2, E, 4 * E, 256) ||
+        !make_map(&w->mB_kv.n128, d_kv, KV, E, 128) || !make_map(&w->mB_kv.n256, d_kv, KV, E, 256))
+      return fail(EVO_ERR_CUDA);
+  }
   if (guarded_malloc(reinterpret_cast<void**>(&w->xln), R * E * 2, &w->guards) != cudaSuccess)
     return fail(EVO_ERR_OOM);
   if (guarded_malloc(reinterpret_cast<void**>(&w->qkv), R * 3 * E * 2, &w->guards) != cudaSuccess)
@@ -852,7 +932,9 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
     return fail(EVO_ERR_CUDA);
   if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
       gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
-      gemm_attr<tc::EPI_RESID, 128>() != cudaSuccess || gemm_attr<tc::EPI_RESID, 256>() != cudaSuccess)
+      gemm_attr<tc::EPI_RESID, 128>() != cudaSuccess || gemm_attr<tc::EPI_RESID, 256>() != cudaSuccess ||
+      gemm_attr<tc::EPI_MISH_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_MISH_BF16, 256>() != cudaSuccess ||
+      gemm_attr<tc::EPI_F32, 128>() != cudaSuccess || gemm_attr<tc::EPI_F32, 256>() != cudaSuccess)
     return fail(EVO_ERR_CUDA);
   {
     int dev = 0;
@@ -883,6 +965,12 @@ void wide_destroy(WideState* w) {
   cudaFree(w->mask);
   cudaFree(w->head_wt);
   cudaFree(w->ln_gb);
+  cudaFree(w->obs16);
+  cudaFree(w->cx16);
+  cudaFree(w->ch16);
+  cudaFree(w->cm16);
+  cudaFree(w->cw_t);
+  cudaFree(w->bkv);
   if (w->exec) cudaGraphExecDestroy(w->exec);
   if (w->cap_stream) cudaStreamDestroy(w->cap_stream);
   delete w;
@@ -932,6 +1020,43 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
   lat.H = H;
   lat.per_sched = c.per_sched;
   lat.force = w->force;
+  if (c.obs) {
+    // observation tokens -> their cross-attention keys/values of every layer:
+    // bf16 features, embedding (+ b_obs + position row), MLP E -> 4E (Mish) -> E,
+    // then one GEMM for the keys|values of all layers (fp32 out)
+    const int ntok = c.obs_mod * w->n_obs;
+    const int tp = (ntok + tc::BM - 1) / tc::BM * tc::BM;
+    const long long nel = (long long)ntok * w->Dp;
+    WCK(launch_pdl(pdl, obs_to_bf16_kernel, dim3((unsigned)std::min<long long>((nel + 255) / 256, 4096)), dim3(256), 0,
+                   st, c.obs, ntok, w->D, w->Dp, w->obs16));
+    tc::GemmArgs q{};
+    q.rows = ntok;
+    q.status = c.status;
+    q.wait_limit = WAIT_POLLS_DEFAULT;
+    q.K = w->Dp;
+    q.bias = w->wf32 + w->woff[W_OBS_B];
+    q.rbias = w->wf32 + w->woff[W_COND_POS] + E;      // position rows 1 .. n_obs
+    q.rbias_mod = w->n_obs;
+    q.out = w->cx16;
+    q.ldo = E;
+    WCK(gemm<tc::EPI_BF16>(w->mA_obs, w->mB_obs, q, tp, E, w->num_sms, pdl, st));
+    q.rbias = nullptr;
+    q.K = E;
+    q.bias = w->wf32 + w->woff[W_CM_B1];
+    q.out = w->ch16;
+    q.ldo = 4 * E;
+    WCK(gemm<tc::EPI_MISH_BF16>(w->mA_cx, w->mB_cw1, q, tp, 4 * E, w->num_sms, pdl, st));
+    q.K = 4 * E;
+    q.bias = w->wf32 + w->woff[W_CM_B2];
+    q.out = w->cm16;
+    q.ldo = E;
+    WCK(gemm<tc::EPI_BF16>(w->mA_ch, w->mB_cw2, q, tp, E, w->num_sms, pdl, st));
+    q.K = E;
+    q.bias = w->bkv;
+    q.out32 = c.kv_obs;
+    q.ldo = L * 2 * E;
+    WCK(gemm<tc::EPI_F32>(w->mA_cm, w->mB_kv, q, tp, L * 2 * E, w->num_sms, pdl, st));
+  }
   WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first, w->mask));
 
   Walk wp{};
@@ -1072,7 +1197,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
 }
 
 bool same_key(const WideState::GraphKey& k, const WideCall& c, size_t lat_bytes) {
-  return k.valid && k.noise == c.noise && k.out == c.out && k.kv_obs == c.kv_obs && k.kv_time == c.kv_time &&
+  return k.valid && k.obs == c.obs && k.noise == c.noise && k.out == c.out && k.kv_obs == c.kv_obs && k.kv_time == c.kv_time &&
          k.stab == c.stab && k.trace == c.trace && k.status == c.status && k.samples == c.samples &&
          k.per_sched == c.per_sched && k.obs_mod == c.obs_mod && k.n_sched == c.n_sched && k.S_rows == c.S_rows &&
          k.S_dev == c.S_dev && k.S.size() == lat_bytes && std::memcmp(k.S.data(), c.S_host, lat_bytes) == 0;
@@ -1080,6 +1205,7 @@ bool same_key(const WideState::GraphKey& k, const WideCall& c, size_t lat_bytes)
 
 void set_key(WideState::GraphKey& k, const WideCall& c, size_t lat_bytes) {
   k.valid = true;
+  k.obs = c.obs;
   k.noise = c.noise;
   k.out = c.out;
   k.kv_obs = c.kv_obs;
