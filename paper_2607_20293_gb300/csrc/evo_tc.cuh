@@ -414,44 +414,35 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       const uint32_t acc = it & 1u;
       mbar_wait(&tfull[acc], (it >> 1) & 1u, g.status, g.wait_limit);
       tc_fence_after();
+      const uint32_t tq = tmem + acc * BN + ((uint32_t)(quad * 32) << 16);   // this warp's TMEM lanes
       if constexpr (MODE == EPI_F32) {
 #pragma unroll 1
         for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
           float v[32];
-          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
+          tmem_ld32(tq + (uint32_t)(c * 32), v);
           epilogue_f32(g, m0 + quad * 32, n0 + c * 32, v, stg, lane);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive1(&tempty[acc]);
-        ++it;
-        continue;
-      }
-      if constexpr (MODE == EPI_RESID) {
+      } else if constexpr (MODE == EPI_RESID) {
         const unsigned rmask = __ballot_sync(0xffffffffu, row_refreshes(g, m0 + quad * 32 + lane));
 #pragma unroll 1
         for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
           float v[32];
-          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)(c * 32), v);
+          tmem_ld32(tq + (uint32_t)(c * 32), v);
           epilogue_resid(g, m0 + quad * 32, n0 + c * 32, v, stg, lane, rmask);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive1(&tempty[acc]);
-        ++it;
-        continue;
-      }
+      } else {
 #pragma unroll 1
-      for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); c += 2) {
+        for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); c += 2) {
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-          float v[32];
-          tmem_ld32(tmem + acc * BN + ((uint32_t)(quad * 32) << 16) + (uint32_t)((c + j) * 32), v);
-          epilogue_chunk<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
+          for (int j = 0; j < 2; ++j) {
+            float v[32];
+            tmem_ld32(tq + (uint32_t)((c + j) * 32), v);
+            epilogue_chunk<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
+          }
+          __syncwarp();
+          epilogue_flush(g, stg, m0 + quad * 32, n0 + c * 32, lane);
+          __syncwarp();
         }
-        __syncwarp();
-        epilogue_flush(g, stg, m0 + quad * 32, n0 + c * 32, lane);
-        __syncwarp();
       }
       tc_fence_before();
       __syncwarp();

@@ -92,10 +92,6 @@ __device__ __forceinline__ bool lat_refresh(const Lat& L, int sample, int b, int
   return L.S[(long long)(sample / L.per_sched) * L.stride + (long long)r * L.T + t] != 0;
 }
 
-// the unit's cache holds a value at step t (it was refreshed at an earlier step)
-__device__ __forceinline__ bool lat_valid(const Lat& L, int sample, int b, int t) {
-  return L.first[(sample / L.per_sched) * L.U + b] < t;
-}
 
 // per lattice: the first step that refreshes each unit, and per step the
 // bitmasks of the units it refreshes and of the units whose cache holds a value
