@@ -13,11 +13,11 @@
 //     accumulator to the epilogue;
 //   * warps 2-9: epilogue.  Warp w reads TMEM lanes (= tile rows) of its
 //     quadrant 32 (w % 4) .. +31 and one half of the tile's columns, 32 at a
-//     time (tcgen05.ld), applies bias (and GELU), packs bf16 into its staging
-//     rows in shared memory, and stores 64 columns at a time as whole 128-byte
-//     row segments (a warp-per-row store: the thread-per-row layout of the
-//     accumulator would scatter every store over 32 rows), then releases the
-//     accumulator.  The residual mode (the output projection of a refreshed
+//     time (tcgen05.ld), applies bias (and GELU / Mish), packs bf16 into its
+//     staging rows in shared memory in the 128-byte-swizzled layout, and
+//     writes each 32 x 64 block with one tiled bulk store (the thread-per-row
+//     layout of the accumulator would scatter every direct store over 32
+//     rows), then releases the accumulator.  The residual mode (the output projection of a refreshed
 //     unit) stages fp32 and, row by row, stores r and the unit's bf16 cache
 //     (Eq. 1) for the rows that refresh the unit.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
@@ -129,6 +129,21 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(su32(bar))
       : "memory");
 }
+
+// tiled bulk store shared -> global (bulk-group completion)
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int y, const void* src) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(su32(src))
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// the source shared memory of every committed bulk store has been read
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// every committed bulk store has completed
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// this thread's generic-proxy shared-memory writes become visible to the async proxy (bulk copies)
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(slot)), "r"(ncols)
@@ -332,6 +347,7 @@ __device__ __forceinline__ void epilogue_f32(const GemmArgs& g, int row0, int n,
 template <int MODE, int BN>
 __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmA,
                                                                 const __grid_constant__ CUtensorMap tmB,
+                                                                const __grid_constant__ CUtensorMap tmC,
                                                                 const GemmArgs g, int m_tiles, int n_tiles) {
   using C = TileCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
@@ -431,17 +447,25 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
           epilogue_resid(g, m0 + quad * 32, n0 + c * 32, v, stg, lane, rmask);
         }
       } else {
+        // 32 rows x 64 columns at a time: packed into the staging rows (the
+        // layout of a 128-byte-swizzled tile), then one tiled bulk store of the
+        // whole block by lane 0 (out of range rows land in the buffer's padding)
 #pragma unroll 1
         for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); c += 2) {
+          if (lane == 0) bulk_wait_read();               // the previous block has left the staging rows
+          __syncwarp();
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
             float v[32];
             tmem_ld32(tq + (uint32_t)((c + j) * 32), v);
             epilogue_chunk<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
           }
+          fence_async_smem();
           __syncwarp();
-          epilogue_flush(g, stg, m0 + quad * 32, n0 + c * 32, lane);
-          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmC, n0 + c * 32, m0 + quad * 32, stg);
+            bulk_commit();
+          }
         }
       }
       tc_fence_before();
@@ -450,6 +474,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
       ++it;
     }
   }
+  if (warp >= 2 && lane == 0) bulk_wait_all();    // this warp's tiled stores are complete
   __syncwarp();
   pdl_trigger();                           // the next kernel may launch while this one drains
   settle_after_timeout(g.status, false);   // after a timeout, copies and MMAs may still be in flight

@@ -677,6 +677,8 @@ struct WideState {
   CUtensorMap mA_xln, mA_att, mA_hid;
   BMaps mB_e, mB_4e;
   CUtensorMap mA_obs, mA_cx, mA_ch, mA_cm;
+  // tiled-store maps of the bf16 GEMM outputs (32-row x 64-column boxes)
+  CUtensorMap mC_qkv, mC_q, mC_hid, mC_cx, mC_ch, mC_cm;
   BMaps mB_obs, mB_cw1, mB_cw2, mB_kv;
   int num_sms = 0;
   GuardList guards;                 // guard bands of the activation buffers
@@ -725,18 +727,19 @@ cudaError_t launch_pdl(bool pdl, void (*k)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, k, args...);
 }
 
+// mc: the output's tiled-store map (bf16 modes; the other modes ignore it)
 template <int MODE>
-cudaError_t gemm(const CUtensorMap& ma, const BMaps& mb, const tc::GemmArgs& g, int rows_p, int N, int num_sms,
-                 bool pdl, cudaStream_t st) {
+cudaError_t gemm(const CUtensorMap& ma, const BMaps& mb, const CUtensorMap& mc, const tc::GemmArgs& g, int rows_p,
+                 int N, int num_sms, bool pdl, cudaStream_t st) {
   const int m_tiles = rows_p / tc::BM;
   if (N % 256 == 0 && m_tiles * (N / 256) >= num_sms) {
     const int total = m_tiles * (N / 256);
     return launch_pdl(pdl, tc::gemm_kernel<MODE, 256>, dim3(std::min(total, num_sms)), dim3(tc::NTHREADS_GEMM),
-                      tc::TileCfg<256>::SMEM_BYTES, st, ma, mb.n256, g, m_tiles, N / 256);
+                      tc::TileCfg<256>::SMEM_BYTES, st, ma, mb.n256, mc, g, m_tiles, N / 256);
   } else {
     const int total = m_tiles * (N / 128);
     return launch_pdl(pdl, tc::gemm_kernel<MODE, 128>, dim3(std::min(total, num_sms)), dim3(tc::NTHREADS_GEMM),
-                      tc::TileCfg<128>::SMEM_BYTES, st, ma, mb.n128, g, m_tiles, N / 128);
+                      tc::TileCfg<128>::SMEM_BYTES, st, ma, mb.n128, mc, g, m_tiles, N / 128);
   }
 }
 
@@ -896,7 +899,9 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
         !make_map(&w->mB_obs.n128, d_wo, E, Dp, 128) || !make_map(&w->mB_obs.n256, d_wo, E, Dp, 256) ||
         !make_map(&w->mB_cw1.n128, d_w1, 4 * E, E, 128) || !make_map(&w->mB_cw1.n256, d_w1, 4 * E, E, 256) ||
         !make_map(&w->mB_cw2.n128, d_w2, E, 4 * E, 128) || !make_map(&w->mB_cw2.n256, d_w2, E, 4 * E, 256) ||
-        !make_map(&w->mB_kv.n128, d_kv, KV, E, 128) || !make_map(&w->mB_kv.n256, d_kv, KV, E, 256))
+        !make_map(&w->mB_kv.n128, d_kv, KV, E, 128) || !make_map(&w->mB_kv.n256, d_kv, KV, E, 256) ||
+        !make_map(&w->mC_cx, w->cx16, TC, E, 32) || !make_map(&w->mC_ch, w->ch16, TC, 4 * E, 32) ||
+        !make_map(&w->mC_cm, w->cm16, TC, E, 32))
       return fail(EVO_ERR_CUDA);
   }
   if (guarded_malloc(reinterpret_cast<void**>(&w->xln), R * E * 2, &w->guards) != cudaSuccess)
@@ -924,7 +929,9 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
       !make_map(&w->mB_e.n128, w->wt_e, (long long)L * 10 * E, E, 128) ||
       !make_map(&w->mB_e.n256, w->wt_e, (long long)L * 10 * E, E, 256) ||
       !make_map(&w->mB_4e.n128, w->wt_4e, (long long)L * E, 4 * E, 128) ||
-      !make_map(&w->mB_4e.n256, w->wt_4e, (long long)L * E, 4 * E, 256))
+      !make_map(&w->mB_4e.n256, w->wt_4e, (long long)L * E, 4 * E, 256) ||
+      !make_map(&w->mC_qkv, w->qkv, R, 3 * E, 32) || !make_map(&w->mC_q, w->qkv, R, E, 32) ||
+      !make_map(&w->mC_hid, w->hid, R, 4 * E, 32))
     return fail(EVO_ERR_CUDA);
   if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
       gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
@@ -1035,23 +1042,23 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
     q.rbias_mod = w->n_obs;
     q.out = w->cx16;
     q.ldo = E;
-    WCK(gemm<tc::EPI_BF16>(w->mA_obs, w->mB_obs, q, tp, E, w->num_sms, pdl, st));
+    WCK(gemm<tc::EPI_BF16>(w->mA_obs, w->mB_obs, w->mC_cx, q, tp, E, w->num_sms, pdl, st));
     q.rbias = nullptr;
     q.K = E;
     q.bias = w->wf32 + w->woff[W_CM_B1];
     q.out = w->ch16;
     q.ldo = 4 * E;
-    WCK(gemm<tc::EPI_MISH_BF16>(w->mA_cx, w->mB_cw1, q, tp, 4 * E, w->num_sms, pdl, st));
+    WCK(gemm<tc::EPI_MISH_BF16>(w->mA_cx, w->mB_cw1, w->mC_ch, q, tp, 4 * E, w->num_sms, pdl, st));
     q.K = 4 * E;
     q.bias = w->wf32 + w->woff[W_CM_B2];
     q.out = w->cm16;
     q.ldo = E;
-    WCK(gemm<tc::EPI_BF16>(w->mA_ch, w->mB_cw2, q, tp, E, w->num_sms, pdl, st));
+    WCK(gemm<tc::EPI_BF16>(w->mA_ch, w->mB_cw2, w->mC_cm, q, tp, E, w->num_sms, pdl, st));
     q.K = E;
     q.bias = w->bkv;
     q.out32 = c.kv_obs;
     q.ldo = L * 2 * E;
-    WCK(gemm<tc::EPI_F32>(w->mA_cm, w->mB_kv, q, tp, L * 2 * E, w->num_sms, pdl, st));
+    WCK(gemm<tc::EPI_F32>(w->mA_cm, w->mB_kv, w->mC_cm, q, tp, L * 2 * E, w->num_sms, pdl, st));
   }
   WCK(launch_pdl(pdl, first_kernel, dim3(c.n_sched), dim3(64), 0, st, lat, c.n_sched, w->first, w->mask));
 
@@ -1151,13 +1158,13 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
       g.bias = wl(w, l, WL_SA_BQKV);
       g.out = w->qkv;
       g.ldo = 3 * E;
-      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, 3 * E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, w->mC_qkv, g, Rp, 3 * E, w->num_sms, pdl, st));
       ap.qkv = w->qkv;
       WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, false> : attn_mma_kernel<1, false>, attn_grid,
                      dim3(SA_WARPS * 32), sa_smem, st, ap));
       g.b_row0 = rowE + 3 * E;
       g.bias = wl(w, l, WL_SA_BO);
-      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else if (u == 1) {
       g.K = E;
@@ -1165,13 +1172,13 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
       g.bias = wl(w, l, WL_CA_BQ);
       g.out = w->qkv;
       g.ldo = E;
-      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_BF16>(w->mA_xln, w->mB_e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
       ap.qkv = w->qkv;
       WCK(launch_pdl(pdl, H == 32 ? attn_mma_kernel<2, true> : attn_mma_kernel<1, true>, attn_grid,
                      dim3(SA_WARPS * 32), ca_smem, st, ap));
       g.b_row0 = rowE + 5 * E;
       g.bias = wl(w, l, WL_CA_BO);
-      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else {
       g.K = E;
@@ -1179,11 +1186,11 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
       g.bias = wl(w, l, WL_FF_B1);
       g.out = w->hid;
       g.ldo = 4 * E;
-      WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, g, Rp, 4 * E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_GELU_BF16>(w->mA_xln, w->mB_e, w->mC_hid, g, Rp, 4 * E, w->num_sms, pdl, st));
       g.K = 4 * E;
       g.b_row0 = l * E;
       g.bias = wl(w, l, WL_FF_B2);
-      WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     }
   }
