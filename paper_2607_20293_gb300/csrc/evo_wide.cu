@@ -177,6 +177,13 @@ struct Walk {
   const float* pos;               // [H][E]
   float* trace;                   // [T][U][rows][E] or null: the residual added at every cell (debug)
   int* status;                    // device status word (index checks of the debug build)
+  // when every sample shares one lattice: per step of the walk, the units that
+  // are skipped with a valid cache (host-computed, so the cache loads need not
+  // wait for a lookup), for steps t0 .. t0 + n_umask - 1; and whether b0 refreshes
+  static constexpr int MAX_UMASK = 16;
+  uint64_t umask[MAX_UMASK];
+  int n_umask;
+  int b0_refresh;                 // -1: look it up per row
   int t0, b0;                     // the unit whose output the launch adds (b0 < 0: start of the call)
   int t1, b1;                     // the next cell some lattice refreshes (t1 = T: none, the call ends)
 };
@@ -223,9 +230,14 @@ __device__ __forceinline__ float* trace_row(const Walk& p, int t, int k, int row
 template <int NV>
 __device__ __forceinline__ void skip_run(const Walk& p, int sample, int row, int lane, int t, int b, int bend,
                                          float4 (&v)[NV]) {
-  const uint64_t* mk = p.lat.mask + ((long long)(sample / p.lat.per_sched) * p.lat.T + t) * 2;
   const uint64_t range = (bend >= 64 ? ~0ull : (1ull << bend) - 1ull) & ~((1ull << b) - 1ull);
-  uint64_t m = ~mk[0] & mk[1] & range;                // skipped units whose cache holds a value
+  uint64_t m;                                         // skipped units whose cache holds a value
+  if (t - p.t0 < p.n_umask && t >= p.t0) {
+    m = p.umask[t - p.t0] & range;
+  } else {
+    const uint64_t* mk = p.lat.mask + ((long long)(sample / p.lat.per_sched) * p.lat.T + t) * 2;
+    m = ~mk[0] & mk[1] & range;
+  }
   if (p.trace) {
     // debug: the value every skipped cell adds, as stored (a cache never written adds 0)
     for (int k = b; k < bend; ++k) {
@@ -419,7 +431,7 @@ __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
     float4 r[NV];
     ld4<NV>(v, p.a + (long long)row * p.E, lane);
     ld4<NV>(r, p.r + (long long)row * p.E, lane);
-    if (lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0)) {
+    if (p.b0_refresh >= 0 ? p.b0_refresh != 0 : lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0)) {
 #pragma unroll
       for (int j = 0; j < NV; ++j) {
         v[j].x += r[j].x;
@@ -1095,6 +1107,40 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
   for (int t = 0; t < T; ++t)
     for (int b = 0; b < U; ++b)
       if (w->any[(size_t)b * T + t]) cells.push_back(t * U + b);
+  // one lattice for every sample: the walks' skip masks are known here
+  const bool uniform = c.n_sched == 1;
+  std::vector<uint64_t> skipm;
+  if (uniform) {
+    std::vector<int> first(U, T);
+    for (int b = 0; b < U; ++b) {
+      const int r = c.S_rows == U ? b : b / 3;
+      if (w->force) first[b] = 0;
+      else
+        for (int t = 0; t < T; ++t)
+          if (c.S_host[(size_t)r * T + t]) {
+            first[b] = t;
+            break;
+          }
+    }
+    skipm.assign(T, 0);
+    for (int t = 0; t < T; ++t)
+      for (int b = 0; b < U; ++b) {
+        const int r = c.S_rows == U ? b : b / 3;
+        const bool ref = (w->force && t == 0) || c.S_host[(size_t)r * T + t];
+        if (!ref && first[b] < t) skipm[t] |= 1ull << b;
+      }
+  }
+  auto set_umask = [&]() {
+    wp.n_umask = 0;
+    wp.b0_refresh = -1;
+    if (!uniform) return;
+    wp.n_umask = std::min(Walk::MAX_UMASK, T - wp.t0);
+    for (int i = 0; i < wp.n_umask; ++i) wp.umask[i] = skipm[wp.t0 + i];
+    if (wp.b0 >= 0) {
+      const int r = c.S_rows == U ? wp.b0 : wp.b0 / 3;
+      wp.b0_refresh = ((w->force && wp.t0 == 0) || c.S_host[(size_t)r * T + wp.t0]) ? 1 : 0;
+    }
+  };
   auto set_next = [&](size_t i) {
     if (i < cells.size()) {
       wp.t1 = cells[i] / U;
@@ -1107,6 +1153,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
   wp.t0 = 0;
   wp.b0 = -1;
   set_next(0);
+  set_umask();
   WCK(walk(wp, pdl, st));
 
   tc::GemmArgs g{};
@@ -1151,6 +1198,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
     wp.t0 = t;
     wp.b0 = b;
     set_next(i + 1);
+    set_umask();
     const int rowE = l * 10 * E;
     if (u == 0) {
       g.K = E;
