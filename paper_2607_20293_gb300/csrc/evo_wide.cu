@@ -523,17 +523,26 @@ __global__ void __launch_bounds__(SA_WARPS * 32) attn_mma_kernel(const AttnArgs 
       cp_async16(sq + i * SA_LDS + ch * 8, base + (long long)i * E + ch * 8);
     }
     const int Cm = 1 + p.n_obs;
-    for (int c = lane; c < NK * SA_DH / 2; c += 32) {   // pairs of head dims of every (padded) key
-      const int j = c / (SA_DH / 2), d = 2 * (c % (SA_DH / 2));
-      float2 kk = make_float2(0.f, 0.f), vv = make_float2(0.f, 0.f);
+    // pairs of head dims of every (padded) key: all of a lane's loads are issued
+    // before any is used (the keys/values come from DRAM)
+    constexpr int PER = NK * SA_DH / 2 / 32;
+    float2 kk[PER], vv[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int c = lane + 32 * i, j = c / (SA_DH / 2), d = 2 * (c % (SA_DH / 2));
+      kk[i] = vv[i] = make_float2(0.f, 0.f);
       if (j < Cm) {
         const float* src = j == 0 ? p.kv_time + ((long long)p.t * p.L + p.l) * 2 * E
                                   : p.kv_obs + (((long long)(s % p.obs_mod) * p.n_obs + (j - 1)) * p.L + p.l) * 2 * E;
-        kk = *reinterpret_cast<const float2*>(src + h * SA_DH + d);
-        vv = *reinterpret_cast<const float2*>(src + E + h * SA_DH + d);
+        kk[i] = *reinterpret_cast<const float2*>(src + h * SA_DH + d);
+        vv[i] = *reinterpret_cast<const float2*>(src + E + h * SA_DH + d);
       }
-      *reinterpret_cast<__nv_bfloat162*>(sk + j * SA_LDS + d) = __floats2bfloat162_rn(kk.x, kk.y);
-      *reinterpret_cast<__nv_bfloat162*>(sv + j * SA_LDS + d) = __floats2bfloat162_rn(vv.x, vv.y);
+    }
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int c = lane + 32 * i, j = c / (SA_DH / 2), d = 2 * (c % (SA_DH / 2));
+      *reinterpret_cast<__nv_bfloat162*>(sk + j * SA_LDS + d) = __floats2bfloat162_rn(kk[i].x, kk[i].y);
+      *reinterpret_cast<__nv_bfloat162*>(sv + j * SA_LDS + d) = __floats2bfloat162_rn(vv[i].x, vv[i].y);
     }
   }
   cp_async_wait_all();
