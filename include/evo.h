@@ -208,6 +208,18 @@ evo_status evo_denoise_noalloc(evo_handle* h, const float* obs, const float* noi
  * it); the handle stays usable.  EVO_ERR_ARG for other helpers or limits. */
 evo_status evo_test_wait_timeout(evo_handle* h, int32_t helper, int64_t limit, void* stream);
 
+/* Diagnostic of the feed-forward activation (the paper has no counterpart).
+ * The FFN units of both paths apply GELU in its erf form, x·Phi(x) =
+ * x/2 (1 + erf(x / sqrt 2)) (the denoiser of Sec. 3.1), evaluating erf with
+ * formula 7.1.26 of Abramowitz & Stegun (absolute error <= 1.5e-7).  This
+ * entry point applies that same device code to n fp32 values: y[i] =
+ * GELU(x[i]), x and y DEVICE pointers (caller-owned, n floats each; they may be
+ * the same buffer), asynchronous on `stream`.  packed = 0 runs the scalar form
+ * of the denoising-loop kernel, packed = 1 the two-value (f32x2) form of the
+ * tensor-core GEMM epilogue; the two give identical bits.  EVO_ERR_ARG for
+ * n < 0, another `packed`, or host / null pointers; n = 0 launches nothing. */
+evo_status evo_test_gelu(const float* x, float* y, int64_t n, int32_t packed, void* stream);
+
 /* Debug aid (the paper has no counterpart): every activation buffer of the
  * handle (unit caches, and on the batch-wide path the residual stream and the
  * GEMM operands) is allocated with a 4 KiB guard band of a fixed pattern on

@@ -88,6 +88,7 @@ def load(debug: bool = False) -> ctypes.CDLL:
         "evo_denoise_noalloc": (I32, [P, P, P, P, I32, I32, P, P]),
         "evo_test_wait_timeout": (I32, [P, I32, ctypes.c_int64, P]),
         "evo_check_guards": (I32, [P]),
+        "evo_test_gelu": (I32, [P, P, ctypes.c_int64, I32, P]),
         "evo_denoise_population": (I32, [P, P, P, P, I32, I32, I32, P, P, P]),
         "evo_flops": (I32, [P, P, I32, ctypes.POINTER(I64)]),
         "evo_flops_cfg": (I32, [cfgp, P, I32, ctypes.POINTER(I64)]),
@@ -329,6 +330,16 @@ def redundancy_map(trace, metric: str = "cosine", stream=None):
     _check(lib.evo_redundancy_map(_ptr(trace), T, U, N, n, m, _ptr(d), _ptr(scratch), _stream(stream)),
            "evo_redundancy_map")
     return d
+
+
+def test_gelu(x, packed: bool = False, stream=None):
+    """evo_test_gelu: the feed-forward units' device GELU (scalar form, or the
+    packed pair form of the GEMM epilogue) applied to a contiguous fp32 CUDA
+    tensor (a new tensor of the same shape)."""
+    import torch
+    y = torch.empty_like(x)
+    _check(load().evo_test_gelu(_ptr(x), _ptr(y), x.numel(), int(packed), _stream(stream)), "evo_test_gelu")
+    return y
 
 
 def guided_schedules(d, K: int, rnd, eps: float = 0.05, gamma: int = 2, stream=None):

@@ -1167,6 +1167,13 @@ evo_status evo_test_wait_timeout(evo_handle* h, int32_t helper, int64_t limit, v
   return EVO_OK;
 }
 
+evo_status evo_test_gelu(const float* x, float* y, int64_t n, int32_t packed, void* stream) {
+  if (n < 0 || (packed != 0 && packed != 1) || (n > 0 && (!x || !y))) return EVO_ERR_ARG;
+  if (n > 0 && (!is_device_ptr(x) || !is_device_ptr(y))) return EVO_ERR_ARG;
+  EVO_CUDA(launch_gelu_probe(x, y, n, packed, reinterpret_cast<cudaStream_t>(stream)));
+  return EVO_OK;
+}
+
 evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop) {
   if (!h || (start == nullptr) != (stop == nullptr)) return EVO_ERR_ARG;
   h->prof_start = reinterpret_cast<cudaEvent_t>(start);

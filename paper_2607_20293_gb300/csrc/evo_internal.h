@@ -67,6 +67,108 @@ __device__ __forceinline__ void settle_after_timeout(const int* status, bool dea
   while (clock64() - t0 < SETTLE_CYCLES) __nanosleep(1000);
 }
 
+// fp32 arithmetic with subnormal inputs and results flushed to zero, scalar and
+// packed in pairs (one f32x2 instruction for two values; each half rounds and
+// flushes exactly like the scalar operation).
+__device__ __forceinline__ float fma_z(float a, float b, float c) {
+  float d;
+  asm("fma.rn.ftz.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ float mul_z(float a, float b) {
+  float d;
+  asm("mul.rn.ftz.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+  return d;
+}
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+      " fma.rn.ftz.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " mul.rn.ftz.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+// exact IEEE addition (no flush): the bias adds of the GEMM epilogues
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+      " add.rn.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+// max(x, 0) that keeps NaN
+__device__ __forceinline__ float relu_nan(float x) {
+  float r;
+  asm("max.NaN.f32 %0, %1, 0f00000000;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// The erf-form GELU of the feed-forward units, x·Φ(x) = ½x(1 + erf(x/√2)),
+// with erf from Abramowitz & Stegun, Handbook of Mathematical Functions,
+// formula 7.1.26 (Hastings' rational form): for z ≥ 0
+//   erf z = 1 − (a1 t + a2 t² + a3 t³ + a4 t⁴ + a5 t⁵) e^(−z²) + ε,  t = 1/(1 + p z),
+// |ε| ≤ 1.5e-7.  With z = |x|/√2 and h = ½|x|·(1 − erf z) ≥ 0 the unit is
+// max(x, 0) − h (one fused multiply-add).  |x| is capped at 16 inside h, where e^(−z²) has long
+// underflowed to 0, so ±inf give inf / 0 and NaN stays NaN; subnormal
+// intermediates (|x| beyond ~13, or subnormal x) flush to zero, an absolute
+// change below 1e-37.  One reciprocal and one base-2 exponential on the
+// special-function unit.  gelu_as2 evaluates two values with packed f32x2
+// arithmetic, rounding and flushing exactly as gelu_as does.
+namespace gelu_k {
+constexpr float P = 0.3275911f * 0.70710678118654752f;                       // p / √2
+constexpr float A1 = 0.5f * 0.254829592f, A2 = 0.5f * -0.284496736f, A3 = 0.5f * 1.421413741f,
+                A4 = 0.5f * -1.453152027f, A5 = 0.5f * 1.061405429f;          // ½ a_i
+constexpr float C = -0.72134752044448170f;                                    // −log2(e) / 2
+constexpr float XMAX = 16.f;
+}  // namespace gelu_k
+
+__device__ __forceinline__ float gelu_as(float x) {
+  using namespace gelu_k;
+  const float ax = fminf(fabsf(x), XMAX);
+  const float t = rcp_approx(fma_z(P, ax, 1.f));
+  const float g = ex2_approx(mul_z(ax, mul_z(ax, C)));                          // e^(−x²/2)
+  float q = fma_z(t, A5, A4);
+  q = fma_z(t, q, A3);
+  q = fma_z(t, q, A2);
+  q = fma_z(t, q, A1);
+  const float w = mul_z(mul_z(t, q), g);                                        // ½(1 − erf z)
+  return fma_z(-ax, w, relu_nan(x));                                            // max(x, 0) − |x| w, one rounding
+}
+
+__device__ __forceinline__ float2 gelu_as2(float2 x) {
+  using namespace gelu_k;
+  const float2 ax = make_float2(fminf(fabsf(x.x), XMAX), fminf(fabsf(x.y), XMAX));
+  const float2 u = fma2(make_float2(P, P), ax, make_float2(1.f, 1.f));
+  const float2 t = make_float2(rcp_approx(u.x), rcp_approx(u.y));
+  const float2 s = mul2(ax, mul2(ax, make_float2(C, C)));
+  const float2 g = make_float2(ex2_approx(s.x), ex2_approx(s.y));
+  float2 q = fma2(t, make_float2(A5, A5), make_float2(A4, A4));
+  q = fma2(t, q, make_float2(A3, A3));
+  q = fma2(t, q, make_float2(A2, A2));
+  q = fma2(t, q, make_float2(A1, A1));
+  const float2 w = mul2(mul2(t, q), g);
+  return fma2(make_float2(-ax.x, -ax.y), w, make_float2(relu_nan(x.x), relu_nan(x.y)));
+}
+
 // Byte offsets of the regions of one CTA's dynamic shared memory.
 struct SmemLayout {
   int ring;    // nslot * slot_bytes: weight slabs (with the unit's LayerNorm/bias vectors) streamed by the producer warp
@@ -166,6 +268,7 @@ cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_
 // the loop kernel's helper (helper 0, limit in cycles) or the tensor-core
 // kernels' helper (helper 1, limit in polls); the wait gives up and sets ST_TIMEOUT
 cudaError_t launch_wait_probe(int helper, long long limit, int* status, cudaStream_t s);
+cudaError_t launch_gelu_probe(const float* x, float* y, long long n, int packed, cudaStream_t s);
 cudaError_t launch_pop_dev(const float* x, int P, int N_obs, int HA, float* dev, cudaStream_t s);
 
 // batch-wide path (evo_wide.cu)

@@ -485,6 +485,29 @@ cudaError_t launch_wait_probe(int helper, long long limit, int* status, cudaStre
   return cudaGetLastError();
 }
 
+// The feed-forward units' GELU applied to n values: the scalar form of the
+// loop kernel (packed = 0) or the packed pair form of the tensor-core GEMM's
+// epilogue (packed = 1; an odd last value takes the scalar form).
+__global__ void gelu_probe_kernel(const float* x, float* y, long long n, int packed) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < (n + 1) / 2; i += stride) {
+    if (packed && 2 * i + 1 < n) {
+      const float2 r = gelu_as2(make_float2(x[2 * i], x[2 * i + 1]));
+      y[2 * i] = r.x;
+      y[2 * i + 1] = r.y;
+    } else {
+      y[2 * i] = gelu_as(x[2 * i]);
+      if (2 * i + 1 < n) y[2 * i + 1] = gelu_as(x[2 * i + 1]);
+    }
+  }
+}
+
+cudaError_t launch_gelu_probe(const float* x, float* y, long long n, int packed, cudaStream_t s) {
+  if (n > 0)
+    gelu_probe_kernel<<<(int)std::min<long long>((n + 511) / 512, 4096), 256, 0, s>>>(x, y, n, packed);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_validate(const uint8_t* S, long long n, int* err, cudaStream_t s) {
   validate_kernel<<<1, 256, 0, s>>>(S, n, err);
   return cudaGetLastError();

@@ -489,7 +489,7 @@ struct Loop {
                 const float v0 = acc[mt][i][2 * h] + bv[i].x, v1 = acc[mt][i][2 * h + 1] + bv[i].y;
                 if constexpr (U == 2) {
                   *reinterpret_cast<__nv_bfloat162*>(hid + m * S::ldh + n) =
-                      __floats2bfloat162_rn(gelu_erf(v0), gelu_erf(v1));
+                      __floats2bfloat162_rn(gelu_as(v0), gelu_as(v1));
                 } else if constexpr (MMA_ATT) {
                   // q -> Q[i], k -> K[i], v -> V[i] of sample m / H
                   __nv_bfloat16* st = reinterpret_cast<__nv_bfloat16*>(att_stage(p, cx)) +
@@ -524,7 +524,7 @@ struct Loop {
           const int m = o / N, n = o % N;
           const float v = acc[i] + bv[i];
           if constexpr (U == 2)
-            hid[m * S::ldh + n] = from_f<T>(gelu_erf(v));
+            hid[m * S::ldh + n] = from_f<T>(gelu_as(v));
           else
             g1[m * S::ldg1 + n] = v;
         }

@@ -17,9 +17,11 @@
 //     staging rows in shared memory in the 128-byte-swizzled layout, and
 //     writes each 32 x 64 block with one tiled bulk store (the thread-per-row
 //     layout of the accumulator would scatter every direct store over 32
-//     rows), then releases the accumulator.  The residual mode (the output projection of a refreshed
-//     unit) stages fp32 and, row by row, stores r and the unit's bf16 cache
-//     (Eq. 1) for the rows that refresh the unit.
+//     rows), releasing the accumulator as soon as its last columns are in
+//     registers.  The residual mode (the output projection of a refreshed
+//     unit) stages fp32 r and stores it (a tiled bulk store through tmC, an
+//     fp32 map of r, when all 32 rows of a warp refresh the unit) together
+//     with the unit's bf16 cache (Eq. 1) for the rows that refresh the unit.
 // With two accumulators the epilogue of one tile overlaps the main loop of the
 // next.  BN = 256 for large problems, 128 when that leaves SMs idle.
 //
@@ -219,8 +221,6 @@ __device__ __forceinline__ float mish_f(float v) {
   return v * tanhf(sp);
 }
 
-__device__ __forceinline__ float gelu_exact(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
-
 // does any row of the tile starting at m0 refresh?  (the same answer in every role)
 __device__ __forceinline__ bool tile_live(const GemmArgs& g, int m0) {
   if (m0 >= g.rows) return false;
@@ -231,35 +231,41 @@ __device__ __forceinline__ bool tile_live(const GemmArgs& g, int m0) {
   return false;
 }
 
-// bias (and GELU) on 32 accumulator columns n .. n + 31 of this thread's row,
-// packed to bf16 and written as 64 bytes of the thread's staging row (chunks
-// j4 .. j4 + 3 of 16 bytes, swizzled by the row within the 8-row group)
+// (a, b) += (c, d) as one packed add
+__device__ __forceinline__ void add2_into(float& a, float& b, float c, float d) {
+  const float2 r = add2(make_float2(a, b), make_float2(c, d));
+  a = r.x;
+  b = r.y;
+}
+
+// bias (and GELU / Mish) on 32 accumulator columns n .. n + 31 of this
+// thread's row, packed to bf16: pk[q] = columns 8q .. 8q + 7 (registers only,
+// so that this work overlaps the bulk store still reading the staging rows)
 template <int MODE>
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n, float (&v)[32], uint8_t* srow,
-                                               int lane, int j4) {
+__device__ __forceinline__ void epilogue_values(const GemmArgs& g, int row, int n, float (&v)[32], uint4* pk) {
   const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
     const float4 bb = __ldg(b4 + q);
-    v[4 * q] += bb.x;
-    v[4 * q + 1] += bb.y;
-    v[4 * q + 2] += bb.z;
-    v[4 * q + 3] += bb.w;
+    add2_into(v[4 * q], v[4 * q + 1], bb.x, bb.y);
+    add2_into(v[4 * q + 2], v[4 * q + 3], bb.z, bb.w);
   }
   if (g.rbias) {
     const float4* r4 = reinterpret_cast<const float4*>(g.rbias + (long long)(row % g.rbias_mod) * g.ldo + n);
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
       const float4 bb = __ldg(r4 + q);
-      v[4 * q] += bb.x;
-      v[4 * q + 1] += bb.y;
-      v[4 * q + 2] += bb.z;
-      v[4 * q + 3] += bb.w;
+      add2_into(v[4 * q], v[4 * q + 1], bb.x, bb.y);
+      add2_into(v[4 * q + 2], v[4 * q + 3], bb.z, bb.w);
     }
   }
   if constexpr (MODE == EPI_GELU_BF16) {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = gelu_exact(v[i]);
+    for (int i = 0; i < 16; ++i) {
+      const float2 y = gelu_as2(make_float2(v[2 * i], v[2 * i + 1]));
+      v[2 * i] = y.x;
+      v[2 * i + 1] = y.y;
+    }
   }
   if constexpr (MODE == EPI_MISH_BF16) {
 #pragma unroll
@@ -267,54 +273,70 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int row, int n
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    uint4 pk;
-    uint32_t* pw = reinterpret_cast<uint32_t*>(&pk);
+    uint32_t* pw = reinterpret_cast<uint32_t*>(&pk[q]);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       __nv_bfloat162 h2 = __floats2bfloat162_rn(v[8 * q + 2 * j], v[8 * q + 2 * j + 1]);
       pw[j] = *reinterpret_cast<uint32_t*>(&h2);
     }
-    *reinterpret_cast<uint4*>(srow + (((j4 + q) ^ (lane & 7)) << 4)) = pk;
-  }
-}
-
-// the warp's staged 32 rows x 64 columns to global memory: 4 rows of 128
-// contiguous bytes per store instruction
-__device__ __forceinline__ void epilogue_flush(const GemmArgs& g, const uint8_t* stg, int row0, int n, int lane) {
-  const int cc = lane & 7;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int r = 4 * i + (lane >> 3);
-    const uint4 val = *reinterpret_cast<const uint4*>(stg + r * 128 + ((cc ^ (r & 7)) << 4));
-    if (row0 + r < g.rows) *reinterpret_cast<uint4*>(g.out + (long long)(row0 + r) * g.ldo + n + 8 * cc) = val;
   }
 }
 
 // EPI_RESID, one chunk of 32 columns n .. n + 31: r = acc + bias goes to the
-// warp's staging rows (fp32, thread = row), then the warp takes the rows one
-// at a time (lane = column, 128 contiguous bytes) and, for the rows whose
-// lattice refreshes the unit (bit r of rmask), stores r and c_b <- bf16(r)
-// (Eq. 1).  The row walk that follows adds r to the residual stream.
-__device__ __forceinline__ void epilogue_resid(const GemmArgs& g, int row0, int n, float (&v)[32], uint8_t* stg,
-                                               int lane, unsigned rmask) {
+// warp's staging rows (fp32, thread = row, the 128-byte-swizzled layout of a
+// 32 x 32 fp32 box), then for the rows whose lattice refreshes the unit (bit r
+// of rmask) r is stored -- by one tiled bulk store through tmR when all 32 rows
+// refresh (and no trace is taken), else by the warp (eight lanes per row, 16
+// bytes each) -- and c_b <- bf16(r) (Eq. 1) by the warp (four lanes per row,
+// eight values each), reading the staging rows alongside the bulk store.  The
+// row walk that follows adds r to the residual stream.
+__device__ __forceinline__ void epilogue_resid(const GemmArgs& g, const CUtensorMap* tmR, int row0, int n,
+                                               float (&v)[32], uint8_t* stg, int lane, unsigned rmask) {
+  const bool bulk = rmask == 0xffffffffu && !g.trace;
+  if (lane == 0) bulk_wait_read();   // the previous chunk's bulk store has left the staging rows
+  __syncwarp();
   const float4* b4 = reinterpret_cast<const float4*>(g.bias + n);
   uint8_t* srow = stg + lane * 128;
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
     const float4 bb = __ldg(b4 + q);
+    add2_into(v[4 * q], v[4 * q + 1], bb.x, bb.y);
+    add2_into(v[4 * q + 2], v[4 * q + 3], bb.z, bb.w);
     *reinterpret_cast<float4*>(srow + ((q ^ (lane & 7)) << 4)) =
-        make_float4(v[4 * q] + bb.x, v[4 * q + 1] + bb.y, v[4 * q + 2] + bb.z, v[4 * q + 3] + bb.w);
+        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
   }
+  if (bulk) fence_async_smem();
   __syncwarp();
-  const long long col = n + lane;
-#pragma unroll 8
-  for (int r = 0; r < 32; ++r) {
-    if (!((rmask >> r) & 1u)) continue;
-    const float rv = *reinterpret_cast<const float*>(stg + r * 128 + (((lane >> 2) ^ (r & 7)) << 4) + (lane & 3) * 4);
-    const long long o = (long long)(row0 + r) * g.ldr + col;
-    g.rout[o] = rv;
-    g.cache[o] = __float2bfloat16_rn(rv);
-    if (g.trace) g.trace[o] = rv;
+  if (bulk) {
+    if (lane == 0) {
+      tma_store_2d(tmR, n, row0, stg);
+      bulk_commit();
+    }
+  } else {
+    const int cc = lane & 7;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int r = 4 * i + (lane >> 3);
+      if ((rmask >> r) & 1u) {
+        const float4 val = *reinterpret_cast<const float4*>(stg + r * 128 + ((cc ^ (r & 7)) << 4));
+        const long long o = (long long)(row0 + r) * g.ldr + n + 4 * cc;
+        *reinterpret_cast<float4*>(g.rout + o) = val;
+        if (g.trace) *reinterpret_cast<float4*>(g.trace + o) = val;
+      }
+    }
+  }
+  const int cp = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = 8 * i + (lane >> 2);
+    if ((rmask >> r) & 1u) {
+      const float4 f0 = *reinterpret_cast<const float4*>(stg + r * 128 + (((2 * cp) ^ (r & 7)) << 4));
+      const float4 f1 = *reinterpret_cast<const float4*>(stg + r * 128 + (((2 * cp + 1) ^ (r & 7)) << 4));
+      __nv_bfloat162 h[4] = {__floats2bfloat162_rn(f0.x, f0.y), __floats2bfloat162_rn(f0.z, f0.w),
+                             __floats2bfloat162_rn(f1.x, f1.y), __floats2bfloat162_rn(f1.z, f1.w)};
+      *reinterpret_cast<uint4*>(g.cache + (long long)(row0 + r) * g.ldr + n + 8 * cp) =
+          *reinterpret_cast<const uint4*>(h);
+    }
   }
   __syncwarp();
 }
@@ -339,6 +361,14 @@ __device__ __forceinline__ void epilogue_f32(const GemmArgs& g, int row0, int n,
         *reinterpret_cast<const float*>(stg + r * 128 + (((lane >> 2) ^ (r & 7)) << 4) + (lane & 3) * 4);
   }
   __syncwarp();
+}
+
+// the warp has read its last columns of the accumulator (tcgen05.ld waited):
+// one arrival of the EPI_WARPS that free it for the next tile's main loop
+__device__ __forceinline__ void release_acc(uint64_t* tempty, int lane) {
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive1(tempty);
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -444,7 +474,8 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
         for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
           float v[32];
           tmem_ld32(tq + (uint32_t)(c * 32), v);
-          epilogue_resid(g, m0 + quad * 32, n0 + c * 32, v, stg, lane, rmask);
+          if (c + 1 == (half + 1) * (BN / 64)) release_acc(&tempty[acc], lane);   // last columns are in registers
+          epilogue_resid(g, &tmC, m0 + quad * 32, n0 + c * 32, v, stg, lane, rmask);
         }
       } else {
         // 32 rows x 64 columns at a time: packed into the staging rows (the
@@ -452,14 +483,19 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
         // whole block by lane 0 (out of range rows land in the buffer's padding)
 #pragma unroll 1
         for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); c += 2) {
-          if (lane == 0) bulk_wait_read();               // the previous block has left the staging rows
-          __syncwarp();
+          uint4 pk[8];
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
             float v[32];
             tmem_ld32(tq + (uint32_t)((c + j) * 32), v);
-            epilogue_chunk<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, stg + lane * 128, lane, 4 * j);
+            epilogue_values<MODE>(g, m0 + quad * 32 + lane, n0 + (c + j) * 32, v, pk + 4 * j);
           }
+          if (c + 2 == (half + 1) * (BN / 64)) release_acc(&tempty[acc], lane);
+          if (lane == 0) bulk_wait_read();               // the previous block has left the staging rows
+          __syncwarp();
+          uint8_t* srow = stg + lane * 128;
+#pragma unroll
+          for (int q = 0; q < 8; ++q) *reinterpret_cast<uint4*>(srow + ((q ^ (lane & 7)) << 4)) = pk[q];
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
@@ -468,9 +504,7 @@ __global__ void __launch_bounds__(NTHREADS_GEMM, 1) gemm_kernel(const __grid_con
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive1(&tempty[acc]);
+      if constexpr (MODE == EPI_F32) release_acc(&tempty[acc], lane);
       ++it;
     }
   }

@@ -69,6 +69,20 @@ bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_r
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// fp32 matrix [rows][cols], cols contiguous, in boxes of 32 x 32 with the
+// 128-byte swizzle (the residual GEMM's bulk stores of r)
+bool make_map_f32(CUtensorMap* m, const void* base, long long rows, int cols) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 4};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t es[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 uint16_t bf16_bits(float f) {
   uint32_t u;
   std::memcpy(&u, &f, 4);
@@ -700,6 +714,7 @@ struct WideState {
   CUtensorMap mA_obs, mA_cx, mA_ch, mA_cm;
   // tiled-store maps of the bf16 GEMM outputs (32-row x 64-column boxes)
   CUtensorMap mC_qkv, mC_q, mC_hid, mC_cx, mC_ch, mC_cm;
+  CUtensorMap mC_r;                 // fp32 r (rbuf), 32 x 32 boxes: the residual GEMM's bulk stores
   BMaps mB_obs, mB_cw1, mB_cw2, mB_kv;
   int num_sms = 0;
   GuardList guards;                 // guard bands of the activation buffers
@@ -952,7 +967,7 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
       !make_map(&w->mB_4e.n128, w->wt_4e, (long long)L * E, 4 * E, 128) ||
       !make_map(&w->mB_4e.n256, w->wt_4e, (long long)L * E, 4 * E, 256) ||
       !make_map(&w->mC_qkv, w->qkv, R, 3 * E, 32) || !make_map(&w->mC_q, w->qkv, R, E, 32) ||
-      !make_map(&w->mC_hid, w->hid, R, 4 * E, 32))
+      !make_map(&w->mC_hid, w->hid, R, 4 * E, 32) || !make_map_f32(&w->mC_r, w->rbuf, R, E))
     return fail(EVO_ERR_CUDA);
   if (gemm_attr<tc::EPI_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_BF16, 256>() != cudaSuccess ||
       gemm_attr<tc::EPI_GELU_BF16, 128>() != cudaSuccess || gemm_attr<tc::EPI_GELU_BF16, 256>() != cudaSuccess ||
@@ -1221,7 +1236,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
                      dim3(SA_WARPS * 32), sa_smem, st, ap));
       g.b_row0 = rowE + 3 * E;
       g.bias = wl(w, l, WL_SA_BO);
-      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_r, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else if (u == 1) {
       g.K = E;
@@ -1235,7 +1250,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
                      dim3(SA_WARPS * 32), ca_smem, st, ap));
       g.b_row0 = rowE + 5 * E;
       g.bias = wl(w, l, WL_CA_BO);
-      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_att, w->mB_e, w->mC_r, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     } else {
       g.K = E;
@@ -1247,7 +1262,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
       g.K = 4 * E;
       g.b_row0 = l * E;
       g.bias = wl(w, l, WL_FF_B2);
-      WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, w->mC_q, g, Rp, E, w->num_sms, pdl, st));
+      WCK(gemm<tc::EPI_RESID>(w->mA_hid, w->mB_4e, w->mC_r, g, Rp, E, w->num_sms, pdl, st));
       WCK(walk(wp, pdl, st));
     }
   }
