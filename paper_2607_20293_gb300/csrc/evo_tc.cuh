@@ -334,8 +334,9 @@ __device__ __forceinline__ void epilogue_resid(const GemmArgs& g, const CUtensor
       const float4 f1 = *reinterpret_cast<const float4*>(stg + r * 128 + (((2 * cp + 1) ^ (r & 7)) << 4));
       __nv_bfloat162 h[4] = {__floats2bfloat162_rn(f0.x, f0.y), __floats2bfloat162_rn(f0.z, f0.w),
                              __floats2bfloat162_rn(f1.x, f1.y), __floats2bfloat162_rn(f1.z, f1.w)};
-      *reinterpret_cast<uint4*>(g.cache + (long long)(row0 + r) * g.ldr + n + 8 * cp) =
-          *reinterpret_cast<const uint4*>(h);
+      // the cache is read again only by later walks: evict-first, r stays in L2 for the next walk
+      __stcs(reinterpret_cast<uint4*>(g.cache + (long long)(row0 + r) * g.ldr + n + 8 * cp),
+             *reinterpret_cast<const uint4*>(h));
     }
   }
   __syncwarp();

@@ -214,6 +214,19 @@ __device__ __forceinline__ void ld4(float4 (&v)[NV], const float* src, int lane)
   for (int j = 0; j < NV; ++j) v[j] = *reinterpret_cast<const float4*>(src + 128 * j + 4 * lane);
 }
 
+// the same with the evict-first (streaming) policy
+template <int NV>
+__device__ __forceinline__ void ld4_cs(float4 (&v)[NV], const float* src, int lane) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) v[j] = __ldcs(reinterpret_cast<const float4*>(src + 128 * j + 4 * lane));
+}
+
+template <int NV>
+__device__ __forceinline__ void st4_cs(float* dst, int lane, const float4 (&v)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) __stcs(reinterpret_cast<float4*>(dst + 128 * j + 4 * lane), v[j]);
+}
+
 template <int NV>
 __device__ __forceinline__ void st4(float* dst, int lane, const float4 (&v)[NV]) {
 #pragma unroll
@@ -267,6 +280,10 @@ __device__ __forceinline__ void skip_run(const Walk& p, int sample, int row, int
       st4<NV>(trace_row<NV>(p, t, k, row), lane, c);
     }
   }
+  // The walk streams the unit caches, r and the residual stream with the
+  // evict-first policy (ld/st .cs): none is read again before hundreds of MB
+  // of other traffic, and the L2 then keeps the GEMM operands (xln, q|k|v,
+  // the hidden layer) that the next kernels read.
   const __nv_bfloat16* base = p.cache + (long long)row * p.E + 4 * lane;
   if (!dcheck(bend <= p.lat.U && (long long)row * p.E < p.cache_unit, p.status)) return;
   while (m) {
@@ -280,7 +297,7 @@ __device__ __forceinline__ void skip_run(const Walk& p, int sample, int row, int
         m &= m - 1;
         ++nk;
 #pragma unroll
-        for (int j = 0; j < NV; ++j) raw[q][j] = *reinterpret_cast<const uint2*>(base + k * p.cache_unit + 128 * j);
+        for (int j = 0; j < NV; ++j) raw[q][j] = __ldcs(reinterpret_cast<const uint2*>(base + k * p.cache_unit + 128 * j));
       }
     }
 #pragma unroll
@@ -408,7 +425,7 @@ __device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t
     b = 0;
   }
   if (!dcheck(row < p.rows && p.b1 < p.lat.U && p.t1 < p.lat.T, p.status)) return;
-  st4<NV>(p.a + (long long)row * p.E, lane, v);
+  st4_cs<NV>(p.a + (long long)row * p.E, lane, v);
   if (lat_refresh(p.lat, sample, p.b1, p.t1)) {
     float mean, rstd;
     row_stats<NV>(v, 1.f / (float)p.E, mean, rstd);
@@ -443,8 +460,8 @@ __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
   } else {
     // the stream, unit b0's output and the lattice bit, loaded together
     float4 r[NV];
-    ld4<NV>(v, p.a + (long long)row * p.E, lane);
-    ld4<NV>(r, p.r + (long long)row * p.E, lane);
+    ld4_cs<NV>(v, p.a + (long long)row * p.E, lane);
+    ld4_cs<NV>(r, p.r + (long long)row * p.E, lane);
     if (p.b0_refresh >= 0 ? p.b0_refresh != 0 : lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0)) {
 #pragma unroll
       for (int j = 0; j < NV; ++j) {
