@@ -187,8 +187,8 @@ evo_status evo_set_profile_events(evo_handle* h, void* start, void* stop);
  * in it (186 samples of the Push-T-shaped model), else EVO_ERR_SHAPE and
  * nothing is launched.  No cudaMalloc, cudaFree or allocating library routine
  * is called.  The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) and keeps it; make that first call before any stream
- * capture.  All calls share the array and every call overwrites all of it
+ * (cudaGetSymbolAddress) and keeps it for later calls.  All calls share the
+ * array and every call overwrites all of it
  * that it reads, so nothing needs clearing; calls that overlap on the GPU
  * (other streams, other handles) race on it.  The handle's device must be the
  * current device (EVO_ERR_ARG otherwise). */
