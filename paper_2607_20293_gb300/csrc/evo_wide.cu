@@ -200,6 +200,11 @@ struct Walk {
   int b0_refresh;                 // -1: look it up per row
   int t0, b0;                     // the unit whose output the launch adds (b0 < 0: start of the call)
   int t1, b1;                     // the next cell some lattice refreshes (t1 = T: none, the call ends)
+  // rows of different lattices (walk_kernel<NV, true>): each row is walked
+  // only after the cells its own lattice refreshes, straight to its lattice's
+  // next refreshed cell (rows that skip (t0, b0) have nothing to do in this
+  // launch); one shared lattice: every row to (t1, b1)
+  int per_row;
 };
 
 __device__ __forceinline__ float warp_sum(float s) {
@@ -412,25 +417,35 @@ __device__ __forceinline__ bool head_step(const Walk& p, int row, int sample, in
 
 // Walk the row from step t, unit b (v = the stream before unit b) to the
 // launch's next refreshed cell (t1, b1), or to the end of the call.
+// the first cell after (t, b) that the sample's lattice refreshes, as t * 64 + b
+// (t = T: none)
+__device__ __forceinline__ int next_refresh(const Walk& p, int sample, int t, int b) {
+  const uint64_t* mk = p.lat.mask + (long long)(sample / p.lat.per_sched) * p.lat.T * 2;
+  uint64_t ref = b + 1 >= 64 ? 0ull : mk[2 * t] & (~0ull << (b + 1));
+  while (!ref && ++t < p.lat.T) ref = mk[2 * t];
+  return t < p.lat.T ? t * 64 + __ffsll((long long)ref) - 1 : p.lat.T * 64;
+}
+
 template <int NV>
-__device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t, int b, float4 (&v)[NV]) {
+__device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t, int b, float4 (&v)[NV], int t1,
+                                         int b1) {
   const int sample = row / p.lat.H, tok = row - sample * p.lat.H;
   for (;;) {
-    const bool last = t == p.t1;
-    const int bend = last ? p.b1 : p.lat.U;
+    const bool last = t == t1;
+    const int bend = last ? b1 : p.lat.U;
     if (b < bend) skip_run<NV>(p, sample, row, lane, t, b, bend, v);
     if (last) break;
     if (!head_step<NV>(p, row, sample, tok, lane, t, v)) return;   // the call's last step: x is final
     ++t;
     b = 0;
   }
-  if (!dcheck(row < p.rows && p.b1 < p.lat.U && p.t1 < p.lat.T, p.status)) return;
+  if (!dcheck(row < p.rows && b1 < p.lat.U && t1 < p.lat.T, p.status)) return;
   st4_cs<NV>(p.a + (long long)row * p.E, lane, v);
-  if (lat_refresh(p.lat, sample, p.b1, p.t1)) {
+  if (lat_refresh(p.lat, sample, b1, t1)) {
     float mean, rstd;
     row_stats<NV>(v, 1.f / (float)p.E, mean, rstd);
     float4 y[NV];
-    ln_apply<NV>(y, v, mean, rstd, p.ln_g + (long long)p.b1 * p.E, p.ln_b + (long long)p.b1 * p.E, lane);
+    ln_apply<NV>(y, v, mean, rstd, p.ln_g + (long long)b1 * p.E, p.ln_b + (long long)b1 * p.E, lane);
     __nv_bfloat16* dst = p.xln + (long long)row * p.E + 4 * lane;
 #pragma unroll
     for (int j = 0; j < NV; ++j) *reinterpret_cast<uint2*>(dst + 128 * j) = pack_bf16x4(y[j]);
@@ -438,31 +453,36 @@ __device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t
 }
 
 // One warp per row: the walk from the launch's position to the next refreshed
-// cell.  b0 < 0: the start of a call (x <- noise[0]; a <- x W_in + b_in +
-// P_pos).  Otherwise the rows that refresh unit b0 add its output r (written by
-// the residual GEMM); the walk starts at b0, so rows that skip b0 add its cache.
-template <int NV>
+// cell (PER_ROW: the next cell the row's own lattice refreshes).  b0 < 0: the
+// start of a call (x <- noise[0]; a <- x W_in + b_in + P_pos).  Otherwise the
+// rows that refresh unit b0 add its output r (written by the residual GEMM);
+// the walk starts at b0, so rows that skip b0 add its cache (PER_ROW: such
+// rows are already past b0 and do nothing).
+template <int NV, bool PER_ROW>
 __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
   tc::pdl_trigger();
   tc::pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (row >= p.rows) return;
+  const int sample = row / p.lat.H;
   float4 v[NV];
   if (p.b0 < 0) {
-    const int H = p.lat.H, sample = row / H, tok = row % H;
+    const int H = p.lat.H, tok = row % H;
     float xv = 0.f;
     if (lane < p.A) {
       xv = p.noise[((long long)(sample % p.obs_mod) * H + tok) * p.A + lane];
       p.x[(long long)row * p.A + lane] = xv;
     }
     embed<NV>(p, tok, lane, xv, v);
-    walk_row<NV>(p, row, lane, 0, 0, v);
+    const int nx = PER_ROW ? next_refresh(p, sample, 0, -1) : p.t1 * 64 + p.b1;
+    walk_row<NV>(p, row, lane, 0, 0, v, nx >> 6, nx & 63);
   } else {
+    if (PER_ROW && !lat_refresh(p.lat, sample, p.b0, p.t0)) return;   // the row waits at its own position
     // the stream, unit b0's output and the lattice bit, loaded together
     float4 r[NV];
     ld4_cs<NV>(v, p.a + (long long)row * p.E, lane);
     ld4_cs<NV>(r, p.r + (long long)row * p.E, lane);
-    if (p.b0_refresh >= 0 ? p.b0_refresh != 0 : lat_refresh(p.lat, row / p.lat.H, p.b0, p.t0)) {
+    if (p.b0_refresh >= 0 ? p.b0_refresh != 0 : lat_refresh(p.lat, sample, p.b0, p.t0)) {
 #pragma unroll
       for (int j = 0; j < NV; ++j) {
         v[j].x += r[j].x;
@@ -471,7 +491,8 @@ __global__ void __launch_bounds__(256, 3) walk_kernel(const Walk p) {
         v[j].w += r[j].w;
       }
     }
-    walk_row<NV>(p, row, lane, p.t0, p.b0, v);
+    const int nx = PER_ROW ? next_refresh(p, sample, p.t0, p.b0) : p.t1 * 64 + p.b1;
+    walk_row<NV>(p, row, lane, p.t0, p.b0, v, nx >> 6, nx & 63);
   }
 }
 
@@ -804,8 +825,12 @@ cudaError_t gemm_attr() {
 
 cudaError_t walk(const Walk& p, bool pdl, cudaStream_t st) {
   const dim3 grid((p.rows + 7) / 8), block(256);
-  if (p.E == 256) return launch_pdl(pdl, walk_kernel<2>, grid, block, 0, st, p);
-  if (p.E == 512) return launch_pdl(pdl, walk_kernel<4>, grid, block, 0, st, p);
+  if (p.E == 256)
+    return p.per_row ? launch_pdl(pdl, walk_kernel<2, true>, grid, block, 0, st, p)
+                     : launch_pdl(pdl, walk_kernel<2, false>, grid, block, 0, st, p);
+  if (p.E == 512)
+    return p.per_row ? launch_pdl(pdl, walk_kernel<4, true>, grid, block, 0, st, p)
+                     : launch_pdl(pdl, walk_kernel<4, false>, grid, block, 0, st, p);
   return cudaErrorInvalidValue;
 }
 
@@ -1171,6 +1196,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
         if (!ref && first[b] < t) skipm[t] |= 1ull << b;
       }
   }
+  wp.per_row = uniform ? 0 : 1;
   auto set_umask = [&]() {
     wp.n_umask = 0;
     wp.b0_refresh = -1;
