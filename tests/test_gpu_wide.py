@@ -128,6 +128,32 @@ def test_wide_population_tiles_mix_lattices(torch, B):
     assert dev[5] < 1e-6 * max(1.0, float(dev.max()))      # the all-ones candidate is the reference itself
 
 
+@pytest.mark.parametrize("empty", ["zero", "force"])
+def test_wide_population_edge_lattices(torch, B, empty):
+    # lattices that differ by sample: each row is walked from its own lattice's
+    # refreshed cells to its next one, so a lattice that refreshes only the very
+    # first or the very last cell, only step 0, only the last step, or nothing
+    # at all must still end at the oracle's actions
+    cfg = synth.config("pusht")
+    W = synth.make_weights(cfg, 0)
+    U, T = 24, 100
+    lat = np.zeros((6, U, T), np.uint8)
+    lat[0, 0, 0] = 1                  # the first cell only
+    lat[1, U - 1, T - 1] = 1          # the last cell only
+    lat[2, :, 0] = 1                  # every unit at step 0, then skips to the end
+    lat[3, :, T - 1] = 1              # every unit at the last step only
+    lat[4, ::5, ::7] = 1              # a sparse grid
+    P, N = lat.shape[0], 2            # lattice 5: nothing refreshed
+    obs, noise = synth.make_obs(cfg, N, 51), synth.make_noise(cfg, N, 52)
+    ev = B.Evo(cfg, W, (P + 1) * N, wide_rows=1, empty=empty)
+    x, _ = ev.population(torch.from_numpy(obs).cuda(), torch.from_numpy(noise).cuda(), lat)
+    assert ev.last_call()["path"] == "wide"
+    x = x.cpu().numpy()
+    for p in range(P):
+        want = O.denoise(W, cfg, obs, noise, lat[p], policy=empty)
+        check(x[p], want, f"lattice {p} ({empty})")
+
+
 @pytest.mark.parametrize("force", [False, True])
 def test_wide_trace_eq1_bitwise(torch, B, force):
     """bf16 caches on the batch-wide path: every skipped cell adds exactly the
