@@ -184,9 +184,9 @@ struct Walk {
   int sampler;
   const float* lnf_g;
   const float* lnf_b;
-  const float* head_wt;           // [A][E] (W_head transposed)
+  const __nv_bfloat16* head_wt;   // [A][E] (W_head transposed), bf16 like every weight matrix of this path
   const float* head_b;            // [A]
-  const float* in_w;              // [A][E]
+  const __nv_bfloat16* in_w;      // [A][E], bf16
   const float* in_b;              // [E]
   const float* pos;               // [H][E]
   float* trace;                   // [T][U][rows][E] or null: the residual added at every cell (debug)
@@ -245,6 +245,12 @@ __device__ __forceinline__ void add_bf16x4(float4& v, uint2 raw) {
   v.y += lo.y;
   v.z += hi.x;
   v.w += hi.y;
+}
+
+__device__ __forceinline__ float4 bf16x4_f(uint2 raw) {
+  const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
+  const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
+  return make_float4(lo.x, lo.y, hi.x, hi.y);
 }
 
 __device__ __forceinline__ uint2 pack_bf16x4(float4 v) {
@@ -360,7 +366,7 @@ __device__ __forceinline__ void embed(const Walk& p, int tok, int lane, float xa
     const float xa = __shfl_sync(0xffffffffu, xa_lane, a);
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
-      const float4 w = *reinterpret_cast<const float4*>(p.in_w + (long long)a * p.E + 128 * j + 4 * lane);
+      const float4 w = bf16x4_f(*reinterpret_cast<const uint2*>(p.in_w + (long long)a * p.E + 128 * j + 4 * lane));
       v[j].x = fmaf(xa, w.x, v[j].x);
       v[j].y = fmaf(xa, w.y, v[j].y);
       v[j].z = fmaf(xa, w.z, v[j].z);
@@ -385,7 +391,7 @@ __device__ __forceinline__ bool head_step(const Walk& p, int row, int sample, in
     float part = 0.f;
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
-      const float4 w = *reinterpret_cast<const float4*>(p.head_wt + (long long)a * p.E + 128 * j + 4 * lane);
+      const float4 w = bf16x4_f(*reinterpret_cast<const uint2*>(p.head_wt + (long long)a * p.E + 128 * j + 4 * lane));
       part = fmaf(y[j].x, w.x, part);
       part = fmaf(y[j].y, w.y, part);
       part = fmaf(y[j].z, w.z, part);
@@ -734,7 +740,7 @@ struct WideState {
   __nv_bfloat16* cache = nullptr;   // [U][rmax][E]
   float* a = nullptr;               // [rmax][E]
   float* rbuf = nullptr;            // [rmax][E]: output of the unit just computed
-  float* head_wt = nullptr;         // [A][E]
+  __nv_bfloat16* head_wt = nullptr; // [2][A][E] bf16: W_head transposed, then W_in (the row walk's head and embedding)
   float* ln_gb = nullptr;           // [2][U][E]: LayerNorm gain and shift of every unit's branch
   // observation conditioning on the tensor cores: embedding, MLP (Mish), keys|values
   int D = 0, Dp = 0;                // observation dim, padded to a multiple of BK
@@ -904,12 +910,17 @@ int wide_create(WideState** out, const evo_config* c, const float* weights, cons
       return fail(EVO_ERR_CUDA);
   }
   {
-    std::vector<float> ht((size_t)w->A * E);
+    // bf16: the walk reads both matrices once per row and step end from L1
+    std::vector<uint16_t> ht((size_t)2 * w->A * E);
     const float* hw = weights + woff[W_HEAD_W];
+    const float* iw = weights + woff[W_IN_W];
     for (int e = 0; e < E; ++e)
-      for (int a = 0; a < w->A; ++a) ht[(size_t)a * E + e] = hw[(size_t)e * w->A + a];
-    if (cudaMalloc(&w->head_wt, ht.size() * 4) != cudaSuccess) return fail(EVO_ERR_OOM);
-    if (cudaMemcpy(w->head_wt, ht.data(), ht.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      for (int a = 0; a < w->A; ++a) {
+        ht[(size_t)a * E + e] = bf16_bits(hw[(size_t)e * w->A + a]);
+        ht[(size_t)(w->A + a) * E + e] = bf16_bits(iw[(size_t)a * E + e]);
+      }
+    if (cudaMalloc(&w->head_wt, ht.size() * 2) != cudaSuccess) return fail(EVO_ERR_OOM);
+    if (cudaMemcpy(w->head_wt, ht.data(), ht.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess)
       return fail(EVO_ERR_CUDA);
   }
   {
@@ -1161,7 +1172,7 @@ cudaError_t wide_launch(WideState* w, const WideCall& c, cudaStream_t st) {
   wp.lnf_b = w->wf32 + w->woff[W_LNF_B];
   wp.head_wt = w->head_wt;
   wp.head_b = w->wf32 + w->woff[W_HEAD_B];
-  wp.in_w = w->wf32 + w->woff[W_IN_W];
+  wp.in_w = w->head_wt + (size_t)w->A * E;
   wp.in_b = w->wf32 + w->woff[W_IN_B];
   wp.pos = w->wf32 + w->woff[W_POS];
   wp.trace = c.trace;
