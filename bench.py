@@ -21,6 +21,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -165,15 +166,23 @@ def measured_peaks() -> dict:
         return {}
 
 
+def _code_only(src: str) -> str:
+    """C/C++/CUDA source without its comments and blank lines."""
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    return "\n".join(line.rstrip() for line in src.splitlines() if line.strip())
+
+
 def kernel_source_hash() -> str:
-    """Hash of every CUDA/C++ source of the library: a recorded ncu figure is
-    used only while the kernels it was taken on are unchanged."""
+    """Hash of the code (comments left out) of every CUDA/C++ source of the
+    library: a recorded ncu figure is used only while the kernels it was taken
+    on are unchanged."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_20293_gb300", "csrc")
     for f in sorted(os.listdir(csrc)):
         if f.endswith((".cu", ".cuh", ".h", ".cpp")):
             h.update(f.encode())
-            h.update(open(os.path.join(csrc, f), "rb").read())
+            h.update(_code_only(open(os.path.join(csrc, f)).read()).encode())
     return h.hexdigest()[:16]
 
 

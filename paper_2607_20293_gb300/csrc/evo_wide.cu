@@ -421,8 +421,6 @@ __device__ __forceinline__ bool head_step(const Walk& p, int row, int sample, in
   return true;
 }
 
-// Walk the row from step t, unit b (v = the stream before unit b) to the
-// launch's next refreshed cell (t1, b1), or to the end of the call.
 // the first cell after (t, b) that the sample's lattice refreshes, as t * 64 + b
 // (t = T: none)
 __device__ __forceinline__ int next_refresh(const Walk& p, int sample, int t, int b) {
@@ -432,6 +430,9 @@ __device__ __forceinline__ int next_refresh(const Walk& p, int sample, int t, in
   return t < p.lat.T ? t * 64 + __ffsll((long long)ref) - 1 : p.lat.T * 64;
 }
 
+// Walk the row from step t, unit b (v = the stream before unit b) to the cell
+// (t1, b1) -- writing the stream and, for that cell's unit, the LayerNorm
+// output -- or, when t1 = T, to the end of the call (x final).
 template <int NV>
 __device__ __forceinline__ void walk_row(const Walk& p, int row, int lane, int t, int b, float4 (&v)[NV], int t1,
                                          int b1) {
