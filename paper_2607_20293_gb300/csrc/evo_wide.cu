@@ -19,7 +19,10 @@
 //                     refreshed cell: the skipped units' cache adds, at step ends
 //                     LN_f, eps = . W_head + b_head, the sampler step (DDPM /
 //                     DDIM) and the next step's input embedding, and finally the
-//                     LayerNorm of the next refreshed unit -> xln (bf16)
+//                     LayerNorm of the next refreshed unit -> xln (bf16).  With
+//                     lattices that differ by sample, only the rows that refreshed
+//                     the cell, each to its own lattice's next refreshed cell.
+//                     Caches, r and the stream move with the evict-first policy.
 // The GEMMs skip 128-row tiles none of whose lattices refresh the unit.  Rows
 // of one lattice are contiguous (samples are ordered by lattice), so with the
 // batch sizes this path serves a 128-row tile rarely mixes lattices.
