@@ -105,3 +105,25 @@ def test_positions_loader_rejects(B):
     with pytest.raises(B.EvoError):
         B.schedule_from_positions([(0, 10)], 6, 10)
     assert B.schedule_from_positions([], 6, 10).sum() == 0
+
+
+def test_argument_checks_before_any_device_work(B):
+    # rejected on the host, before the CUDA runtime is touched
+    lib = B.load()
+    assert lib.evo_test_gelu(None, None, -1, 0, None) == B.ERR_ARG
+    assert lib.evo_test_gelu(None, None, 4, 0, None) == B.ERR_ARG
+    assert lib.evo_test_gelu(None, None, 0, 2, None) == B.ERR_ARG
+    assert lib.evo_test_wait_timeout(None, 0, 100, None) == B.ERR_ARG
+
+
+def test_binding_rejects_non_contiguous_buffers(B):
+    a = np.zeros((4, 6), np.float32)
+    with pytest.raises(ValueError):
+        B._ptr(a[:, ::2])
+    assert B._ptr(a) == a.ctypes.data
+    assert B._ptr(None) is None
+    torch = pytest.importorskip("torch")
+    t = torch.zeros(4, 6)
+    with pytest.raises(ValueError):
+        B._ptr(t.t())
+    assert B._ptr(t) == t.data_ptr()
